@@ -1,0 +1,431 @@
+"""Benchmark of the reshuffle A = alpha * op(B) + beta * A on GB300.
+
+Default workload (the metric's configuration): 8192 x 8192 f64, B block-cyclic
+64x64 on a 4x4 grid -> A block-cyclic 128x128 on a 4x4 grid with a seeded
+rank permutation, op = T, alpha = 2, beta = 0.5, P = 16 virtual ranks,
+relabeling on.  One step = one costa_transform call (direct mode) through the
+C ABI; its plan (overlay, volume kernel, relabeling, tile lists) is built once
+before the timed region and reported separately, like a reused transformer.
+
+Prints one JSON line.  `value` = algorithmic bytes (read B + read A if
+beta != 0 + write A) of all ranks / max-over-ranks device time.  `e2e` = the
+same metric through the same call with the inputs in pinned host memory:
+every step copies B (and A when beta != 0) host->device, transforms, and
+copies A back.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2|c3|c4|c5|c1]
+                  [--mode direct|message] [--impl gb300|reference]
+
+Multi-GPU (torchrun): one independent replica per GPU (the reshuffle of one
+problem uses one GPU here), scaling "weak".
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from workloads import configs as C  # noqa: E402
+from workloads.materialize import DeviceMatrix, HostMatrix  # noqa: E402
+
+L2_BYTES = 129 * 1024 * 1024
+KERNEL_SOURCES = ["paper_2106_06601_gb300/csrc/remap_impl.cuh",
+                  "paper_2106_06601_gb300/csrc/remap_f64.cu",
+                  "paper_2106_06601_gb300/csrc/remap_f32.cu",
+                  "paper_2106_06601_gb300/csrc/remap_c64.cu",
+                  "paper_2106_06601_gb300/csrc/remap_c128.cu"]
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="c2", choices=list(C.CONFIGS))
+    ap.add_argument("--mode", default="direct", choices=["direct", "message"])
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    return ap.parse_args()
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch from the committed ncu summary of this workload,
+    if it was taken on the current kernel sources."""
+    path = os.path.join(ROOT, "profiles", f"remap_{workload}_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        if d.get("kernel_sources_sha256_16") == kernel_hash():
+            return d.get("dram_bytes_per_launch")
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.samples = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        if not self.proc:
+            return None
+        win = [s for t, s in self.samples if t0 <= t <= t1]
+        window = "timed"
+        if not win:
+            win = [s for _, s in self.samples]
+            window = "whole run"
+        if not win:
+            return None
+        sm = []
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        smax = None
+        for s in win:
+            try:
+                sm.append(float(s[1]))
+                smax = float(s[2])
+            except ValueError:
+                continue
+            for k, nm in enumerate(names):
+                if len(s) > 5 + k and s[5 + k].lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm), "window": window}
+
+
+def problems(workload):
+    p = C.CONFIGS[workload]()
+    return p if isinstance(p, list) else [p]
+
+
+def esize(dtype):
+    return {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[dtype]
+
+
+def algorithmic_bytes(probs) -> int:
+    return sum(p.algorithmic_bytes() for p in probs)
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import paper_2106_06601_gb300 as costa
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    probs = problems(args.workload)
+    mats = []
+    for p in probs:
+        Bd = DeviceMatrix(p.B, p.dtype, dev).fill(p.b_kind, p.seed, p.src_stream)
+        Ad = DeviceMatrix(p.A, p.dtype, dev).fill(p.a_kind, p.seed, p.tgt_stream)
+        LA = costa.costa_layout_from_spec(p.A, p.dtype, Ad.block_ptrs())
+        LB = costa.costa_layout_from_spec(p.B, p.dtype, Bd.block_ptrs())
+        mats.append((p, Bd, Ad, LA, LB))
+    stream = torch.cuda.Stream(dev)
+    sh = stream.cuda_stream
+    As = [m[3] for m in mats]
+    Bs = [m[4] for m in mats]
+    ops = [p.op for p in probs]
+    alphas = [p.alpha for p in probs]
+    betas = [p.beta for p in probs]
+    batched = len(probs) > 1
+
+    def step():
+        if batched:
+            costa.costa_transform_batched(As, Bs, ops, alphas, betas, relabel=True, stream=sh,
+                                          mode=args.mode)
+        else:
+            costa.costa_transform(As[0], Bs[0], ops[0], alphas[0], betas[0], relabel=True,
+                                  stream=sh, mode=args.mode)
+
+    # plan (overlay, volume kernel, relabeling, tiles): built once, timed apart
+    t0 = time.perf_counter()
+    stats = costa.costa_plan_stats_get(As, Bs, ops, relabel=True, stream=sh)
+    plan_s = time.perf_counter() - t0
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            step()
+    torch.cuda.synchronize(dev)
+    if args.mode == "message":
+        stats = costa.costa_plan_stats_get(As, Bs, ops, relabel=True, stream=sh)
+
+    nbytes = algorithmic_bytes(probs)
+    clocks = ClockSampler(local_rank)
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    n0 = costa.costa_kernel_launch_count()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        end.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    if world > 1:
+        torch.distributed.barrier()
+    launches = costa.costa_kernel_launch_count() - n0
+    total_ms = start.elapsed_time(end)
+    per = [a.elapsed_time(b) for a, b in ev]
+    clocks.stop()
+    clk = clocks.summary(t_wall0, t_wall1)
+
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = t.item()
+    ms_per_step = total_ms / args.steps
+    value = nbytes * world * args.steps / (total_ms * 1e-3) / 1e9
+
+    # ---- end to end: pinned host inputs, copies inside the timed region ----
+    e2e = None
+    if args.e2e_steps > 0:
+        hostB = [torch.empty(m[1].arena.shape, dtype=m[1].arena.dtype, pin_memory=True)
+                 for m in mats]
+        hostA = [torch.empty(m[2].arena.shape, dtype=m[2].arena.dtype, pin_memory=True)
+                 for m in mats]
+        for (p, Bd, Ad, _, _), hb, ha in zip(mats, hostB, hostA):
+            hb.copy_(Bd.arena)
+            ha.copy_(Ad.arena)
+        h2d = sum(hb.numel() * hb.element_size() for hb in hostB)
+        h2d += sum(ha.numel() * ha.element_size() for (p, *_), ha in zip(mats, hostA)
+                   if p.beta != 0)
+        d2h = sum(ha.numel() * ha.element_size() for ha in hostA)
+
+        def e2e_step():
+            with torch.cuda.stream(stream):
+                for (p, Bd, Ad, _, _), hb, ha in zip(mats, hostB, hostA):
+                    Bd.arena.copy_(hb, non_blocking=True)
+                    if p.beta != 0:
+                        Ad.arena.copy_(ha, non_blocking=True)
+                step()
+                for (p, Bd, Ad, _, _), ha in zip(mats, hostA):
+                    ha.copy_(Ad.arena, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            torch.distributed.barrier()
+        s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e2.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = s2.elapsed_time(e2)
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e2e_ms = t.item()
+        e2e = {"value": round(nbytes * world * args.e2e_steps / (e2e_ms * 1e-3) / 1e9, 3),
+               "unit": "GB/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "ms_per_step": round(e2e_ms / args.e2e_steps, 4), "steps": args.e2e_steps}
+
+    for m in mats:
+        m[3].destroy()
+        m[4].destroy()
+    peak, peak_kind = measured_peaks()
+    avg_launch_ms = statistics.mean(per)
+    achieved = nbytes / (avg_launch_ms * 1e-3) / 1e9
+    traffic = recorded_traffic(args.workload) if args.mode == "direct" else None
+    return dict(value=value, ms_per_step=ms_per_step, total_ms=total_ms, per=per,
+                launches=launches, clocks=clk, e2e=e2e, plan_s=plan_s, stats=stats,
+                nbytes=nbytes, achieved=achieved, peak=peak, peak_kind=peak_kind,
+                traffic=traffic, probs=probs)
+
+
+def run_cpu_oracle(args, probs, seconds_target: float):
+    """The oracle, as it stands, on a bounded row slab of the first instance
+    (the same layouts and values); returns (GB/s, threads, description)."""
+    import oracle
+    p = probs[0]
+    threads = oracle.default_threads()
+    Bh = HostMatrix(p.B, p.dtype).fill(p.b_kind, p.seed, p.src_stream)
+    Ah = HostMatrix(p.A, p.dtype).fill(p.a_kind, p.seed, p.tgt_stream)
+    per_row_bytes = p.A.n * p.esize * (3 if p.beta != 0 else 2)
+    # calibrate on a few rows, then size the slab for the target time
+    rows = max(1, min(p.A.m, 8))
+    t0 = time.perf_counter()
+    oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B, Bh.buffers(),
+                     rows=(0, rows), threads=threads)
+    dt = max(time.perf_counter() - t0, 1e-6)
+    rows2 = int(min(p.A.m, max(rows, rows * seconds_target / dt)))
+    t0 = time.perf_counter()
+    oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B, Bh.buffers(),
+                     rows=(0, rows2), threads=threads)
+    dt2 = time.perf_counter() - t0
+    gbs = rows2 * per_row_bytes / dt2 / 1e9
+    desc = (f"rows 0..{rows2} of A ({rows2 * p.A.n} of {p.A.m * p.A.n} elements"
+            f"{' of instance 0 of ' + str(len(probs)) if len(probs) > 1 else ''}), {dt2:.1f} s")
+    return gbs, threads, desc, rows2, dt2
+
+
+def workload_config(args, probs, world):
+    p = probs[0]
+    nbytes = algorithmic_bytes(probs)
+    return {"workload": f"{args.workload}: {C.WORKLOAD_TEXT[args.workload]}",
+            "dtype": p.dtype, "op": p.op, "alpha": str(p.alpha), "beta": str(p.beta),
+            "P": p.A.nranks, "instances": len(probs), "relabel": True, "mode": args.mode,
+            "bytes_per_step_per_gpu": nbytes,
+            "l2": f"no flush: inputs larger than L2 ({nbytes / 1e9:.2f} GB moved per step "
+                  f"vs {L2_BYTES / 1e6:.0f} MB L2)",
+            "parallelism": f"replicas x{world}"}
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    probs = problems(args.workload)
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        steps, warmup = max(1, args.steps), max(0, args.warmup)
+        # each step: the oracle on a bounded sample sized so the whole run
+        # stays within a few minutes
+        per_step = max(0.5, min(10.0, 150.0 / (steps + warmup)))
+        import oracle
+        threads = oracle.default_threads()
+        gbs, threads, desc, rows, dt = run_cpu_oracle(args, probs, per_step)
+        p = probs[0]
+        per_row_bytes = p.A.n * p.esize * (3 if p.beta != 0 else 2)
+        Bh = HostMatrix(p.B, p.dtype).fill(p.b_kind, p.seed, p.src_stream)
+        Ah = HostMatrix(p.A, p.dtype).fill(p.a_kind, p.seed, p.tgt_stream)
+        for _ in range(warmup):
+            oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
+                             Bh.buffers(), rows=(0, rows), threads=threads)
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
+                             Bh.buffers(), rows=(0, rows), threads=threads)
+        dt = time.perf_counter() - t0
+        value = rows * per_row_bytes * steps / dt / 1e9
+        print(json.dumps({
+            "impl": "reference", "metric": "reshuffle GB/s (A = alpha*op(B) + beta*A)",
+            "value": round(value, 4), "unit": "GB/s", "n_gpus": args.gpus, "steps": steps,
+            "warmup": warmup, "ms_per_step": round(dt / steps * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": p.dtype, "data": "synthetic (seeded counter-based generator)",
+            "config": workload_config(args, probs, 1),
+            "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads,
+                             "kind": "oracle", "sample": f"each step: {desc.split(',')[0]}"},
+            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}), flush=True)
+        return
+
+    import torch
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    r = run_gpu(args, rank, world, local_rank)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        gbs, threads, desc, _, _ = run_cpu_oracle(args, probs, args.cpu_seconds)
+        cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+               "sample": desc}
+    if rank == 0:
+        st = r["stats"]
+        out = {
+            "metric": "reshuffle GB/s (A = alpha*op(B) + beta*A), % of GB300 HBM peak",
+            "value": round(r["value"], 3), "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup),
+            "ms_per_step": round(r["ms_per_step"], 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": probs[0].dtype,
+            "data": "synthetic (seeded counter-based generator, values per the workload)",
+            "config": workload_config(args, probs, world),
+            "elements_per_s": round(sum(p.A.m * p.A.n for p in probs) * world / (r["ms_per_step"] * 1e-3), 1),
+            "pct_of_hbm_peak": {"measured": round(100 * r["value"] / world / r["peak"], 2),
+                                "nominal_8TBs": round(100 * r["value"] / world / 8000.0, 2)},
+            "roofline": {"bound": "hbm", "achieved": round(r["achieved"], 2),
+                         "peak": r["peak"], "unit": "GB/s",
+                         "frac": round(r["achieved"] / r["peak"], 4),
+                         "traffic": r["traffic"],
+                         "kernel": "remap_kernel (direct)" if args.mode == "direct" else
+                                   "pack + remap(local) + unpack",
+                         "peak_source": f"{r['peak_kind']} (MEASURED_PEAKS.json hbm_gbs)",
+                         "algorithmic_bytes_per_launch": r["nbytes"],
+                         "avg_launch_ms": round(statistics.mean(r["per"]), 5),
+                         "median_launch_ms": round(statistics.median(r["per"]), 5),
+                         "best_launch_ms": round(min(r["per"]), 5)},
+            "plan": {"ms": round(r["plan_s"] * 1e3, 2), "volume_ms": round(st["volume_ms"], 3),
+                     "relabel_ms": round(st["relabel_ms"], 3), "cells": st["n_cells"],
+                     "tiles": st["n_tiles"], "total_volume": st["total_volume"],
+                     "local_identity": st["local_identity"],
+                     "local_relabeled": st["local_relabeled"],
+                     "staging_bytes": st["staging_bytes"]},
+            "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,232 @@
+/*
+ * costa_gb300.h: C ABI of a single-GPU (sm_103a) implementation of COSTA's
+ * shuffle-and-transpose
+ *
+ *     A = alpha * op(B) + beta * A,   op in {N (identity), T (transpose),
+ *                                           C (conjugate transpose)}       (Eq. 1, Sec. 5)
+ *
+ * between two grid-like layouts, together with the communication volumes of
+ * the reshuffle (Alg. 2) and the communication-optimal process relabeling
+ * (COPR, Def. 3 / Thm. 1 / Alg. 1, Sec. 4).
+ *
+ * The P "processes" of the paper are virtual ranks: a rank is just an owner
+ * label, and the blocks it owns live wherever their pointers say (normally
+ * one device buffer per rank).  All entry points take plain host or device
+ * pointers and sizes; none takes a framework type.
+ *
+ * Conventions shared by every call:
+ *  - Status: each call returns COSTA_OK or an error code, and on error sets a
+ *    thread-local message readable with costa_last_error().  All validation
+ *    happens before any device work, so a call that fails validation writes
+ *    nothing.
+ *  - Streams: `stream` is a cudaStream_t passed as void* (NULL = legacy
+ *    default stream).  Transform calls are asynchronous on that stream and
+ *    return once the kernels are enqueued; the caller keeps every buffer
+ *    alive and unmodified until the stream reaches that point.
+ *  - Plans: the first transform of a (layouts, op, relabel) combination
+ *    builds a plan (grid overlay, volumes, relabeling, tile lists; see
+ *    costa_plan_stats) and caches it.  Building a plan synchronizes `stream`.
+ *    Plans are freed when one of their layouts is destroyed or by
+ *    costa_release_plans().
+ *  - Aliasing: A's and B's storage must not overlap; a layout's blocks must
+ *    not overlap each other.  Overlap is not detected and gives undefined
+ *    results.
+ */
+#ifndef COSTA_GB300_H
+#define COSTA_GB300_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    COSTA_OK = 0,
+    COSTA_ERR_INVALID_ARG = 1, /* null pointer, bad enum, count out of range */
+    COSTA_ERR_LAYOUT = 2,      /* inconsistent layout description            */
+    COSTA_ERR_SHAPE = 3,       /* dims(A) != dims(op(B)) or rank counts differ */
+    COSTA_ERR_DTYPE = 4,       /* element types of A and B (or of a batch) differ */
+    COSTA_ERR_ALLOC = 5,       /* host or device allocation failed           */
+    COSTA_ERR_CUDA = 6,        /* a CUDA call failed (message has the error) */
+    COSTA_ERR_INTERNAL = 7
+} costa_status;
+
+/* Element types: real and complex (interleaved re, im), single and double. */
+typedef enum { COSTA_F32 = 0, COSTA_F64 = 1, COSTA_C64 = 2, COSTA_C128 = 3 } costa_dtype;
+
+/* op(B): identity, transpose, conjugate transpose (on real types C == T). */
+typedef enum { COSTA_OP_N = 0, COSTA_OP_T = 1, COSTA_OP_C = 2 } costa_op;
+
+/* Element order inside one block (Sec. 6: "row- or col-major ordering"). */
+typedef enum { COSTA_COL_MAJOR = 0, COSTA_ROW_MAJOR = 1 } costa_order;
+
+/* How the data moves on the device:
+ *  DIRECT  - one fused kernel reads B's blocks and writes A's blocks
+ *            (every pair is treated like the paper's "local blocks", Sec. 6);
+ *  MESSAGE - the paper's data flow (Alg. 3, Sec. 6): packages for remote
+ *            (source, relabeled target) pairs are packed into one staging
+ *            buffer at the exclusive-scan offsets of V, then unpacked and
+ *            transformed into A; pairs that are local after relabeling are
+ *            remapped directly.  Results are bit-identical to DIRECT. */
+typedef enum { COSTA_MODE_DIRECT = 0, COSTA_MODE_MESSAGE = 1 } costa_mode;
+
+/* Storage of one block (Sec. 6, Fig. 1: pointer, stride, ordering).
+ *  ptr   - device address of the block's (0, 0) element; aligned to the
+ *          element size (16 bytes for COSTA_C128).
+ *  ld    - leading dimension in elements: the distance between consecutive
+ *          columns (column-major) or rows (row-major); ld >= rows
+ *          (column-major) or ld >= cols (row-major); ld < 2^31.
+ *  order - costa_order. */
+typedef struct {
+    void *ptr;
+    int64_t ld;
+    int32_t order;
+    int32_t reserved; /* must be 0 */
+} costa_block;
+
+typedef struct costa_layout_s *costa_layout;
+
+/* Statistics of a cached plan (volumes in elements). */
+typedef struct {
+    int64_t total_volume;     /* m * n: elements moved                            */
+    int64_t local_identity;   /* trace(V): volume local without relabeling         */
+    int64_t local_relabeled;  /* sum_q V[sigma(q)][q]: local volume under sigma     */
+    int64_t n_cells;          /* grid-overlay cells (Sec. 5, "Grid Overlay")        */
+    int64_t n_tiles;          /* kernel tiles (overlay cells cut to tile size)      */
+    int64_t staging_bytes;    /* MESSAGE mode staging size (remote volume x size)   */
+    double plan_ms;           /* host + device time to build the plan              */
+    double volume_ms;         /* of which: the volume kernel incl. its copy back   */
+    double relabel_ms;        /* of which: the assignment solve                    */
+} costa_plan_stats;
+
+/* Layout L(A) = (Grid, P, Owners) (Sec. 5, "Matrix Layout") with the block
+ * storage of Sec. 6 (Fig. 1).
+ *  dt          - element type of the matrix.
+ *  nranks      - P >= 1.
+ *  nbr, nbc    - block rows / columns (>= 0; 0 gives an empty matrix).
+ *  row_splits  - host, nbr + 1 non-decreasing values, row_splits[0] == 0;
+ *                block row i holds rows [row_splits[i], row_splits[i+1]);
+ *                the matrix has m = row_splits[nbr] rows.  Likewise col_splits.
+ *  owners      - host, nbr * nbc ranks in [0, nranks), block (i, j) at i*nbc + j.
+ *  blocks      - host, nbr * nbc storage descriptors (same indexing); entries
+ *                of empty blocks are ignored.
+ * The layout copies all host arrays; device pointers are borrowed.
+ * Errors: COSTA_ERR_INVALID_ARG (null pointer, counts), COSTA_ERR_LAYOUT
+ * (unsorted splits, owner out of range, ld too small or too large, misaligned
+ * or null block pointer, bad order). */
+costa_status costa_layout_create(costa_layout *out, costa_dtype dt, int nranks,
+                                 int nbr, const int64_t *row_splits,
+                                 int nbc, const int64_t *col_splits,
+                                 const int *owners, const costa_block *blocks);
+
+/* ScaLAPACK-style block-cyclic layout (zero source offsets) of an m x n matrix
+ * with mb x nb blocks on a pr x pc process grid.  Block (bi, bj) sits on grid
+ * process (bi mod pr, bj mod pc), whose grid rank is r = i*pc + j for
+ * grid_order 'R' or i + j*pr for 'C'; its owner is rank_perm[r] (identity if
+ * rank_perm is NULL).  Each owner o stores its local matrix (NUMROC rows x
+ * NUMROC cols) column-major at rank_ptrs[o] with leading dimension lld[o]
+ * (>= local rows), so block (bi, bj) starts at local row (bi div pr)*mb and
+ * local column (bj div pc)*nb.  rank_ptrs and lld are host arrays of pr*pc
+ * entries indexed by owner.  Errors as costa_layout_create. */
+costa_status costa_layout_create_block_cyclic(costa_layout *out, costa_dtype dt,
+                                              int64_t m, int64_t n, int64_t mb, int64_t nb,
+                                              int pr, int pc, char grid_order,
+                                              const int *rank_perm,
+                                              void *const *rank_ptrs, const int64_t *lld);
+
+/* Frees a layout and every cached plan that uses it.  Synchronizes the
+ * device if a plan held device memory.  NULL is accepted. */
+costa_status costa_layout_destroy(costa_layout layout);
+
+/* Shape queries. */
+costa_status costa_layout_info(costa_layout layout, int64_t *m, int64_t *n,
+                               int *nranks, int *dtype);
+
+/* Communication volumes of the reshuffle of B into A's layout (Alg. 2 with
+ * the volume V(s) of Sec. 2): V[p * P + q] = number of elements whose source
+ * block in L(B) is owned by p and whose target block in L(A) is owned by q.
+ * V is a host array of P * P int64.  Runs the overlay/volume kernel on
+ * `stream` and synchronizes it.  Errors: INVALID_ARG, SHAPE, CUDA. */
+costa_status costa_volume(costa_layout A, costa_layout B, costa_op op, int64_t *V,
+                          void *stream);
+
+/* Communication-optimal process relabeling for the locally-free volume cost
+ * (Eq. 2; Remark on the gain and Thm. 1 / Thm. 2, Sec. 4): sigma maximizes
+ * sum_q V[sigma[q] * P + q], i.e. target label q is taken by process
+ * sigma[q].  Exact (Hungarian algorithm, O(P^3), host).  Ties: when the
+ * identity attains the optimum the identity is returned.  V: host P * P
+ * int64, entries >= 0.  sigma: host, P ints.  local_volume (nullable):
+ * receives the optimal sum.  Errors: INVALID_ARG (P < 1, null, negative V). */
+costa_status costa_relabel(int P, const int64_t *V, int *sigma, int64_t *local_volume);
+
+/* A = alpha * op(B) + beta * A (Eq. 1, Alg. 3) in COSTA_MODE_DIRECT.
+ *  alpha, beta - host pointers to one scalar of the layouts' element type
+ *                (float, double, or {re, im} pairs for the complex types).
+ *                When beta == 0, A is not read (NaN in A does not propagate).
+ *  relabel     - nonzero: compute sigma (costa_relabel on the volumes);
+ *                sigma only re-tags target owners, so A's contents are the
+ *                same either way.
+ *  sigma_out   - nullable host array of P ints; receives sigma (identity when
+ *                relabel == 0).
+ * Errors: INVALID_ARG, SHAPE (dims(A) != dims(op(B)), P differs), DTYPE,
+ * ALLOC, CUDA. */
+costa_status costa_transform(costa_layout A, costa_layout B, costa_op op,
+                             const void *alpha, const void *beta, int relabel,
+                             int *sigma_out, void *stream);
+
+/* costa_transform with an explicit costa_mode. */
+costa_status costa_transform_ex(costa_layout A, costa_layout B, costa_op op,
+                                const void *alpha, const void *beta, int relabel,
+                                int *sigma_out, costa_mode mode, void *stream);
+
+/* Batched transformation (Sec. 6, "Batched Transformation"): n independent
+ * pairs A[k] = alphas[k] * op_k(B[k]) + betas[k] * A[k] in one launch.  All
+ * layouts share one element type and one rank count P.  alphas / betas are
+ * host arrays of n scalars of that type.  With relabel, one sigma is computed
+ * from V summed over the batch (the batch forms one communication round).
+ * sigma_out: nullable, P ints. */
+costa_status costa_transform_batched(int n, const costa_layout *A, const costa_layout *B,
+                                     const costa_op *ops, const void *alphas,
+                                     const void *betas, int relabel, int *sigma_out,
+                                     void *stream);
+
+/* costa_transform_batched with an explicit costa_mode. */
+costa_status costa_transform_batched_ex(int n, const costa_layout *A,
+                                        const costa_layout *B, const costa_op *ops,
+                                        const void *alphas, const void *betas,
+                                        int relabel, int *sigma_out, costa_mode mode,
+                                        void *stream);
+
+/* Statistics of the plan for (A, B, op, relabel), building it if needed
+ * (which synchronizes `stream`).  For a batch use n > 1 with arrays. */
+costa_status costa_plan_stats_get(int n, const costa_layout *A, const costa_layout *B,
+                                  const costa_op *ops, int relabel,
+                                  costa_plan_stats *stats, void *stream);
+
+/* Diagnostics (host only, no device work): the pieces into which the plan
+ * cuts one axis of A (axis 0 = rows, 1 = columns) for the pair (A, B, op).
+ * Each piece is 6 int32: {A block index, op(B) block index, offset in A's
+ * block, offset in op(B)'s block, length, overlay interval index}; the
+ * kernel's tiles are the products of row pieces and column pieces.  Writes
+ * min(*count, cap) pieces to out (6 * cap int32) and the total to *count. */
+costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op, int axis,
+                                     int32_t *out, int64_t cap, int64_t *count);
+
+/* Frees every cached plan (synchronizes the device). */
+costa_status costa_release_plans(void);
+
+/* Thread-local message of the last failed call on this thread ("" if none). */
+const char *costa_last_error(void);
+
+/* Number of kernels this library has launched in this process. */
+int64_t costa_kernel_launch_count(void);
+
+/* ABI version of this header (1). */
+int costa_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* COSTA_GB300_H */

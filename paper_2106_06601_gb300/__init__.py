@@ -1,0 +1,273 @@
+"""Python binding of the COSTA GB300 library (include/costa_gb300.h).
+
+Argument marshalling only: every step of the reshuffle (overlay, volume,
+relabeling, data movement) runs in the native library.  The functions have
+the C entry points' names.  Device buffers are passed as integer addresses
+(e.g. torch's ``data_ptr()``), streams as ``cudaStream_t`` integers (e.g.
+``torch.cuda.current_stream().cuda_stream``).
+
+The library must have been built (``paper_2106_06601_gb300.build.build()``);
+importing the binding without it raises ImportError: there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from .build import LIB as _LIB_PATH
+
+COSTA_OK = 0
+STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "LAYOUT", 3: "SHAPE", 4: "DTYPE", 5: "ALLOC",
+                6: "CUDA", 7: "INTERNAL"}
+DTYPES = {"f32": 0, "f64": 1, "c64": 2, "c128": 3}
+OPS = {"N": 0, "T": 1, "C": 2}
+MODES = {"direct": 0, "message": 1}
+ORDERS = {"C": 0, "R": 1}
+_SCALAR_NP = {"f32": np.float32, "f64": np.float64, "c64": np.complex64, "c128": np.complex128}
+
+
+class CostaError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class _Block(ctypes.Structure):
+    _fields_ = [("ptr", ctypes.c_void_p), ("ld", ctypes.c_int64), ("order", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
+
+
+class PlanStats(ctypes.Structure):
+    _fields_ = [("total_volume", ctypes.c_int64), ("local_identity", ctypes.c_int64),
+                ("local_relabeled", ctypes.c_int64), ("n_cells", ctypes.c_int64),
+                ("n_tiles", ctypes.c_int64), ("staging_bytes", ctypes.c_int64),
+                ("plan_ms", ctypes.c_double), ("volume_ms", ctypes.c_double),
+                ("relabel_ms", ctypes.c_double)]
+
+    def as_dict(self):
+        return {k: getattr(self, k) for k, _ in self._fields_}
+
+
+def _load():
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(f"COSTA CUDA library not built ({_LIB_PATH}); "
+                          "run paper_2106_06601_gb300.build.build()")
+    lib = ctypes.CDLL(_LIB_PATH)
+    P, I, I64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64
+    sigs = {
+        "costa_layout_create": [P, I, I, I, P, I, P, P, P],
+        "costa_layout_create_block_cyclic": [P, I, I64, I64, I64, I64, I, I, ctypes.c_char, P, P, P],
+        "costa_layout_destroy": [P],
+        "costa_layout_info": [P, P, P, P, P],
+        "costa_volume": [P, P, I, P, P],
+        "costa_relabel": [I, P, P, P],
+        "costa_transform": [P, P, I, P, P, I, P, P],
+        "costa_transform_ex": [P, P, I, P, P, I, P, I, P],
+        "costa_transform_batched": [I, P, P, P, P, P, I, P, P],
+        "costa_transform_batched_ex": [I, P, P, P, P, P, I, P, I, P],
+        "costa_plan_stats_get": [I, P, P, P, I, P, P],
+        "costa_release_plans": [],
+        "costa_debug_axis_pieces": [P, P, I, I, P, I64, P],
+    }
+    for name, args in sigs.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = ctypes.c_int
+    lib.costa_last_error.argtypes = []
+    lib.costa_last_error.restype = ctypes.c_char_p
+    lib.costa_kernel_launch_count.argtypes = []
+    lib.costa_kernel_launch_count.restype = ctypes.c_int64
+    lib.costa_abi_version.argtypes = []
+    lib.costa_abi_version.restype = ctypes.c_int
+    return lib
+
+
+_lib = _load()
+
+
+def library():
+    """The loaded ctypes library (for symbol checks)."""
+    return _lib
+
+
+def _check(status: int) -> None:
+    if status != COSTA_OK:
+        raise CostaError(status, _lib.costa_last_error().decode())
+
+
+def _i64(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.int64)
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def _p(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+class Layout:
+    """Owning handle of a costa_layout."""
+
+    def __init__(self, handle: int, dtype: str):
+        self.handle = ctypes.c_void_p(handle)
+        self.dtype = dtype
+
+    def info(self):
+        m, n = ctypes.c_int64(), ctypes.c_int64()
+        P, dt = ctypes.c_int(), ctypes.c_int()
+        _check(_lib.costa_layout_info(self.handle, ctypes.byref(m), ctypes.byref(n),
+                                      ctypes.byref(P), ctypes.byref(dt)))
+        return m.value, n.value, P.value, dt.value
+
+    def destroy(self):
+        if self.handle:
+            _check(_lib.costa_layout_destroy(self.handle))
+            self.handle = ctypes.c_void_p(0)
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def costa_layout_create(dtype: str, nranks: int, row_splits, col_splits, owners, block_ptrs,
+                        block_ld, block_order) -> Layout:
+    """Layout from splits, an owners grid and per-block storage (device
+    address, leading dimension, order 0 = column-major / 1 = row-major)."""
+    R, C = _i64(row_splits), _i64(col_splits)
+    nbr, nbc = len(R) - 1, len(C) - 1
+    own = _i32(owners).reshape(-1)
+    ptrs = np.ascontiguousarray(block_ptrs, dtype=np.uint64).reshape(-1)
+    ld = _i64(block_ld).reshape(-1)
+    order = _i32(block_order).reshape(-1)
+    nblk = nbr * nbc
+    assert own.size == nblk and ptrs.size == nblk and ld.size == nblk and order.size == nblk
+    blocks = (_Block * max(1, nblk))()
+    for k in range(nblk):
+        blocks[k].ptr = int(ptrs[k])
+        blocks[k].ld = int(ld[k])
+        blocks[k].order = int(order[k])
+        blocks[k].reserved = 0
+    out = ctypes.c_void_p()
+    _check(_lib.costa_layout_create(ctypes.byref(out), DTYPES[dtype], nranks, nbr, _p(R), nbc,
+                                    _p(C), _p(own), blocks))
+    return Layout(out.value, dtype)
+
+
+def costa_layout_create_block_cyclic(dtype: str, m: int, n: int, mb: int, nb: int, pr: int,
+                                     pc: int, grid_order: str, rank_perm, rank_ptrs,
+                                     lld) -> Layout:
+    P = pr * pc
+    perm = None if rank_perm is None else _i32(rank_perm)
+    ptrs = (ctypes.c_void_p * P)(*[int(x) for x in rank_ptrs])
+    lld = _i64(lld)
+    out = ctypes.c_void_p()
+    _check(_lib.costa_layout_create_block_cyclic(
+        ctypes.byref(out), DTYPES[dtype], m, n, mb, nb, pr, pc, grid_order.encode(),
+        None if perm is None else _p(perm), ptrs, _p(lld)))
+    return Layout(out.value, dtype)
+
+
+def costa_layout_destroy(layout: Layout) -> None:
+    layout.destroy()
+
+
+def costa_volume(A: Layout, B: Layout, op: str, stream: int = 0) -> np.ndarray:
+    """V[p, q]: elements sent from rank p (owner in L(B)) to rank q (owner in L(A))."""
+    _, _, P, _ = A.info()
+    V = np.zeros((P, P), dtype=np.int64)
+    _check(_lib.costa_volume(A.handle, B.handle, OPS[op], _p(V), ctypes.c_void_p(stream)))
+    return V
+
+
+def costa_relabel(V):
+    """(sigma, local_volume): sigma[q] is the process that takes target label q."""
+    V = _i64(V)
+    P = V.shape[0]
+    sigma = np.zeros(P, dtype=np.int32)
+    lv = ctypes.c_int64()
+    _check(_lib.costa_relabel(P, _p(V), _p(sigma), ctypes.byref(lv)))
+    return sigma, lv.value
+
+
+def _scalars(dtype: str, values) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(values, dtype=_SCALAR_NP[dtype]).reshape(-1))
+
+
+def costa_transform(A: Layout, B: Layout, op: str, alpha, beta, relabel: bool = False,
+                    stream: int = 0, mode: str = "direct") -> np.ndarray:
+    """A = alpha * op(B) + beta * A, asynchronous on `stream`; returns sigma."""
+    _, _, P, _ = A.info()
+    sigma = np.zeros(P, dtype=np.int32)
+    al, be = _scalars(A.dtype, [alpha]), _scalars(A.dtype, [beta])
+    _check(_lib.costa_transform_ex(A.handle, B.handle, OPS[op], _p(al), _p(be), int(relabel),
+                                   _p(sigma), MODES[mode], ctypes.c_void_p(stream)))
+    return sigma
+
+
+def costa_transform_batched(As, Bs, ops, alphas, betas, relabel: bool = False,
+                            stream: int = 0, mode: str = "direct") -> np.ndarray:
+    n = len(As)
+    _, _, P, _ = As[0].info()
+    sigma = np.zeros(P, dtype=np.int32)
+    ha = (ctypes.c_void_p * n)(*[a.handle.value for a in As])
+    hb = (ctypes.c_void_p * n)(*[b.handle.value for b in Bs])
+    op = _i32([OPS[o] for o in ops])
+    al, be = _scalars(As[0].dtype, alphas), _scalars(As[0].dtype, betas)
+    assert al.size == n and be.size == n
+    _check(_lib.costa_transform_batched_ex(n, ha, hb, _p(op), _p(al), _p(be), int(relabel),
+                                           _p(sigma), MODES[mode], ctypes.c_void_p(stream)))
+    return sigma
+
+
+def costa_plan_stats_get(As, Bs, ops, relabel: bool = False, stream: int = 0) -> dict:
+    if isinstance(As, Layout):
+        As, Bs, ops = [As], [Bs], [ops]
+    n = len(As)
+    ha = (ctypes.c_void_p * n)(*[a.handle.value for a in As])
+    hb = (ctypes.c_void_p * n)(*[b.handle.value for b in Bs])
+    op = _i32([OPS[o] for o in ops])
+    st = PlanStats()
+    _check(_lib.costa_plan_stats_get(n, ha, hb, _p(op), int(relabel), ctypes.byref(st),
+                                     ctypes.c_void_p(stream)))
+    return st.as_dict()
+
+
+def costa_release_plans() -> None:
+    _check(_lib.costa_release_plans())
+
+
+def costa_last_error() -> str:
+    return _lib.costa_last_error().decode()
+
+
+def costa_kernel_launch_count() -> int:
+    return _lib.costa_kernel_launch_count()
+
+
+def costa_abi_version() -> int:
+    return _lib.costa_abi_version()
+
+
+def costa_layout_from_spec(spec, dtype: str, block_ptrs) -> Layout:
+    """costa_layout_create from any object with the fields rsplit, csplit,
+    owner, nranks, ld, order (one entry per block) and per-block device
+    addresses `block_ptrs`."""
+    return costa_layout_create(dtype, spec.nranks, spec.rsplit, spec.csplit, spec.owner,
+                               block_ptrs, spec.ld, spec.order)
+
+
+def costa_debug_axis_pieces(A: Layout, B: Layout, op: str, axis: int) -> np.ndarray:
+    """The plan's pieces of one axis of A, as an int32 array [count, 6]."""
+    cnt = ctypes.c_int64()
+    _check(_lib.costa_debug_axis_pieces(A.handle, B.handle, OPS[op], axis, None, 0,
+                                        ctypes.byref(cnt)))
+    out = np.zeros((max(1, cnt.value), 6), dtype=np.int32)
+    _check(_lib.costa_debug_axis_pieces(A.handle, B.handle, OPS[op], axis, _p(out), cnt.value,
+                                        ctypes.byref(cnt)))
+    return out[:cnt.value]

@@ -1,0 +1,854 @@
+// Host side of the library: layout descriptors (Sec. 5 "Matrix Layout",
+// Sec. 6 Fig. 1), the grid overlay and tile lists (Sec. 5 "Grid Overlay",
+// Alg. 2), the volume / relabeling plan (Alg. 1, Thm. 1), the message-mode
+// package offsets (Sec. 6), and the C entry points declared in
+// include/costa_gb300.h.
+#include <algorithm>
+#include <atomic>
+#include <chrono>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime_api.h>
+
+#include "costa_internal.h"
+
+struct costa_layout_s {
+    uint64_t id;
+    costa_dtype dt;
+    int nranks;
+    int nbr, nbc;
+    int64_t m, n;
+    std::vector<int64_t> R, C;
+    std::vector<int32_t> owner;
+    std::vector<costa::DevBlock> blocks;
+};
+
+namespace costa {
+
+int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
+                   std::vector<int64_t> *u_out, std::vector<int64_t> *v_out);
+
+namespace {
+
+thread_local std::string g_err;
+std::atomic<uint64_t> g_next_id{1};
+
+costa_status fail(costa_status s, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return s;
+}
+
+costa_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(COSTA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int esize_of(int dt) {
+    switch (dt) {
+    case COSTA_F32: return 4;
+    case COSTA_F64: return 8;
+    case COSTA_C64: return 8;
+    case COSTA_C128: return 16;
+    default: return 0;
+    }
+}
+
+double ms_since(std::chrono::steady_clock::time_point t0) {
+    return std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
+}
+
+// ---------------------------------------------------------------------------
+// Grid overlay along one axis (Sec. 5): the sorted union of A's splits and
+// op(B)'s splits cuts the axis into intervals, each inside exactly one block
+// of A and one block of op(B) (the unique cover).  Empty blocks are skipped.
+// ---------------------------------------------------------------------------
+struct AxisCut {
+    std::vector<Interval> intervals;
+    std::vector<AxisTile> tiles;
+};
+
+// Cuts one axis.  The pieces of an interval are aligned to `align_a` (true:
+// multiples of ts from the start of A's block, else of op(B)'s block), so
+// that the side whose contiguous axis this is gets 16-byte aligned runs.
+AxisCut cut_axis(const std::vector<int64_t> &SA, const std::vector<int64_t> &SB, int64_t extent,
+                 int ts, bool align_a) {
+    AxisCut out;
+    const int nA = static_cast<int>(SA.size()) - 1, nB = static_cast<int>(SB.size()) - 1;
+    int ka = 0, kb = 0;
+    int64_t pos = 0;
+    while (pos < extent) {
+        while (ka + 1 < nA && SA[ka + 1] <= pos) ++ka;
+        while (kb + 1 < nB && SB[kb + 1] <= pos) ++kb;
+        const int64_t end = std::min(SA[ka + 1], SB[kb + 1]);
+        const int64_t len = end - pos;
+        const int cell = static_cast<int>(out.intervals.size());
+        out.intervals.push_back(Interval{ka, kb, len});
+        const int64_t a0 = pos - SA[ka], b0 = pos - SB[kb];
+        int64_t q = 0;
+        while (q < len) {
+            const int64_t phase = (align_a ? a0 + q : b0 + q) % ts;
+            const int64_t piece = std::min<int64_t>(ts - phase, len - q);
+            out.tiles.push_back(AxisTile{ka, kb, static_cast<int32_t>(a0 + q),
+                                         static_cast<int32_t>(b0 + q),
+                                         static_cast<int32_t>(piece), cell});
+            q += piece;
+        }
+        pos = end;
+    }
+    return out;
+}
+
+// Cuts axis 0 (rows) or 1 (columns) of A for the pair (A, op(B)).  Each axis
+// is aligned to the side whose contiguous axis it is (decided by the first
+// block's order: column-major makes rows contiguous), so that side's runs
+// start on 16-byte boundaries.
+AxisCut cut_pair_axis(const costa_layout_s *A, const costa_layout_s *B, int op, int axis, int ts) {
+    const bool tr = op != COSTA_OP_N;
+    const bool a_rows_fast = A->blocks.empty() || A->blocks[0].order == COSTA_COL_MAJOR;
+    const bool b_col = B->blocks.empty() || B->blocks[0].order == COSTA_COL_MAJOR;
+    const bool b_rows_fast = tr ? !b_col : b_col;  // op(B)'s contiguous axis is rows
+    if (axis == 0) return cut_axis(A->R, tr ? B->C : B->R, A->m, ts, a_rows_fast || !b_rows_fast);
+    return cut_axis(A->C, tr ? B->R : B->C, A->n, ts, !a_rows_fast || b_rows_fast);
+}
+
+struct ProblemHost {
+    const costa_layout_s *A;
+    const costa_layout_s *B;
+    costa_op op;
+    AxisCut rows, cols;
+};
+
+// One device allocation holding all tables of a plan, built on the host
+// with 256-byte aligned sections and copied once.
+struct Arena {
+    std::vector<char> host;
+    size_t add(const void *p, size_t bytes) {
+        const size_t off = (host.size() + 255) & ~size_t(255);
+        host.resize(off + std::max<size_t>(bytes, 1));
+        if (bytes) std::memcpy(host.data() + off, p, bytes);
+        return off;
+    }
+    template <typename V> size_t add_vec(const std::vector<V> &v) {
+        return add(v.data(), v.size() * sizeof(V));
+    }
+};
+
+struct MessageData {
+    bool built = false;
+    void *d_mem = nullptr;       // stage_off, stage_ld, ProblemDev[]
+    ProblemDev *d_probs = nullptr;
+    void *d_staging = nullptr;
+    int64_t staging_bytes = 0;
+    int64_t remote_tiles = 0;
+};
+
+struct Plan {
+    int device = 0;
+    int dtype = 0, esize = 0, P = 0, ts = 32;
+    std::vector<ProblemHost> probs;
+    void *d_mem = nullptr;
+    ProblemDev *d_probs = nullptr;
+    std::vector<ProblemDev> h_probs;
+    Scalars *d_scalars = nullptr;
+    std::vector<Scalars> cached_scalars;
+    int64_t total_tiles = 0, total_cells = 0;
+    std::vector<int64_t> V;      // P * P, V[p * P + q]
+    bool sigma_done = false;
+    std::vector<int> sigma;      // optimal relabeling
+    costa_plan_stats stats{};
+    MessageData msg[2];          // [relabel]
+
+    ~Plan() {
+        for (auto &m : msg) {
+            if (m.d_mem) cudaFree(m.d_mem);
+            if (m.d_staging) cudaFree(m.d_staging);
+        }
+        if (d_mem) cudaFree(d_mem);
+    }
+};
+
+std::mutex g_mu;
+std::map<std::vector<uint64_t>, std::unique_ptr<Plan>> g_plans;
+
+bool plan_uses(const std::vector<uint64_t> &key, uint64_t id) {
+    // key = [device, n, (A.id, B.id, op) x n]
+    for (size_t i = 2; i + 1 < key.size(); i += 3)
+        if (key[i] == id || key[i + 1] == id) return true;
+    return false;
+}
+
+// ---- relabeling: sigma maximizing sum_q V[sigma(q)][q] ----
+void solve_relabel(int P, const int64_t *V, std::vector<int> &sigma, int64_t &best) {
+    // rows = target labels q, columns = processes p, cost = -V[p][q]
+    std::vector<int64_t> cost(static_cast<size_t>(P) * P);
+    for (int q = 0; q < P; ++q)
+        for (int p = 0; p < P; ++p) cost[static_cast<size_t>(q) * P + p] = -V[static_cast<size_t>(p) * P + q];
+    std::vector<int> row_to_col;
+    best = -assign_min(P, cost, row_to_col, nullptr, nullptr);
+    int64_t trace = 0;
+    for (int q = 0; q < P; ++q) trace += V[static_cast<size_t>(q) * P + q];
+    sigma.resize(P);
+    if (trace == best) {  // tie rule: keep the identity when it is optimal
+        for (int q = 0; q < P; ++q) sigma[q] = q;
+    } else {
+        for (int q = 0; q < P; ++q) sigma[q] = row_to_col[q];
+    }
+}
+
+costa_status validate_pair(const costa_layout_s *A, const costa_layout_s *B, int op) {
+    if (!A || !B) return fail(COSTA_ERR_INVALID_ARG, "null layout");
+    if (op < COSTA_OP_N || op > COSTA_OP_C) return fail(COSTA_ERR_INVALID_ARG, "bad op %d", op);
+    if (A->dt != B->dt)
+        return fail(COSTA_ERR_DTYPE, "element types differ (A %d, B %d)", A->dt, B->dt);
+    if (A->nranks != B->nranks)
+        return fail(COSTA_ERR_SHAPE, "rank counts differ (A %d, B %d)", A->nranks, B->nranks);
+    const int64_t bm = op == COSTA_OP_N ? B->m : B->n, bn = op == COSTA_OP_N ? B->n : B->m;
+    if (A->m != bm || A->n != bn)
+        return fail(COSTA_ERR_SHAPE, "A is %lld x %lld but op(B) is %lld x %lld", (long long)A->m,
+                    (long long)A->n, (long long)bm, (long long)bn);
+    return COSTA_OK;
+}
+
+// Builds the overlay, tiles and device tables, and runs the volume kernel.
+costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, const costa_op *ops,
+                        cudaStream_t stream, std::unique_ptr<Plan> &out) {
+    auto t0 = std::chrono::steady_clock::now();
+    auto plan = std::make_unique<Plan>();
+    cudaError_t ce = cudaGetDevice(&plan->device);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaGetDevice");
+    plan->dtype = As[0]->dt;
+    plan->esize = esize_of(plan->dtype);
+    plan->P = As[0]->nranks;
+    plan->ts = tile_extent(plan->esize);
+    const int P = plan->P, ts = plan->ts;
+
+    Arena arena;
+    struct Off { size_t rows, cols, descA, descB, irows, icols, ownA, ownB; };
+    std::vector<Off> offs(n);
+    for (int k = 0; k < n; ++k) {
+        ProblemHost ph;
+        ph.A = As[k];
+        ph.B = Bs[k];
+        ph.op = ops[k];
+        ph.rows = cut_pair_axis(ph.A, ph.B, ph.op, 0, ts);
+        ph.cols = cut_pair_axis(ph.A, ph.B, ph.op, 1, ts);
+        Off &o = offs[k];
+        o.rows = arena.add_vec(ph.rows.tiles);
+        o.cols = arena.add_vec(ph.cols.tiles);
+        o.descA = arena.add_vec(ph.A->blocks);
+        o.descB = arena.add_vec(ph.B->blocks);
+        o.irows = arena.add_vec(ph.rows.intervals);
+        o.icols = arena.add_vec(ph.cols.intervals);
+        o.ownA = arena.add_vec(ph.A->owner);
+        o.ownB = arena.add_vec(ph.B->owner);
+        plan->probs.push_back(std::move(ph));
+    }
+    std::vector<ProblemDev> pd(n);
+    std::vector<VolumeProblemDev> vd(n);
+    const size_t off_pd = arena.add(pd.data(), sizeof(ProblemDev) * n);
+    const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
+    std::vector<Scalars> sc(n);
+    const size_t off_sc = arena.add(sc.data(), sizeof(Scalars) * n);
+    std::vector<unsigned long long> vz(static_cast<size_t>(P) * P, 0ull);
+    const size_t off_V = arena.add_vec(vz);
+
+    void *d = nullptr;
+    ce = cudaMalloc(&d, arena.host.size());
+    if (ce != cudaSuccess) return fail(COSTA_ERR_ALLOC, "cudaMalloc(%zu): %s", arena.host.size(),
+                                       cudaGetErrorString(ce));
+    plan->d_mem = d;
+    char *dbase = static_cast<char *>(d);
+    int64_t tiles = 0, cells = 0;
+    for (int k = 0; k < n; ++k) {
+        const ProblemHost &ph = plan->probs[k];
+        const Off &o = offs[k];
+        ProblemDev &p = pd[k];
+        p.rows = reinterpret_cast<const AxisTile *>(dbase + o.rows);
+        p.cols = reinterpret_cast<const AxisTile *>(dbase + o.cols);
+        p.descA = reinterpret_cast<const DevBlock *>(dbase + o.descA);
+        p.descB = reinterpret_cast<const DevBlock *>(dbase + o.descB);
+        p.stage_off = nullptr;
+        p.stage_ld = nullptr;
+        p.tile_begin = tiles;
+        p.nu = static_cast<int32_t>(ph.rows.tiles.size());
+        p.nv = static_cast<int32_t>(ph.cols.tiles.size());
+        p.nbcA = ph.A->nbc;
+        p.nbcB = ph.B->nbc;
+        p.op = ph.op;
+        p.pad = 0;
+        tiles += static_cast<int64_t>(p.nu) * p.nv;
+        VolumeProblemDev &v = vd[k];
+        v.rows = reinterpret_cast<const Interval *>(dbase + o.irows);
+        v.cols = reinterpret_cast<const Interval *>(dbase + o.icols);
+        v.ownerA = reinterpret_cast<const int32_t *>(dbase + o.ownA);
+        v.ownerB = reinterpret_cast<const int32_t *>(dbase + o.ownB);
+        v.cell_begin = cells;
+        v.nr = static_cast<int32_t>(ph.rows.intervals.size());
+        v.nc = static_cast<int32_t>(ph.cols.intervals.size());
+        v.nbcA = ph.A->nbc;
+        v.nbcB = ph.B->nbc;
+        v.op = ph.op;
+        v.pad = 0;
+        cells += static_cast<int64_t>(v.nr) * v.nc;
+    }
+    std::memcpy(arena.host.data() + off_pd, pd.data(), sizeof(ProblemDev) * n);
+    std::memcpy(arena.host.data() + off_vd, vd.data(), sizeof(VolumeProblemDev) * n);
+    ce = cudaMemcpy(d, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(plan tables)");
+    plan->d_probs = reinterpret_cast<ProblemDev *>(dbase + off_pd);
+    plan->d_scalars = reinterpret_cast<Scalars *>(dbase + off_sc);
+    plan->h_probs = pd;
+    plan->total_tiles = tiles;
+    plan->total_cells = cells;
+
+    // volume kernel: V[p][q] over the overlay cells
+    auto tv = std::chrono::steady_clock::now();
+    VolumeLaunch vl;
+    vl.probs = reinterpret_cast<const VolumeProblemDev *>(dbase + off_vd);
+    vl.nprob = n;
+    vl.P = P;
+    vl.total_cells = cells;
+    vl.V = reinterpret_cast<unsigned long long *>(dbase + off_V);
+    ce = launch_volume(vl, stream);
+    if (ce != cudaSuccess) return cuda_fail(ce, "volume kernel launch");
+    plan->V.assign(static_cast<size_t>(P) * P, 0);
+    ce = cudaMemcpyAsync(plan->V.data(), vl.V, sizeof(int64_t) * P * P, cudaMemcpyDeviceToHost, stream);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpyAsync(V)");
+    ce = cudaStreamSynchronize(stream);
+    if (ce != cudaSuccess) return cuda_fail(ce, "volume kernel");
+    plan->stats.volume_ms = ms_since(tv);
+
+    int64_t total = 0, trace = 0;
+    for (int p = 0; p < P; ++p)
+        for (int q = 0; q < P; ++q) total += plan->V[static_cast<size_t>(p) * P + q];
+    for (int q = 0; q < P; ++q) trace += plan->V[static_cast<size_t>(q) * P + q];
+    int64_t want = 0;
+    for (int k = 0; k < n; ++k) want += As[k]->m * As[k]->n;
+    if (total != want)
+        return fail(COSTA_ERR_INTERNAL, "volume check failed: sum V = %lld, expected %lld",
+                    (long long)total, (long long)want);
+    plan->stats.total_volume = total;
+    plan->stats.local_identity = trace;
+    plan->stats.local_relabeled = trace;
+    plan->stats.n_cells = cells;
+    plan->stats.n_tiles = tiles;
+    plan->stats.plan_ms = ms_since(t0);
+    out = std::move(plan);
+    return COSTA_OK;
+}
+
+costa_status ensure_sigma(Plan &plan) {
+    if (plan.sigma_done) return COSTA_OK;
+    auto t0 = std::chrono::steady_clock::now();
+    int64_t best = 0;
+    solve_relabel(plan.P, plan.V.data(), plan.sigma, best);
+    plan.stats.relabel_ms = ms_since(t0);
+    plan.stats.local_relabeled = best;
+    plan.sigma_done = true;
+    return COSTA_OK;
+}
+
+// Message mode (Alg. 3, Sec. 6): every tile whose source process p differs
+// from the process sigma(q) that takes its target label q is "remote" and
+// travels through the staging buffer.  Packages are ordered by (p, receiver)
+// at the exclusive-scan offsets of their sizes; inside a package the tiles
+// keep the tile order.  Each staged tile is dense in the source's element
+// order with its leading dimension rounded up to 16 bytes.
+costa_status ensure_message(Plan &plan, bool relabel) {
+    MessageData &m = plan.msg[relabel ? 1 : 0];
+    if (m.built) return COSTA_OK;
+    const int P = plan.P;
+    std::vector<int> sig(P);
+    if (relabel) {
+        costa_status s = ensure_sigma(plan);
+        if (s != COSTA_OK) return s;
+        sig = plan.sigma;
+    } else {
+        for (int q = 0; q < P; ++q) sig[q] = q;
+    }
+    const int vec = 16 / plan.esize;
+    const int64_t T = plan.total_tiles;
+    std::vector<int64_t> stage_off(static_cast<size_t>(std::max<int64_t>(T, 1)), -1);
+    std::vector<int32_t> stage_ld(static_cast<size_t>(std::max<int64_t>(T, 1)), 0);
+    std::vector<int32_t> pkg(static_cast<size_t>(std::max<int64_t>(T, 1)), -1);
+    std::vector<int64_t> size(static_cast<size_t>(P) * P, 0);
+    int64_t t = 0, remote = 0;
+    for (const ProblemHost &ph : plan.probs) {
+        const bool tr = ph.op != COSTA_OP_N;
+        for (const AxisTile &rt : ph.rows.tiles) {
+            for (const AxisTile &ct : ph.cols.tiles) {
+                const int q = ph.A->owner[static_cast<size_t>(rt.a_blk) * ph.A->nbc + ct.a_blk];
+                const size_t bidx = tr ? static_cast<size_t>(ct.b_blk) * ph.B->nbc + rt.b_blk
+                                       : static_cast<size_t>(rt.b_blk) * ph.B->nbc + ct.b_blk;
+                const int p = ph.B->owner[bidx];
+                const int r = sig[q];
+                if (p != r) {
+                    const bool b_col = ph.B->blocks[bidx].order == COSTA_COL_MAJOR;
+                    const bool src_fast_i = tr ? !b_col : b_col;
+                    const int fast = src_fast_i ? rt.len : ct.len;
+                    const int other = src_fast_i ? ct.len : rt.len;
+                    const int ld = (fast + vec - 1) / vec * vec;
+                    stage_ld[t] = ld;
+                    pkg[t] = p * P + r;
+                    stage_off[t] = static_cast<int64_t>(ld) * other;  // size for now
+                    size[static_cast<size_t>(p) * P + r] += stage_off[t];
+                    ++remote;
+                }
+                ++t;
+            }
+        }
+    }
+    std::vector<int64_t> base(static_cast<size_t>(P) * P, 0);
+    int64_t acc = 0;
+    for (size_t k = 0; k < base.size(); ++k) {
+        base[k] = acc;
+        acc += size[k];
+    }
+    for (int64_t i = 0; i < T; ++i) {
+        if (pkg[i] < 0) continue;
+        const int64_t sz = stage_off[i];
+        stage_off[i] = base[pkg[i]];
+        base[pkg[i]] += sz;
+    }
+    const int n = static_cast<int>(plan.probs.size());
+    Arena arena;
+    const size_t o_off = arena.add_vec(stage_off);
+    const size_t o_ld = arena.add_vec(stage_ld);
+    std::vector<ProblemDev> pd = plan.h_probs;
+    const size_t o_pd = arena.add(pd.data(), sizeof(ProblemDev) * n);
+    cudaError_t ce = cudaMalloc(&m.d_mem, arena.host.size());
+    if (ce != cudaSuccess) return fail(COSTA_ERR_ALLOC, "cudaMalloc(message tables): %s", cudaGetErrorString(ce));
+    char *db = static_cast<char *>(m.d_mem);
+    for (int k = 0; k < n; ++k) {
+        pd[k].stage_off = reinterpret_cast<const int64_t *>(db + o_off) + pd[k].tile_begin;
+        pd[k].stage_ld = reinterpret_cast<const int32_t *>(db + o_ld) + pd[k].tile_begin;
+    }
+    std::memcpy(arena.host.data() + o_pd, pd.data(), sizeof(ProblemDev) * n);
+    ce = cudaMemcpy(m.d_mem, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(message tables)");
+    m.d_probs = reinterpret_cast<ProblemDev *>(db + o_pd);
+    m.staging_bytes = acc * plan.esize;
+    if (m.staging_bytes > 0) {
+        ce = cudaMalloc(&m.d_staging, static_cast<size_t>(m.staging_bytes));
+        if (ce != cudaSuccess)
+            return fail(COSTA_ERR_ALLOC, "cudaMalloc(staging %lld B): %s", (long long)m.staging_bytes,
+                        cudaGetErrorString(ce));
+    }
+    m.remote_tiles = remote;
+    m.built = true;
+    plan.stats.staging_bytes = m.staging_bytes;
+    return COSTA_OK;
+}
+
+costa_status get_plan(int n, const costa_layout *A, const costa_layout *B, const costa_op *ops,
+                      cudaStream_t stream, Plan *&out) {
+    int dev = 0;
+    cudaError_t ce = cudaGetDevice(&dev);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaGetDevice");
+    std::vector<uint64_t> key;
+    key.reserve(2 + 3 * static_cast<size_t>(n));
+    key.push_back(static_cast<uint64_t>(dev));
+    key.push_back(static_cast<uint64_t>(n));
+    for (int k = 0; k < n; ++k) {
+        key.push_back(A[k]->id);
+        key.push_back(B[k]->id);
+        key.push_back(static_cast<uint64_t>(ops[k]));
+    }
+    auto it = g_plans.find(key);
+    if (it != g_plans.end()) {
+        out = it->second.get();
+        return COSTA_OK;
+    }
+    std::unique_ptr<Plan> plan;
+    costa_status s = build_plan(n, A, B, ops, stream, plan);
+    if (s != COSTA_OK) return s;
+    out = plan.get();
+    g_plans.emplace(std::move(key), std::move(plan));
+    return COSTA_OK;
+}
+
+// Reads one scalar of element type dt at p[index].
+void read_scalar(int dt, const void *p, int index, double out[2]) {
+    switch (dt) {
+    case COSTA_F32: out[0] = static_cast<const float *>(p)[index]; out[1] = 0.0; break;
+    case COSTA_F64: out[0] = static_cast<const double *>(p)[index]; out[1] = 0.0; break;
+    case COSTA_C64:
+        out[0] = static_cast<const float *>(p)[2 * index];
+        out[1] = static_cast<const float *>(p)[2 * index + 1];
+        break;
+    default:
+        out[0] = static_cast<const double *>(p)[2 * index];
+        out[1] = static_cast<const double *>(p)[2 * index + 1];
+        break;
+    }
+}
+
+Scalars make_scalars(int dt, const void *alpha, const void *beta, int index) {
+    Scalars s{};
+    read_scalar(dt, alpha, index, s.alpha);
+    read_scalar(dt, beta, index, s.beta);
+    s.flags = 0;
+    if (s.beta[0] == 0.0 && s.beta[1] == 0.0) s.flags |= SF_BETA0;
+    if (s.alpha[0] == 1.0 && s.alpha[1] == 0.0) s.flags |= SF_ALPHA1;
+    if (s.alpha[1] != 0.0 || s.beta[1] != 0.0) s.flags |= SF_CPLX;
+    return s;
+}
+
+bool same_scalars(const Scalars &a, const Scalars &b) { return std::memcmp(&a, &b, sizeof(Scalars)) == 0; }
+
+costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B, const costa_op *ops,
+                            const void *alphas, const void *betas, int relabel, int *sigma_out,
+                            int mode, void *stream_v) {
+    if (n < 1) return fail(COSTA_ERR_INVALID_ARG, "batch size %d < 1", n);
+    if (!A || !B || !ops || !alphas || !betas) return fail(COSTA_ERR_INVALID_ARG, "null argument");
+    if (mode != COSTA_MODE_DIRECT && mode != COSTA_MODE_MESSAGE)
+        return fail(COSTA_ERR_INVALID_ARG, "bad mode %d", mode);
+    for (int k = 0; k < n; ++k) {
+        costa_status s = validate_pair(A[k], B[k], ops[k]);
+        if (s != COSTA_OK) return s;
+        if (A[k]->dt != A[0]->dt) return fail(COSTA_ERR_DTYPE, "batch mixes element types");
+        if (A[k]->nranks != A[0]->nranks) return fail(COSTA_ERR_SHAPE, "batch mixes rank counts");
+    }
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+    std::lock_guard<std::mutex> lock(g_mu);
+    Plan *plan = nullptr;
+    costa_status s = get_plan(n, A, B, ops, stream, plan);
+    if (s != COSTA_OK) return s;
+    const int P = plan->P;
+    if (relabel) {
+        s = ensure_sigma(*plan);
+        if (s != COSTA_OK) return s;
+    }
+    if (sigma_out)
+        for (int q = 0; q < P; ++q) sigma_out[q] = relabel ? plan->sigma[q] : q;
+    if (plan->total_tiles == 0) return COSTA_OK;
+
+    RemapLaunch L{};
+    L.probs = plan->d_probs;
+    L.nprob = n;
+    L.dtype = plan->dtype;
+    L.total_tiles = plan->total_tiles;
+    L.s = make_scalars(plan->dtype, alphas, betas, 0);
+    L.per_problem = nullptr;
+    bool uniform = true;
+    std::vector<Scalars> sc(n);
+    for (int k = 0; k < n; ++k) {
+        sc[k] = make_scalars(plan->dtype, alphas, betas, k);
+        if (!same_scalars(sc[k], sc[0])) uniform = false;
+    }
+    if (!uniform) {
+        bool same = plan->cached_scalars.size() == sc.size();
+        for (int k = 0; same && k < n; ++k) same = same_scalars(sc[k], plan->cached_scalars[k]);
+        if (!same) {
+            // pageable source: the copy is staged before the call returns, and
+            // stream order places it after earlier kernels of this stream
+            cudaError_t ce = cudaMemcpyAsync(plan->d_scalars, sc.data(), sizeof(Scalars) * n,
+                                             cudaMemcpyHostToDevice, stream);
+            if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpyAsync(scalars)");
+            plan->cached_scalars = sc;
+        }
+        L.per_problem = plan->d_scalars;
+    }
+    // one launch per combine kind present in the batch
+    bool kinds[4] = {false, false, false, false};
+    for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
+    auto launch_all = [&](int km) -> cudaError_t {
+        for (int kind = 0; kind < 4; ++kind) {
+            if (!kinds[kind]) continue;
+            cudaError_t e = launch_remap(L, km, kind, stream);
+            if (e != cudaSuccess) return e;
+        }
+        return cudaSuccess;
+    };
+    cudaError_t ce;
+    if (mode == COSTA_MODE_DIRECT) {
+        ce = launch_all(KM_DIRECT_ALL);
+        if (ce != cudaSuccess) return cuda_fail(ce, "remap kernel launch");
+        return COSTA_OK;
+    }
+    s = ensure_message(*plan, relabel != 0);
+    if (s != COSTA_OK) return s;
+    MessageData &m = plan->msg[relabel ? 1 : 0];
+    L.probs = m.d_probs;
+    L.staging = m.d_staging;
+    ce = launch_remap(L, KM_PACK, K_COPY, stream);
+    if (ce != cudaSuccess) return cuda_fail(ce, "pack kernel launch");
+    ce = launch_all(KM_DIRECT_LOCAL);
+    if (ce != cudaSuccess) return cuda_fail(ce, "local remap kernel launch");
+    ce = launch_all(KM_UNPACK);
+    if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
+    return COSTA_OK;
+}
+
+costa_status create_layout(costa_layout *out, int dt, int nranks, int nbr, const int64_t *R, int nbc,
+                           const int64_t *C, const int *owners, const costa_block *blocks) {
+    if (!out) return fail(COSTA_ERR_INVALID_ARG, "out is null");
+    *out = nullptr;
+    const int es = esize_of(dt);
+    if (!es) return fail(COSTA_ERR_DTYPE, "unknown dtype %d", dt);
+    if (nranks < 1) return fail(COSTA_ERR_INVALID_ARG, "nranks %d < 1", nranks);
+    if (nbr < 0 || nbc < 0) return fail(COSTA_ERR_INVALID_ARG, "negative block counts");
+    if (!R || !C) return fail(COSTA_ERR_INVALID_ARG, "null splits");
+    const int64_t nblk = static_cast<int64_t>(nbr) * nbc;
+    if (nblk > 0 && (!owners || !blocks)) return fail(COSTA_ERR_INVALID_ARG, "null owners or blocks");
+    if (R[0] != 0 || C[0] != 0) return fail(COSTA_ERR_LAYOUT, "splits must start at 0");
+    for (int i = 0; i < nbr; ++i)
+        if (R[i + 1] < R[i]) return fail(COSTA_ERR_LAYOUT, "row splits not sorted at %d", i);
+    for (int j = 0; j < nbc; ++j)
+        if (C[j + 1] < C[j]) return fail(COSTA_ERR_LAYOUT, "column splits not sorted at %d", j);
+    for (int i = 0; i < nbr; ++i)
+        if (R[i + 1] - R[i] >= (int64_t(1) << 31)) return fail(COSTA_ERR_LAYOUT, "block row %d too tall", i);
+    for (int j = 0; j < nbc; ++j)
+        if (C[j + 1] - C[j] >= (int64_t(1) << 31)) return fail(COSTA_ERR_LAYOUT, "block column %d too wide", j);
+    auto L = std::make_unique<costa_layout_s>();
+    L->id = g_next_id.fetch_add(1);
+    L->dt = static_cast<costa_dtype>(dt);
+    L->nranks = nranks;
+    L->nbr = nbr;
+    L->nbc = nbc;
+    L->m = R[nbr];
+    L->n = C[nbc];
+    L->R.assign(R, R + nbr + 1);
+    L->C.assign(C, C + nbc + 1);
+    L->owner.resize(static_cast<size_t>(nblk));
+    L->blocks.resize(static_cast<size_t>(nblk));
+    for (int i = 0; i < nbr; ++i) {
+        const int64_t h = R[i + 1] - R[i];
+        for (int j = 0; j < nbc; ++j) {
+            const int64_t w = C[j + 1] - C[j];
+            const int64_t b = static_cast<int64_t>(i) * nbc + j;
+            if (owners[b] < 0 || owners[b] >= nranks)
+                return fail(COSTA_ERR_LAYOUT, "owner %d of block (%d, %d) not in [0, %d)", owners[b], i, j,
+                            nranks);
+            L->owner[b] = owners[b];
+            const costa_block &blk = blocks[b];
+            DevBlock d{reinterpret_cast<uint64_t>(blk.ptr), 0, blk.order};
+            if (h > 0 && w > 0) {
+                if (blk.order != COSTA_COL_MAJOR && blk.order != COSTA_ROW_MAJOR)
+                    return fail(COSTA_ERR_LAYOUT, "block (%d, %d): bad order %d", i, j, blk.order);
+                if (blk.reserved != 0) return fail(COSTA_ERR_LAYOUT, "block (%d, %d): reserved != 0", i, j);
+                if (!blk.ptr) return fail(COSTA_ERR_LAYOUT, "block (%d, %d): null pointer", i, j);
+                if (reinterpret_cast<uintptr_t>(blk.ptr) % es)
+                    return fail(COSTA_ERR_LAYOUT, "block (%d, %d): pointer not aligned to %d bytes", i, j, es);
+                const int64_t need = blk.order == COSTA_COL_MAJOR ? h : w;
+                if (blk.ld < need)
+                    return fail(COSTA_ERR_LAYOUT, "block (%d, %d): ld %lld < %lld", i, j, (long long)blk.ld,
+                                (long long)need);
+                if (blk.ld >= (int64_t(1) << 31))
+                    return fail(COSTA_ERR_LAYOUT, "block (%d, %d): ld %lld >= 2^31", i, j, (long long)blk.ld);
+                d.ld = static_cast<int32_t>(blk.ld);
+            } else {
+                d.ld = 1;
+                d.order = COSTA_COL_MAJOR;
+            }
+            L->blocks[b] = d;
+        }
+    }
+    *out = L.release();
+    return COSTA_OK;
+}
+
+int64_t numroc(int64_t n, int64_t nb, int iproc, int nprocs) {
+    const int64_t nblocks = n / nb;
+    int64_t r = (nblocks / nprocs) * nb;
+    const int64_t extra = nblocks % nprocs;
+    if (iproc < extra) r += nb;
+    else if (iproc == extra) r += n % nb;
+    return r;
+}
+
+}  // namespace
+}  // namespace costa
+
+using namespace costa;
+
+extern "C" {
+
+costa_status costa_layout_create(costa_layout *out, costa_dtype dt, int nranks, int nbr,
+                                 const int64_t *row_splits, int nbc, const int64_t *col_splits,
+                                 const int *owners, const costa_block *blocks) {
+    return create_layout(out, dt, nranks, nbr, row_splits, nbc, col_splits, owners, blocks);
+}
+
+costa_status costa_layout_create_block_cyclic(costa_layout *out, costa_dtype dt, int64_t m, int64_t n,
+                                              int64_t mb, int64_t nb, int pr, int pc, char grid_order,
+                                              const int *rank_perm, void *const *rank_ptrs,
+                                              const int64_t *lld) {
+    if (!out) return fail(COSTA_ERR_INVALID_ARG, "out is null");
+    *out = nullptr;
+    if (m < 0 || n < 0 || mb < 1 || nb < 1 || pr < 1 || pc < 1)
+        return fail(COSTA_ERR_INVALID_ARG, "bad block-cyclic sizes");
+    if (grid_order != 'R' && grid_order != 'C') return fail(COSTA_ERR_INVALID_ARG, "grid_order must be 'R' or 'C'");
+    if (!rank_ptrs || !lld) return fail(COSTA_ERR_INVALID_ARG, "null rank pointers or lld");
+    const int P = pr * pc;
+    const int es = esize_of(dt);
+    if (!es) return fail(COSTA_ERR_DTYPE, "unknown dtype %d", dt);
+    std::vector<int> perm(P);
+    std::vector<char> seen(P, 0);
+    for (int r = 0; r < P; ++r) {
+        perm[r] = rank_perm ? rank_perm[r] : r;
+        if (perm[r] < 0 || perm[r] >= P || seen[perm[r]])
+            return fail(COSTA_ERR_LAYOUT, "rank_perm is not a permutation of [0, %d)", P);
+        seen[perm[r]] = 1;
+    }
+    const int64_t nbr64 = (m + mb - 1) / mb, nbc64 = (n + nb - 1) / nb;
+    if (nbr64 > (1 << 30) || nbc64 > (1 << 30)) return fail(COSTA_ERR_INVALID_ARG, "too many blocks");
+    const int nbr = static_cast<int>(nbr64), nbc = static_cast<int>(nbc64);
+    std::vector<int64_t> R(nbr + 1), C(nbc + 1);
+    for (int i = 0; i <= nbr; ++i) R[i] = std::min<int64_t>(i * mb, m);
+    for (int j = 0; j <= nbc; ++j) C[j] = std::min<int64_t>(j * nb, n);
+    std::vector<int> owners(static_cast<size_t>(nbr) * nbc);
+    std::vector<costa_block> blocks(static_cast<size_t>(nbr) * nbc);
+    for (int bi = 0; bi < nbr; ++bi) {
+        const int i = bi % pr;
+        for (int bj = 0; bj < nbc; ++bj) {
+            const int j = bj % pc;
+            const int grank = grid_order == 'R' ? i * pc + j : i + j * pr;
+            const int o = perm[grank];
+            const size_t b = static_cast<size_t>(bi) * nbc + bj;
+            owners[b] = o;
+            const int64_t lr = static_cast<int64_t>(bi / pr) * mb, lc = static_cast<int64_t>(bj / pc) * nb;
+            const int64_t need = numroc(m, mb, i, pr);
+            if (lld[o] < std::max<int64_t>(1, need))
+                return fail(COSTA_ERR_LAYOUT, "lld[%d] = %lld < local rows %lld", o, (long long)lld[o],
+                            (long long)need);
+            blocks[b].ptr = static_cast<char *>(rank_ptrs[o]) + (lr + lc * lld[o]) * es;
+            blocks[b].ld = lld[o];
+            blocks[b].order = COSTA_COL_MAJOR;
+            blocks[b].reserved = 0;
+        }
+    }
+    return create_layout(out, dt, P, nbr, R.data(), nbc, C.data(), owners.data(), blocks.data());
+}
+
+costa_status costa_layout_destroy(costa_layout layout) {
+    if (!layout) return COSTA_OK;
+    {
+        std::lock_guard<std::mutex> lock(g_mu);
+        for (auto it = g_plans.begin(); it != g_plans.end();) {
+            if (plan_uses(it->first, layout->id)) it = g_plans.erase(it);
+            else ++it;
+        }
+    }
+    delete layout;
+    return COSTA_OK;
+}
+
+costa_status costa_layout_info(costa_layout layout, int64_t *m, int64_t *n, int *nranks, int *dtype) {
+    if (!layout) return fail(COSTA_ERR_INVALID_ARG, "null layout");
+    if (m) *m = layout->m;
+    if (n) *n = layout->n;
+    if (nranks) *nranks = layout->nranks;
+    if (dtype) *dtype = layout->dt;
+    return COSTA_OK;
+}
+
+costa_status costa_volume(costa_layout A, costa_layout B, costa_op op, int64_t *V, void *stream) {
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    if (!V) return fail(COSTA_ERR_INVALID_ARG, "V is null");
+    std::lock_guard<std::mutex> lock(g_mu);
+    Plan *plan = nullptr;
+    s = get_plan(1, &A, &B, &op, static_cast<cudaStream_t>(stream), plan);
+    if (s != COSTA_OK) return s;
+    std::memcpy(V, plan->V.data(), sizeof(int64_t) * plan->V.size());
+    return COSTA_OK;
+}
+
+costa_status costa_relabel(int P, const int64_t *V, int *sigma, int64_t *local_volume) {
+    if (P < 1) return fail(COSTA_ERR_INVALID_ARG, "P %d < 1", P);
+    if (!V || !sigma) return fail(COSTA_ERR_INVALID_ARG, "null argument");
+    for (int64_t k = 0; k < static_cast<int64_t>(P) * P; ++k)
+        if (V[k] < 0) return fail(COSTA_ERR_INVALID_ARG, "negative volume at %lld", (long long)k);
+    std::vector<int> sig;
+    int64_t best = 0;
+    solve_relabel(P, V, sig, best);
+    std::copy(sig.begin(), sig.end(), sigma);
+    if (local_volume) *local_volume = best;
+    return COSTA_OK;
+}
+
+costa_status costa_transform(costa_layout A, costa_layout B, costa_op op, const void *alpha, const void *beta,
+                             int relabel, int *sigma_out, void *stream) {
+    return transform_impl(1, &A, &B, &op, alpha, beta, relabel, sigma_out, COSTA_MODE_DIRECT, stream);
+}
+
+costa_status costa_transform_ex(costa_layout A, costa_layout B, costa_op op, const void *alpha,
+                                const void *beta, int relabel, int *sigma_out, costa_mode mode,
+                                void *stream) {
+    return transform_impl(1, &A, &B, &op, alpha, beta, relabel, sigma_out, mode, stream);
+}
+
+costa_status costa_transform_batched(int n, const costa_layout *A, const costa_layout *B, const costa_op *ops,
+                                     const void *alphas, const void *betas, int relabel, int *sigma_out,
+                                     void *stream) {
+    return transform_impl(n, A, B, ops, alphas, betas, relabel, sigma_out, COSTA_MODE_DIRECT, stream);
+}
+
+costa_status costa_transform_batched_ex(int n, const costa_layout *A, const costa_layout *B,
+                                        const costa_op *ops, const void *alphas, const void *betas,
+                                        int relabel, int *sigma_out, costa_mode mode, void *stream) {
+    return transform_impl(n, A, B, ops, alphas, betas, relabel, sigma_out, mode, stream);
+}
+
+costa_status costa_plan_stats_get(int n, const costa_layout *A, const costa_layout *B, const costa_op *ops,
+                                  int relabel, costa_plan_stats *stats, void *stream) {
+    if (n < 1 || !A || !B || !ops || !stats) return fail(COSTA_ERR_INVALID_ARG, "bad arguments");
+    for (int k = 0; k < n; ++k) {
+        costa_status s = validate_pair(A[k], B[k], ops[k]);
+        if (s != COSTA_OK) return s;
+    }
+    std::lock_guard<std::mutex> lock(g_mu);
+    Plan *plan = nullptr;
+    costa_status s = get_plan(n, A, B, ops, static_cast<cudaStream_t>(stream), plan);
+    if (s != COSTA_OK) return s;
+    if (relabel) {
+        s = ensure_sigma(*plan);
+        if (s != COSTA_OK) return s;
+    }
+    *stats = plan->stats;
+    if (!relabel) stats->local_relabeled = stats->local_identity;
+    stats->staging_bytes = plan->msg[relabel ? 1 : 0].built ? plan->msg[relabel ? 1 : 0].staging_bytes : -1;
+    return COSTA_OK;
+}
+
+costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op, int axis, int32_t *out,
+                                     int64_t cap, int64_t *count) {
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    if ((axis != 0 && axis != 1) || !count || (cap > 0 && !out))
+        return fail(COSTA_ERR_INVALID_ARG, "bad arguments");
+    const AxisCut cut = cut_pair_axis(A, B, op, axis, tile_extent(esize_of(A->dt)));
+    *count = static_cast<int64_t>(cut.tiles.size());
+    for (int64_t k = 0; k < std::min<int64_t>(cap, *count); ++k) {
+        const AxisTile &t = cut.tiles[static_cast<size_t>(k)];
+        const int32_t v[6] = {t.a_blk, t.b_blk, t.a_off, t.b_off, t.len, t.cell};
+        std::memcpy(out + 6 * k, v, sizeof v);
+    }
+    return COSTA_OK;
+}
+
+costa_status costa_release_plans(void) {
+    std::lock_guard<std::mutex> lock(g_mu);
+    g_plans.clear();
+    return COSTA_OK;
+}
+
+const char *costa_last_error(void) { return g_err.c_str(); }
+
+int64_t costa_kernel_launch_count(void) { return launches_so_far(); }
+
+int costa_abi_version(void) { return 1; }
+
+}  // extern "C"

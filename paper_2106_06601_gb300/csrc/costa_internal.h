@@ -1,0 +1,135 @@
+// Internal types shared by the host planner (costa.cpp) and the kernels
+// (remap_*.cu, volume.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __CUDACC__
+#define COSTA_HD __host__ __device__
+#else
+#define COSTA_HD
+#endif
+
+#include "costa_gb300.h"
+
+namespace costa {
+
+// Storage of one block as the kernels see it (Sec. 6, Fig. 1).
+struct DevBlock {
+    uint64_t ptr;   // device address of element (0, 0)
+    int32_t ld;     // leading dimension (elements)
+    int32_t order;  // 0 column-major, 1 row-major
+};
+static_assert(sizeof(DevBlock) == 16, "DevBlock layout");
+
+// One piece of a grid-overlay interval along one axis (rows or columns of A),
+// at most the kernel tile extent long.  The overlay (Sec. 5, "Grid Overlay")
+// is the product of the row intervals and the column intervals, so the
+// kernel's tile grid is the product of the row pieces and the column pieces.
+struct AxisTile {
+    int32_t a_blk;  // block index of A along this axis
+    int32_t b_blk;  // block index of op(B) along this axis (a B row block for
+                    // A's rows when op = N, a B column block when op = T/C)
+    int32_t a_off;  // offset of the piece inside A's block
+    int32_t b_off;  // offset of the piece inside op(B)'s block
+    int32_t len;    // extent of the piece
+    int32_t cell;   // index of the overlay interval it belongs to
+};
+static_assert(sizeof(AxisTile) == 24, "AxisTile layout");
+
+// One grid-overlay interval along one axis (used by the volume kernel).
+struct Interval {
+    int32_t a_blk;
+    int32_t b_blk;
+    int64_t len;
+};
+
+// One (A, B, op) pair as the kernels see it.
+struct ProblemDev {
+    const AxisTile *rows;
+    const AxisTile *cols;
+    const DevBlock *descA;      // nbrA * nbcA
+    const DevBlock *descB;      // nbrB * nbcB
+    const int64_t *stage_off;   // per tile (MESSAGE mode): element offset in staging, -1 = local
+    const int32_t *stage_ld;    // per tile (MESSAGE mode): leading dimension of the staged tile
+    int64_t tile_begin;         // first tile id of this problem in the launch
+    int32_t nu, nv;             // row pieces, column pieces
+    int32_t nbcA, nbcB;         // block columns of A and of B (descriptor indexing)
+    int32_t op;                 // costa_op
+    int32_t pad;
+};
+
+// Scalars of one problem, as doubles ({re, im}); float data carries values
+// that are exactly representable in float.
+struct Scalars {
+    double alpha[2];
+    double beta[2];
+    int32_t flags;
+    int32_t pad;
+};
+enum : int32_t { SF_BETA0 = 1, SF_ALPHA1 = 2, SF_CPLX = 4 };
+
+// Combine kinds: each kernel is compiled for one, so every path keeps only
+// the registers it needs.
+//   K_COPY  alpha = 1, beta = 0        out = op(b)
+//   K_SCALE real alpha, beta = 0       out = alpha * op(b)
+//   K_AXPBY real alpha, beta != 0      out = fma(alpha, op(b), beta * a)
+//   K_CPLX  complex alpha or beta      complex products as chains of fma
+enum : int { K_COPY = 0, K_SCALE = 1, K_AXPBY = 2, K_CPLX = 3 };
+
+COSTA_HD inline int kind_of(int32_t flags) {
+    if (flags & SF_CPLX) return K_CPLX;
+    if (!(flags & SF_BETA0)) return K_AXPBY;
+    if (!(flags & SF_ALPHA1)) return K_SCALE;
+    return K_COPY;
+}
+
+enum KernelMode : int { KM_DIRECT_ALL = 0, KM_DIRECT_LOCAL = 1, KM_PACK = 2, KM_UNPACK = 3 };
+
+struct RemapLaunch {
+    const ProblemDev *probs;
+    int32_t nprob;
+    int32_t dtype;
+    int64_t total_tiles;
+    const Scalars *per_problem;  // device array of nprob, or nullptr: use `s`
+    Scalars s;
+    void *staging;
+};
+
+struct VolumeProblemDev {
+    const Interval *rows;
+    const Interval *cols;
+    const int32_t *ownerA;      // nbrA * nbcA
+    const int32_t *ownerB;      // nbrB * nbcB
+    int64_t cell_begin;
+    int32_t nr, nc;
+    int32_t nbcA, nbcB;
+    int32_t op;
+    int32_t pad;
+};
+
+struct VolumeLaunch {
+    const VolumeProblemDev *probs;
+    int32_t nprob;
+    int32_t P;
+    int64_t total_cells;
+    unsigned long long *V;      // P * P, zeroed by the caller
+};
+
+// Tile extent (elements along each axis of A) for an element size.
+inline int tile_extent(int esize) { return esize == 16 ? 16 : 32; }
+
+// Launches the remap kernel for (args.dtype, mode, kind).  With
+// args.per_problem set, the kernel skips the tiles of problems of another kind.
+cudaError_t launch_remap(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
+cudaError_t launch_remap_f32(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
+cudaError_t launch_remap_f64(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
+cudaError_t launch_remap_c64(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
+cudaError_t launch_remap_c128(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
+cudaError_t launch_volume(const VolumeLaunch &args, cudaStream_t stream);
+void count_launch();
+int64_t launches_so_far();
+
+}  // namespace costa

@@ -1,0 +1,79 @@
+// Exact linear assignment for the process relabeling (Thm. 1 / Thm. 2,
+// Sec. 4): the Hungarian method (Kuhn 1955; Munkres 1957) in its O(n^3)
+// shortest-augmenting-path form.
+//
+// Rows are inserted one at a time.  Each insertion grows a Dijkstra-like
+// search over columns under the reduced costs c[i][j] - u[i] - v[j] >= 0,
+// updating the potentials (u, v) so that the edges of the matching stay
+// tight, until it reaches a free column; the matching is then flipped along
+// the alternating path.  After n insertions the matching is a minimum-cost
+// perfect assignment and (u, v) is a feasible dual solution whose objective
+// equals its cost (LP duality, the certificate of optimality).
+#include <cstdint>
+#include <limits>
+#include <vector>
+
+namespace costa {
+
+// cost: row-major n x n.  row_to_col[i] receives the column assigned to row i.
+// Returns the minimum total cost.  u (n rows) and v (n columns) receive the
+// dual potentials when non-null: u[i] + v[j] <= cost[i][j] for all (i, j),
+// with equality on the assignment.
+int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
+                   std::vector<int64_t> *u_out, std::vector<int64_t> *v_out) {
+    const int64_t INF = std::numeric_limits<int64_t>::max() / 4;
+    // 1-based internally; column 0 is a virtual source column.
+    std::vector<int64_t> u(n + 1, 0), v(n + 1, 0), dist(n + 1);
+    std::vector<int> col_row(n + 1, 0), prev(n + 1, 0);
+    std::vector<char> done(n + 1);
+    for (int i = 1; i <= n; ++i) {
+        col_row[0] = i;
+        int j0 = 0;
+        std::fill(dist.begin(), dist.end(), INF);
+        std::fill(done.begin(), done.end(), 0);
+        do {
+            done[j0] = 1;
+            const int i0 = col_row[j0];
+            int64_t delta = INF;
+            int j1 = 0;
+            const int64_t *crow = cost.data() + static_cast<size_t>(i0 - 1) * n;
+            for (int j = 1; j <= n; ++j) {
+                if (done[j]) continue;
+                const int64_t red = crow[j - 1] - u[i0] - v[j];
+                if (red < dist[j]) {
+                    dist[j] = red;
+                    prev[j] = j0;
+                }
+                if (dist[j] < delta) {
+                    delta = dist[j];
+                    j1 = j;
+                }
+            }
+            for (int j = 0; j <= n; ++j) {
+                if (done[j]) {
+                    u[col_row[j]] += delta;
+                    v[j] -= delta;
+                } else {
+                    dist[j] -= delta;
+                }
+            }
+            j0 = j1;
+        } while (col_row[j0] != 0);
+        do {  // flip the alternating path back to the source column
+            const int j1 = prev[j0];
+            col_row[j0] = col_row[j1];
+            j0 = j1;
+        } while (j0 != 0);
+    }
+    row_to_col.assign(n, -1);
+    int64_t total = 0;
+    for (int j = 1; j <= n; ++j) {
+        row_to_col[col_row[j] - 1] = j - 1;
+        total += cost[static_cast<size_t>(col_row[j] - 1) * n + (j - 1)];
+    }
+    if (u_out) u_out->assign(u.begin() + 1, u.end());
+    if (v_out) v_out->assign(v.begin() + 1, v.end());
+    return total;
+}
+
+}  // namespace costa

@@ -1,0 +1,186 @@
+"""Host-side checks of the C ABI (no GPU): the library loads and exports every
+declared entry point, validation rejects bad input with the documented status
+before any device work, and the host relabeling solve is exact."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from workloads import configs as C
+from workloads import gen
+
+costa = pytest.importorskip("paper_2106_06601_gb300")
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "costa_gb300.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(costa_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported():
+    names = declared_functions()
+    assert len(names) >= 14
+    lib = costa.library()
+    for n in names:
+        assert hasattr(lib, n), n
+    assert costa.costa_abi_version() == 1
+    assert costa.costa_kernel_launch_count() >= 0
+
+
+FAKE = 1 << 40  # a device-looking address; layout creation never dereferences it
+
+
+def _spec_arrays(spec, esize=8):
+    ptrs = FAKE + (spec.off + spec.buf.astype(np.int64) * (1 << 30)) * esize
+    return ptrs
+
+
+def test_layout_create_accepts_valid_specs():
+    for p in (C.c1(), C.c2(), C.fuzz_problem(3)):
+        L = costa.costa_layout_from_spec(p.A, p.dtype, _spec_arrays(p.A, {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[p.dtype]))
+        m, n, P, dt = L.info()
+        assert (m, n, P) == (p.A.m, p.A.n, p.A.nranks)
+        L.destroy()
+
+
+def _expect(status, fn, *a):
+    with pytest.raises(costa.CostaError) as e:
+        fn(*a)
+    assert e.value.status == status, str(e.value)
+    assert costa.costa_last_error()
+
+
+def test_layout_validation_errors():
+    R = [0, 4, 8]
+    Cs = [0, 3, 6]
+    own = [[0, 1], [1, 0]]
+    ptr = [[FAKE, FAKE + 4096], [FAKE + 8192, FAKE + 12288]]
+    ld = [[4, 4], [4, 4]]
+    order = [[0, 0], [0, 0]]
+    mk = costa.costa_layout_create
+    mk("f64", 2, R, Cs, own, ptr, ld, order).destroy()
+    _expect(2, mk, "f64", 2, [0, 5, 4], Cs, own, ptr, ld, order)          # unsorted
+    _expect(2, mk, "f64", 2, [1, 4, 8], Cs, own, ptr, ld, order)          # not from 0
+    _expect(2, mk, "f64", 2, R, Cs, [[0, 2], [1, 0]], ptr, ld, order)     # owner range
+    _expect(2, mk, "f64", 2, R, Cs, own, ptr, [[3, 4], [4, 4]], order)    # ld < rows
+    _expect(2, mk, "f64", 2, R, Cs, own, [[FAKE + 4, 0], [8, 16]], ld, order)  # misaligned / null
+    _expect(2, mk, "f64", 2, R, Cs, own, ptr, ld, [[0, 2], [0, 0]])       # bad order
+    _expect(2, mk, "f64", 2, R, Cs, own, ptr, [[4, 1 << 31], [4, 4]], order)  # ld too large
+    _expect(1, mk, "f64", 0, R, Cs, own, ptr, ld, order)                  # nranks
+    # row-major blocks need ld >= cols
+    _expect(2, mk, "f64", 2, R, Cs, own, ptr, [[2, 3], [3, 3]], [[1, 1], [1, 1]])
+    mk("f64", 2, R, Cs, own, ptr, [[3, 3], [3, 3]], [[1, 1], [1, 1]]).destroy()
+    # c128 pointers must be 16-byte aligned
+    _expect(2, mk, "c128", 2, R, Cs, own, [[FAKE + 8, FAKE], [FAKE, FAKE]], ld, order)
+
+
+def test_block_cyclic_factory_matches_explicit_layout():
+    p = C.c2(n=512)
+    # rank r's buffer at FAKE + r * 2^30 bytes, column-major, lld = local rows
+    lld = [128] * 16
+    perm = np.zeros(16, np.int32)
+    # the spec's owner of grid rank g is p.A.meta's permutation; recover it
+    for bi in range(4):
+        for bj in range(4):
+            perm[bi * 4 + bj] = p.A.owner[bi, bj]
+    L = costa.costa_layout_create_block_cyclic("f64", 512, 512, 128, 128, 4, 4, "R", perm,
+                                               [FAKE + r * (1 << 30) for r in range(16)], lld)
+    assert L.info()[:3] == (512, 512, 16)
+    L.destroy()
+    _expect(2, costa.costa_layout_create_block_cyclic, "f64", 512, 512, 128, 128, 4, 4, "R",
+            [0] * 16, [FAKE] * 16, lld)                                   # not a permutation
+    _expect(2, costa.costa_layout_create_block_cyclic, "f64", 512, 512, 128, 128, 4, 4, "R",
+            None, [FAKE] * 16, [64] * 16)                                 # lld < local rows
+    _expect(1, costa.costa_layout_create_block_cyclic, "f64", 512, 512, 128, 128, 4, 4, "X",
+            None, [FAKE] * 16, lld)
+
+
+def test_transform_validation_before_device_work():
+    p = C.c1()
+    A = costa.costa_layout_from_spec(p.A, "f64", _spec_arrays(p.A))
+    B = costa.costa_layout_from_spec(p.B, "f64", _spec_arrays(p.B))
+    Bs = costa.costa_layout_from_spec(p.B, "f32", _spec_arrays(p.B, 4))
+    q = C.fuzz_problem(2, dtype="f64", op="T")
+    Bq = costa.costa_layout_from_spec(q.B, "f64", _spec_arrays(q.B))
+    n0 = costa.costa_kernel_launch_count()
+    _expect(4, costa.costa_transform, A, Bs, "N", 1.0, 0.0)               # dtype mismatch
+    _expect(3, costa.costa_transform, A, Bq, "N", 1.0, 0.0)               # shape / ranks
+    # a non-square problem: op = T needs swapped dims
+    r = C.fuzz_problem(7, op="N")
+    while r.A.m == r.A.n:
+        r = C.fuzz_problem(r.index + 64, op="N")
+    Ar = costa.costa_layout_from_spec(r.A, r.dtype, _spec_arrays(r.A, {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[r.dtype]))
+    Br = costa.costa_layout_from_spec(r.B, r.dtype, _spec_arrays(r.B, {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[r.dtype]))
+    _expect(3, costa.costa_transform, Ar, Br, "T", 1.0, 0.0)
+    lib = costa.library()
+    import ctypes
+    one = np.array([1.0])
+    st = lib.costa_transform_ex(A.handle, B.handle, 7, one.ctypes.data, one.ctypes.data, 0,
+                                None, 0, None)
+    assert st == 1
+    st = lib.costa_transform_ex(A.handle, B.handle, 0, None, one.ctypes.data, 0, None, 0, None)
+    assert st == 1
+    st = lib.costa_transform_ex(A.handle, B.handle, 0, one.ctypes.data, one.ctypes.data, 0,
+                                None, 5, None)
+    assert st == 1
+    st = lib.costa_transform_batched(0, None, None, None, None, None, 0, None, None)
+    assert st == 1
+    assert costa.costa_kernel_launch_count() == n0
+    for L in (A, B, Bs, Bq, Ar, Br):
+        L.destroy()
+
+
+# ----------------------------------------------------------------------------
+# relabeling (host Hungarian) against the oracle's exact solvers
+# ----------------------------------------------------------------------------
+
+def _rand_V(P, seed):
+    rng = gen.IntStream(seed, 9)
+    V = np.array([[rng.below(50) for _ in range(P)] for _ in range(P)], np.int64)
+    V[V % 4 == 0] = 0
+    return V
+
+
+@pytest.mark.parametrize("P", [1, 2, 3, 5, 8, 13, 16, 20, 31, 64])
+def test_relabel_is_optimal(P):
+    for s in range(6):
+        V = _rand_V(P, 1000 * P + s)
+        sigma, lv = costa.costa_relabel(V)
+        assert sorted(sigma.tolist()) == list(range(P))
+        assert oracle.objective(V, sigma) == lv == oracle.lap_optimum(V)
+
+
+def test_relabel_large_and_exact_integers():
+    V = _rand_V(256, 5) * (1 << 30)
+    sigma, lv = costa.costa_relabel(V)
+    assert lv == oracle.objective(V, sigma) == oracle.lap_library(V)[0]
+
+
+def test_relabel_tie_rule_keeps_identity():
+    V = np.full((4, 4), 4096, np.int64)          # c1: every permutation optimal
+    sigma, lv = costa.costa_relabel(V)
+    assert sigma.tolist() == [0, 1, 2, 3] and lv == 16384
+    V = np.diag([5, 5, 5]).astype(np.int64) + 1
+    sigma, _ = costa.costa_relabel(V)
+    assert sigma.tolist() == [0, 1, 2]
+
+
+def test_relabel_finds_permutation():
+    perm = gen.IntStream(3, 3).permutation(12)
+    V = np.zeros((12, 12), np.int64)
+    for q in range(12):
+        V[perm[q], q] = 100 + q
+    sigma, lv = costa.costa_relabel(V)
+    assert sigma.tolist() == perm and lv == sum(100 + q for q in range(12))
+
+
+def test_relabel_rejects_bad_input():
+    _expect(1, costa.costa_relabel, np.array([[-1, 0], [0, 0]]))
+    lib = costa.library()
+    sig = np.zeros(2, np.int32)
+    assert lib.costa_relabel(0, None, sig.ctypes.data, None) == 1

@@ -1,0 +1,172 @@
+"""The five workload configurations at full size, in the launch configuration
+the bench times (one costa_transform / costa_transform_batched call, direct
+mode, cached plan).
+
+Inputs are filled on the device by the seeded generator.  Sampled outputs are
+checked element by element against the oracle, which gets the sampled input
+values read back before the transform: random samples plus every block corner
+and edge sample of A.  Volumes and optima are checked against the hand-derived
+closed forms (tests/golden/closed_forms.json), and properties that hold at
+any size (no NaN left where A was pre-filled with NaN, B untouched) are
+checked on whole buffers.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from tests._util import assert_close, exact_case
+from workloads import configs as C
+from workloads.materialize import DeviceMatrix
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "closed_forms.json")
+
+
+@pytest.fixture(scope="module")
+def dev():
+    d = torch.device("cuda:0")
+    torch.cuda.set_device(d)
+    return d
+
+
+def sample_points(spec, n_random: int, seed: int) -> np.ndarray:
+    rng = np.random.default_rng(seed)
+    pts = [np.stack([rng.integers(0, spec.m, n_random), rng.integers(0, spec.n, n_random)], 1)]
+    # corners and edge midpoints of (up to) 4096 blocks
+    nb = spec.nbr * spec.nbc
+    pick = rng.choice(nb, size=min(nb, 4096), replace=False)
+    bi, bj = pick // spec.nbc, pick % spec.nbc
+    r0, r1 = spec.rsplit[bi], spec.rsplit[bi + 1] - 1
+    c0, c1 = spec.csplit[bj], spec.csplit[bj + 1] - 1
+    ok = (r1 >= r0) & (c1 >= c0)
+    for a, b in ((r0, c0), (r0, c1), (r1, c0), (r1, c1), ((r0 + r1) // 2, c1), (r1, (c0 + c1) // 2)):
+        pts.append(np.stack([a[ok], b[ok]], 1))
+    return np.concatenate(pts).astype(np.int64)
+
+
+class Mat:
+    def __init__(self, p, dev):
+        import paper_2106_06601_gb300 as costa
+        self.p = p
+        self.Bd = DeviceMatrix(p.B, p.dtype, dev).fill(p.b_kind, p.seed, p.src_stream)
+        self.Ad = DeviceMatrix(p.A, p.dtype, dev).fill(p.a_kind, p.seed, p.tgt_stream)
+        self.LA = costa.costa_layout_from_spec(p.A, p.dtype, self.Ad.block_ptrs())
+        self.LB = costa.costa_layout_from_spec(p.B, p.dtype, self.Bd.block_ptrs())
+
+    def sample_index(self, ij):
+        _, abuf, aoff = oracle.locate(self.p.A, ij)
+        src = ij if self.p.op == "N" else ij[:, ::-1].copy()
+        _, bbuf, boff = oracle.locate(self.p.B, src)
+        ia = torch.as_tensor(self.Ad.starts[abuf] + aoff, device=self.Ad.arena.device)
+        ib = torch.as_tensor(self.Bd.starts[bbuf] + boff, device=self.Bd.arena.device)
+        return ia, ib
+
+    def close(self):
+        self.LA.destroy()
+        self.LB.destroy()
+
+
+def check_samples(p, a_pre, b, a_post):
+    want = oracle.combine(p.dtype, p.op, p.alpha, p.beta, b, a_pre)
+    al, be = oracle.scalar(p.dtype, p.alpha), oracle.scalar(p.dtype, p.beta)
+    bvals = b.astype(np.complex128)
+    if p.op == "C":
+        bvals = np.conj(bvals)
+    assert_close(p.dtype, a_post, want, al, be,
+                 bvals if p.dtype in ("c64", "c128") else bvals.real, a_pre,
+                 exact=exact_case(p.dtype, al, be))
+
+
+def blocks_have_no_nan(p, Ad):
+    """A was pre-filled with NaN and beta = 0: every block element is written."""
+    for r in range(p.A.nbuf):
+        buf = Ad.buffer(r)
+        covered = int(p.A.bufsize[r])
+        assert covered == buf.numel()
+        if torch.isnan(torch.view_as_real(buf) if buf.is_complex() else buf).any():
+            return False
+    return True
+
+
+@pytest.mark.parametrize("name", ["c2", "c3", "c5"])
+def test_config_full_size(name, dev):
+    import paper_2106_06601_gb300 as costa
+    p = C.CONFIGS[name]()
+    mat = Mat(p, dev)
+    try:
+        ij = sample_points(p.A, 200_000, 7)
+        ia, ib = mat.sample_index(ij)
+        a_pre = mat.Ad.arena[ia].cpu().numpy()
+        b = mat.Bd.arena[ib].cpu().numpy()
+        b_sum = torch.view_as_real(mat.Bd.arena).sum(dtype=torch.float64).item() \
+            if mat.Bd.arena.is_complex() else mat.Bd.arena.sum(dtype=torch.float64).item()
+        stream = torch.cuda.current_stream().cuda_stream
+        sigma = costa.costa_transform(mat.LA, mat.LB, p.op, p.alpha, p.beta, relabel=True,
+                                      stream=stream)
+        torch.cuda.synchronize()
+        a_post = mat.Ad.arena[ia].cpu().numpy()
+        check_samples(p, a_pre, b, a_post)
+        # B is read-only
+        b_sum2 = torch.view_as_real(mat.Bd.arena).sum(dtype=torch.float64).item() \
+            if mat.Bd.arena.is_complex() else mat.Bd.arena.sum(dtype=torch.float64).item()
+        assert b_sum == b_sum2
+        if p.a_kind == "nan":
+            assert blocks_have_no_nan(p, mat.Ad)
+        V = costa.costa_volume(mat.LA, mat.LB, p.op, stream)
+        assert V.sum() == p.A.m * p.A.n
+        cf = json.load(open(GOLDEN)).get(name)
+        best = oracle.lap_optimum(V)
+        if cf:
+            assert V.sum() == cf["total"] and best == cf["optimum"]
+            assert set(np.unique(V).tolist()) == {0, cf["package"]}
+        assert oracle.objective(V, sigma) == best
+        st = costa.costa_plan_stats_get(mat.LA, mat.LB, p.op, relabel=True)
+        assert st["local_relabeled"] == best
+    finally:
+        mat.close()
+
+
+def test_config_c3_volume_matches_oracle_count(dev):
+    """c3's irregular target grid has no closed form: compare V with the
+    oracle's element-by-element count."""
+    import paper_2106_06601_gb300 as costa
+    p = C.c3()
+    mat = Mat(p, dev)
+    try:
+        V = costa.costa_volume(mat.LA, mat.LB, p.op, torch.cuda.current_stream().cuda_stream)
+        assert np.array_equal(V, oracle.volume(p.op, p.A, p.B, 64))
+    finally:
+        mat.close()
+
+
+def test_config_c4_batched(dev):
+    import paper_2106_06601_gb300 as costa
+    probs = C.c4()
+    mats = [Mat(p, dev) for p in probs]
+    try:
+        idx = []
+        for k, (p, m) in enumerate(zip(probs, mats)):
+            ij = sample_points(p.A, 20_000, 100 + k)
+            ia, ib = m.sample_index(ij)
+            idx.append((ia, ib, m.Ad.arena[ia].cpu().numpy(), m.Bd.arena[ib].cpu().numpy()))
+        stream = torch.cuda.current_stream().cuda_stream
+        sigma = costa.costa_transform_batched([m.LA for m in mats], [m.LB for m in mats],
+                                              [p.op for p in probs], [p.alpha for p in probs],
+                                              [p.beta for p in probs], relabel=True,
+                                              stream=stream)
+        torch.cuda.synchronize()
+        for p, m, (ia, ib, a_pre, b) in zip(probs, mats, idx):
+            check_samples(p, a_pre, b, m.Ad.arena[ia].cpu().numpy())
+            assert blocks_have_no_nan(p, m.Ad)
+        st = costa.costa_plan_stats_get([m.LA for m in mats], [m.LB for m in mats],
+                                        [p.op for p in probs], relabel=True)
+        assert st["total_volume"] == 64 * 2048 * 3072
+        assert sorted(sigma.tolist()) == list(range(16))
+    finally:
+        for m in mats:
+            m.close()

@@ -1,0 +1,185 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Small seeded problems are compared element by element over whole buffers:
+bit-exact where the arithmetic allows it (beta = 0, or power-of-two scalars),
+otherwise within the tolerance derived in tests/_util.tolerance; padding and
+guard elements must stay untouched.  Volumes and relabelings are compared
+exactly.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from tests._gpu import OnDevice, compare
+from workloads import configs as C
+from workloads import layouts as L
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def dev():
+    d = torch.device("cuda:0")
+    torch.cuda.set_device(d)
+    return d
+
+
+def check_problem(p, dev, mode="direct", relabel=True, guard=0):
+    g = OnDevice(p, dev, guard=guard)
+    try:
+        sigma = g.run(relabel=relabel, mode=mode)
+        got = g.Ad.download()
+        want = g.oracle_result()
+        compare(p, got, want, g.Ah, g.Bh)
+        # B is read-only
+        assert np.array_equal(g.Bd.download().arena, g.Bh.arena, equal_nan=True)
+        return sigma, got
+    finally:
+        g.close()
+
+
+@pytest.mark.parametrize("case", range(120))
+def test_fuzz_direct(case, dev):
+    check_problem(C.fuzz_problem(case), dev, guard=3 if case % 4 == 0 else 0)
+
+
+@pytest.mark.parametrize("case", range(120, 180))
+def test_fuzz_message_equals_direct(case, dev):
+    p = C.fuzz_problem(case)
+    _, direct = check_problem(p, dev, mode="direct")
+    for relabel in (False, True):
+        _, msg = check_problem(p, dev, mode="message", relabel=relabel)
+        assert np.array_equal(msg.arena, direct.arena, equal_nan=True)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64", "c64", "c128"])
+@pytest.mark.parametrize("op", ["N", "T", "C"])
+def test_all_dtypes_ops_multi_tile(dtype, op, dev):
+    """Several tiles in each direction plus a ragged tail, both storage orders."""
+    for storage_b, storage_a in (("C", "C"), ("R", "C"), ("C", "R"), ("R", "R")):
+        m, n = 133, 97
+        B = L.block_cyclic(m, n, 40, 24, 2, 3, storage=storage_b, ld_pad=1)
+        am, an = (m, n) if op == "N" else (n, m)
+        A = L.block_cyclic(am, an, 33, 64, 3, 2, grid_order="C", storage=storage_a)
+        for alpha, beta in ((1.0, 0.0), (2.0, 0.5), (-0.3, 0.7)):
+            p = C.Problem("grid", dtype, op, alpha, beta, A, B, "uniform",
+                          "nan" if beta == 0 else "uniform", C.SEED0 + 9)
+            check_problem(p, dev)
+
+
+def test_c1_bit_exact_and_relabel(dev):
+    p = C.c1()
+    sigma, _ = check_problem(p, dev, relabel=True, guard=5)
+    V = oracle.volume(p.op, p.A, p.B, 4)
+    assert oracle.objective(V, sigma) == oracle.lap_optimum(V) == 16384
+    assert sigma.tolist() == [0, 1, 2, 3]         # all ties: identity kept
+
+
+@pytest.mark.parametrize("case", range(30))
+def test_volume_matches_oracle(case, dev):
+    import paper_2106_06601_gb300 as costa
+    p = C.fuzz_problem(case)
+    g = OnDevice(p, dev)
+    try:
+        V = costa.costa_volume(g.LA, g.LB, p.op, torch.cuda.current_stream().cuda_stream)
+        assert np.array_equal(V, oracle.volume(p.op, p.A, p.B, p.A.nranks))
+        st = costa.costa_plan_stats_get(g.LA, g.LB, p.op, relabel=True)
+        assert st["total_volume"] == p.A.m * p.A.n
+        assert st["local_identity"] == int(np.trace(V))
+        assert st["local_relabeled"] == oracle.lap_optimum(V)
+    finally:
+        g.close()
+
+
+def test_relabel_does_not_change_result(dev):
+    for case in (5, 17, 33):
+        p = C.fuzz_problem(case)
+        _, a = check_problem(p, dev, relabel=False)
+        _, b = check_problem(p, dev, relabel=True)
+        assert np.array_equal(a.arena, b.arena, equal_nan=True)
+
+
+def test_repeat_calls_deterministic(dev):
+    p = C.fuzz_problem(44, dtype="c128")
+    p.alpha, p.beta = complex(0.3, -0.2), complex(1.1, 0.4)
+    g = OnDevice(p, dev)
+    try:
+        g.run()
+        first = g.Ad.download().arena.copy()
+        g.reset_A()
+        g.run()
+        assert np.array_equal(first, g.Ad.download().arena)
+    finally:
+        g.close()
+
+
+def test_edge_cases(dev):
+    # 1 x 1, P = 1
+    B = L.block_cyclic(1, 1, 1, 1, 1, 1)
+    A = L.block_cyclic(1, 1, 4, 4, 1, 1)
+    check_problem(C.Problem("1x1", "f64", "T", 2.0, 0.0, A, B, "uniform", "nan"), dev)
+    # a single tall column and a single wide row
+    for (m, n) in ((1000, 1), (1, 777)):
+        B = L.block_cyclic(m, n, 7, 5, 2, 1)
+        A = L.block_cyclic(n, m, 3, 11, 1, 2, storage="R")
+        check_problem(C.Problem("thin", "f32", "T", 1.0, 0.0, A, B, "uniform", "nan"), dev)
+    # empty blocks inside irregular splits
+    rs = np.array([0, 0, 5, 5, 17, 40], np.int64)
+    cs = np.array([0, 9, 9, 30], np.int64)
+    own = np.arange(15, dtype=np.int32).reshape(5, 3) % 4
+    A = L.packed_blocks(rs, cs, own, 4)
+    B = L.block_cyclic(40, 30, 6, 4, 2, 2)
+    check_problem(C.Problem("empty-blocks", "c64", "N", 0.5, -1.0, A, B, "uniform", "uniform"),
+                  dev)
+
+
+def test_empty_matrix(dev):
+    import paper_2106_06601_gb300 as costa
+    A = L.packed_blocks([0], [0, 5], np.zeros((0, 1), np.int32), 2)
+    B = L.packed_blocks([0, 5], [0], np.zeros((1, 0), np.int32), 2)
+    LA = costa.costa_layout_create("f64", 2, A.rsplit, A.csplit, A.owner, np.zeros((0, 1)),
+                                   A.ld, A.order)
+    LB = costa.costa_layout_create("f64", 2, B.rsplit, B.csplit, B.owner, np.zeros((1, 0)),
+                                   B.ld, B.order)
+    sigma = costa.costa_transform(LA, LB, "T", 1.0, 0.0, relabel=True)
+    assert sigma.tolist() == [0, 1]
+    assert costa.costa_volume(LA, LB, "T").sum() == 0
+
+
+def test_batched_matches_oracle(dev):
+    import paper_2106_06601_gb300 as costa
+    probs = []
+    scal = [(1.0, 0.0), (2.0, 0.5), (-0.3, 0.7), (1.0, 0.0), (0.5, 0.0)]
+    for k in range(10):
+        p = C.fuzz_problem(300 + k, dtype="f64", P=4)
+        p.alpha, p.beta = scal[k % len(scal)]
+        p.a_kind = "nan" if p.beta == 0 else "uniform"
+        probs.append(p)
+    gs = [OnDevice(p, dev) for p in probs]
+    try:
+        stream = torch.cuda.current_stream().cuda_stream
+        sigma = costa.costa_transform_batched([g.LA for g in gs], [g.LB for g in gs],
+                                              [p.op for p in probs], [p.alpha for p in probs],
+                                              [p.beta for p in probs], relabel=True,
+                                              stream=stream)
+        torch.cuda.synchronize()
+        Vsum = sum(oracle.volume(p.op, p.A, p.B, 4) for p in probs)
+        assert oracle.objective(Vsum, sigma) == oracle.lap_optimum(Vsum)
+        for p, g in zip(probs, gs):
+            compare(p, g.Ad.download(), g.oracle_result(), g.Ah, g.Bh)
+        # message mode of the same batch gives the same bits
+        results = [g.Ad.download().arena.copy() for g in gs]
+        for g in gs:
+            g.reset_A()
+        costa.costa_transform_batched([g.LA for g in gs], [g.LB for g in gs],
+                                      [p.op for p in probs], [p.alpha for p in probs],
+                                      [p.beta for p in probs], relabel=True, stream=stream,
+                                      mode="message")
+        torch.cuda.synchronize()
+        for g, r in zip(gs, results):
+            assert np.array_equal(g.Ad.download().arena, r, equal_nan=True)
+    finally:
+        for g in gs:
+            g.close()
