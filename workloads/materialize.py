@@ -56,7 +56,8 @@ class HostMatrix:
     def __init__(self, spec, dtype: str, guard: int = 0, sentinel=None):
         self.spec, self.dtype, self.guard = spec, dtype, guard
         self.starts, total = arena_offsets(spec.bufsize, ESIZE[dtype], guard)
-        self.arena = np.empty(total, dtype=gen.np_dtype(dtype))
+        # zeroed (or sentinel-filled) so that alignment gaps are deterministic
+        self.arena = np.zeros(total, dtype=gen.np_dtype(dtype))
         if sentinel is not None:
             self.arena[...] = sentinel
 
