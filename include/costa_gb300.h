@@ -213,6 +213,33 @@ costa_status costa_plan_stats_get(int n, const costa_layout *A, const costa_layo
 costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op, int axis,
                                      int32_t *out, int64_t cap, int64_t *count);
 
+/* The volumes of costa_volume (same V, same layout of the result) computed
+ * without allocating device memory.  The paper has no counterpart: it exists
+ * for callers that cannot let a library call cudaMalloc, such as an
+ * application whose framework owns all device memory through its own pool,
+ * or code on a latency-critical path where cudaMalloc / cudaFree would
+ * synchronize the device.
+ *  - Memory: all device work happens in one fixed scratch array of 4 MiB
+ *    that is part of the library's device image; every GPU that loads the
+ *    library holds it until the process exits.  No cudaMalloc, cudaFree or
+ *    other allocating call is made, and no plan is built or cached.
+ *  - Limit: the pair needs 8 * P^2 bytes for V plus its split and owner
+ *    arrays (8 bytes per split, 4 per block of A and of B, each section
+ *    rounded up to 256 bytes); more than 4 MiB is rejected with
+ *    COSTA_ERR_INVALID_ARG and a message giving both sizes.
+ *  - Set-up: the first call on a device, with that device current, looks up
+ *    the array's device address (cudaGetSymbolAddress).  Make that first call
+ *    before any stream capture.
+ *  - Sharing: every call uses the same array, which keeps the last call's
+ *    contents (V is zeroed on the stream at the start of each call).  Calls
+ *    that overlap on the GPU would race; this entry point is synchronous and
+ *    serializes its own calls, so they do not overlap within one process.
+ *  - Synchronization: runs on `stream` and synchronizes it before returning.
+ * V: host array of P * P int64, as in costa_volume.  Errors: INVALID_ARG,
+ * SHAPE, DTYPE, CUDA. */
+costa_status costa_volume_noalloc(costa_layout A, costa_layout B, costa_op op, int64_t *V,
+                                  void *stream);
+
 /* Frees every cached plan (synchronizes the device). */
 costa_status costa_release_plans(void);
 

@@ -62,6 +62,7 @@ def _load():
         "costa_layout_destroy": [P],
         "costa_layout_info": [P, P, P, P, P],
         "costa_volume": [P, P, I, P, P],
+        "costa_volume_noalloc": [P, P, I, P, P],
         "costa_relabel": [I, P, P, P],
         "costa_transform": [P, P, I, P, P, I, P, P],
         "costa_transform_ex": [P, P, I, P, P, I, P, I, P],
@@ -182,6 +183,14 @@ def costa_volume(A: Layout, B: Layout, op: str, stream: int = 0) -> np.ndarray:
     _, _, P, _ = A.info()
     V = np.zeros((P, P), dtype=np.int64)
     _check(_lib.costa_volume(A.handle, B.handle, OPS[op], _p(V), ctypes.c_void_p(stream)))
+    return V
+
+
+def costa_volume_noalloc(A: Layout, B: Layout, op: str, stream: int = 0) -> np.ndarray:
+    """costa_volume without device allocation (fixed 4 MiB scratch)."""
+    _, _, P, _ = A.info()
+    V = np.zeros((P, P), dtype=np.int64)
+    _check(_lib.costa_volume_noalloc(A.handle, B.handle, OPS[op], _p(V), ctypes.c_void_p(stream)))
     return V
 
 

@@ -19,17 +19,6 @@
 
 #include "costa_internal.h"
 
-struct costa_layout_s {
-    uint64_t id;
-    costa_dtype dt;
-    int nranks;
-    int nbr, nbc;
-    int64_t m, n;
-    std::vector<int64_t> R, C;
-    std::vector<int32_t> owner;
-    std::vector<costa::DevBlock> blocks;
-};
-
 namespace costa {
 
 int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
@@ -669,6 +658,13 @@ int64_t numroc(int64_t n, int64_t nb, int iproc, int nprocs) {
 }
 
 }  // namespace
+
+costa_status report_error(costa_status s, const char *message) { return fail(s, "%s", message); }
+
+costa_status check_pair(const costa_layout_s *A, const costa_layout_s *B, int op) {
+    return validate_pair(A, B, op);
+}
+
 }  // namespace costa
 
 using namespace costa;

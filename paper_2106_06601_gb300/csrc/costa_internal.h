@@ -1,8 +1,9 @@
 // Internal types shared by the host planner (costa.cpp) and the kernels
-// (remap_*.cu, volume.cu).  Not part of the public ABI.
+// (remap_*.cu, volume.cu and the other .cu files).  Not part of the public ABI.
 #pragma once
 
 #include <cstdint>
+#include <vector>
 
 #include <cuda_runtime_api.h>
 
@@ -23,6 +24,22 @@ struct DevBlock {
     int32_t order;  // 0 column-major, 1 row-major
 };
 static_assert(sizeof(DevBlock) == 16, "DevBlock layout");
+
+}  // namespace costa
+
+// A layout as the library holds it (host copies of the description).
+struct costa_layout_s {
+    uint64_t id;
+    costa_dtype dt;
+    int nranks;
+    int nbr, nbc;
+    int64_t m, n;
+    std::vector<int64_t> R, C;
+    std::vector<int32_t> owner;
+    std::vector<costa::DevBlock> blocks;
+};
+
+namespace costa {
 
 // One piece of a grid-overlay interval along one axis (rows or columns of A),
 // at most the kernel tile extent long.  The overlay (Sec. 5, "Grid Overlay")
@@ -131,5 +148,10 @@ cudaError_t launch_remap_c128(const RemapLaunch &args, int mode, int kind, cudaS
 cudaError_t launch_volume(const VolumeLaunch &args, cudaStream_t stream);
 void count_launch();
 int64_t launches_so_far();
+
+// Error reporting and pair validation shared with entry points defined
+// outside costa.cpp.
+costa_status report_error(costa_status s, const char *message);
+costa_status check_pair(const costa_layout_s *A, const costa_layout_s *B, int op);
 
 }  // namespace costa
