@@ -6,23 +6,31 @@
 // Overlay") is the product of row intervals and column intervals; the host
 // cuts each interval into pieces of at most TS elements, so the kernel's tile
 // grid is (row pieces) x (column pieces), and every tile lies inside one block
-// of A and one block of B.  Inside a tile both storages are affine, so one
-// warp moves it with 16-byte vector accesses where alignment allows:
-//   - if A and the source share their contiguous axis, the warp copies runs
-//     straight through registers;
-//   - otherwise it transposes through a padded shared-memory tile (Sec. 6:
-//     "cache-friendly ... kernel for matrix transposition"): source runs in,
-//     target runs out, with alpha / beta applied as one fma on the way out
-//     (Sec. 5: transform after receive).
-// Warps sweep the tile list in a grid-stride loop over a persistent grid.
+// of A and one block of B.  Inside a tile both storages are affine.
+//
+// One warp moves one tile at a time, in a software pipeline over its tiles:
+//   1. the source tile is staged into shared memory with 16-byte cp.async
+//      copies (no registers held while in flight), one run of the source's
+//      contiguous axis per shared-memory row, chunks XOR-swizzled per row so
+//      that reading it transposed is free of avoidable bank conflicts;
+//   2. while that is in flight the warp issues the copies of its next tile
+//      into the other buffer and, when beta != 0, loads its A chunks into
+//      registers;
+//   3. it then writes A in A's contiguous order, 16 bytes per lane, applying
+//      alpha and beta as one fma per element on the way out (Sec. 5:
+//      transform after receive).
+// If A and the source share their contiguous axis the staged rows are read
+// straight; otherwise they are read across rows (the transpose of Sec. 6's
+// "cache-friendly ... kernel for matrix transposition").  Ragged or
+// misaligned tiles take an element-wise path.
 //
 // Modes: DIRECT_ALL (B -> A for every tile), and the message path of Alg. 3 /
 // Sec. 6: PACK (remote tiles: B -> staging, an exact copy), DIRECT_LOCAL
 // (tiles local after relabeling: B -> A), UNPACK (remote tiles: staging -> A
 // with the transform).
 //
-// No kernel here waits on another block or on a flag: there are no
-// spin-waits, so no wait can fail to end.
+// No kernel here waits on another block or on a flag.  cp.async.wait_group
+// waits only for this thread's own copies, which always complete.
 
 #pragma once
 
@@ -43,17 +51,21 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 
 // Per element type: tile extent TS, 16-byte chunk width VEC (elements), and
 // the lane mapping: CPR chunks cover one run of TS elements, a warp pass
-// covers RPP runs, NPASS passes cover TS runs.
+// covers RPP runs, NPASS passes cover TS runs.  A staged tile is TS rows of
+// CPR chunks (TS * TS elements); the element-wise path uses a TS x (TS + 1)
+// array in the same buffer.
 template <typename T> struct Cfg {
     static constexpr int TS = sizeof(T) == 16 ? 16 : 32;
     static constexpr int VEC = ET<T>::VEC;
     static constexpr int CPR = TS / VEC;
     static constexpr int RPP = 32 / CPR;
     static constexpr int NPASS = TS / RPP;
-    static constexpr int PITCH = TS + 1;  // odd pitch: conflict-light columns
-    static constexpr int SMEM_ELEMS = TS * PITCH;
+    static constexpr int PITCH = TS + 1;
+    static constexpr int BUF_BYTES_RAW = TS * PITCH * static_cast<int>(sizeof(T));
+    static constexpr int BUF_BYTES = (BUF_BYTES_RAW + 127) / 128 * 128;
 };
-constexpr int kWarps = 8;
+constexpr int kWarps = 4;
+constexpr int kMinBlocks = 3;
 
 template <typename T> struct Chunk {
     union {
@@ -62,12 +74,14 @@ template <typename T> struct Chunk {
     };
 };
 
-template <typename T>
-__device__ __forceinline__ Chunk<T> load_ro(const T *p) {
-    Chunk<T> c;
-    c.raw = __ldg(reinterpret_cast<const uint4 *>(p));
-    return c;
+// ---- asynchronous 16-byte global -> shared copies (sm_80+ cp.async) ----
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+    const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
 }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
 template <typename T>
 __device__ __forceinline__ Chunk<T> load_rw(const T *p) {
@@ -94,7 +108,6 @@ struct Sc {
 
 // Combine of one element for a kind K_* (costa_internal.h); the kernel is
 // compiled per kind.  b arrives conjugated (op = C) via conj_mask.
-
 template <int KIND, typename R>
 __device__ __forceinline__ R comb_real(R b, R a, const Sc &s) {
     if (KIND == K_COPY) return b;
@@ -145,160 +158,125 @@ __device__ __forceinline__ double2 combine(double2 b, double2 a, const Sc &s) {
 //   target element (x, y) at dst + x + y * dld
 //   source element (x, y) at src + x + y * sld        (copy tile)
 //                         or src + x * sld + y        (transposed tile)
+// The source's runs (its contiguous axis) are rows of the staged tile: for a
+// copy tile row y holds x = 0..nx-1, for a transposed tile row x holds
+// y = 0..ny-1.
 template <typename T> struct Geom {
     T *dst;
     const T *src;
     int64_t dld, sld;
     int nx, ny;
-    bool transpose, dvec, svec;
+    bool transpose, fast;
 };
 
-// Fast paths: every chunk is a full, 16-byte aligned vector (checked by the
-// caller), so the unrolled loops carry no element-level branches.
+// Chunk c of staged row r lives in slot c ^ swz(r): across the VEC rows that
+// one output chunk reads, and across neighbouring chunks, the slots differ,
+// so a transposed read needs only the minimum number of wavefronts.
+template <typename T>
+__device__ __forceinline__ int swz(int r) { return (r / Cfg<T>::VEC) & 7; }
 
-template <typename T, int KIND>
-__device__ __forceinline__ void tile_copy_vec(const Geom<T> &g, const Sc &s, int lane) {
-    constexpr bool READ_A = KIND >= K_AXPBY;
+template <typename T>
+__device__ __forceinline__ unsigned char *slot(unsigned char *buf, int r, int c) {
+    return buf + (r * Cfg<T>::CPR + (c ^ swz<T>(r))) * 16;
+}
+
+// Issue the cp.async copies of a fast tile's source into `buf`.
+template <typename T>
+__device__ __forceinline__ void stage_issue(const Geom<T> &g, unsigned char *buf, int lane) {
     using C = Cfg<T>;
-    constexpr int G = C::NPASS > 8 ? 8 : C::NPASS;  // passes in flight per group
+    const int runs = g.transpose ? g.nx : g.ny;            // source runs
+    const int chunks = (g.transpose ? g.ny : g.nx) / C::VEC;  // chunks per run
+    const int c = lane % C::CPR, r0 = lane / C::CPR;
+    if (c >= chunks) return;
+#pragma unroll 4
+    for (int r = r0; r < runs; r += C::RPP)
+        cp_async16(slot<T>(buf, r, c), g.src + static_cast<int64_t>(r) * g.sld + c * C::VEC);
+}
+
+// Write a staged fast tile to A, combining with A when the kind reads it.
+template <typename T, int KIND>
+__device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsigned char *buf,
+                                            const Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
+    using C = Cfg<T>;
     const int c = lane % C::CPR, yr = lane / C::CPR, x0 = c * C::VEC;
-    const bool lane_on = x0 < g.nx;
+    if (x0 >= g.nx) return;
 #pragma unroll
-    for (int p0 = 0; p0 < C::NPASS; p0 += G) {
-        Chunk<T> bv[G], av[G];
+    for (int p = 0; p < C::NPASS; ++p) {
+        const int y = p * C::RPP + yr;
+        if (y < g.ny) {
+            Chunk<T> b;
+            if (g.transpose) {
+                // element (x0 + e, y) sits in row x0 + e, chunk y / VEC, lane y % VEC
+                const int cy = y / C::VEC, ey = y % C::VEC;
 #pragma unroll
-        for (int p = 0; p < G; ++p) {
-            av[p].raw = make_uint4(0, 0, 0, 0);
-            const int y = (p0 + p) * C::RPP + yr;
-            if (lane_on && y < g.ny) {
-                bv[p] = load_ro(g.src + y * g.sld + x0);
-                if (READ_A) av[p] = load_rw(g.dst + y * g.dld + x0);
+                for (int e = 0; e < C::VEC; ++e)
+                    b.e[e] = reinterpret_cast<const T *>(slot<T>(buf, x0 + e, cy))[ey];
+            } else {
+                b.raw = *reinterpret_cast<const uint4 *>(slot<T>(buf, y, c));
             }
-        }
+            Chunk<T> o;
 #pragma unroll
-        for (int p = 0; p < G; ++p) {
-            const int y = (p0 + p) * C::RPP + yr;
-            if (lane_on && y < g.ny) {
-                Chunk<T> o;
-#pragma unroll
-                for (int e = 0; e < C::VEC; ++e) o.e[e] = combine<KIND>(bv[p].e[e], av[p].e[e], s);
-                store(g.dst + y * g.dld + x0, o);
-            }
+            for (int e = 0; e < C::VEC; ++e) o.e[e] = combine<KIND>(b.e[e], av[p].e[e], s);
+            store(g.dst + static_cast<int64_t>(y) * g.dld + x0, o);
         }
     }
 }
 
 template <typename T, int KIND>
-__device__ __forceinline__ void tile_transpose_vec(const Geom<T> &g, const Sc &s, T *sm, int lane) {
+__device__ __forceinline__ void load_a(const Geom<T> &g, Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
     using C = Cfg<T>;
-    constexpr bool READ_A = KIND >= K_AXPBY;
-    constexpr int G = C::NPASS > 8 ? 8 : C::NPASS;  // target passes per group
-    {   // source runs (along y) -> sm[y][x]
-        const int c = lane % C::CPR, xr = lane / C::CPR, y0 = c * C::VEC;
-        const bool lane_on = y0 < g.ny;
+    const int c = lane % C::CPR, yr = lane / C::CPR, x0 = c * C::VEC;
 #pragma unroll
-        for (int p0 = 0; p0 < C::NPASS; p0 += G) {
-            Chunk<T> bv[G];
-#pragma unroll
-            for (int p = 0; p < G; ++p) {
-                const int x = (p0 + p) * C::RPP + xr;
-                if (lane_on && x < g.nx) bv[p] = load_ro(g.src + x * g.sld + y0);
-            }
-#pragma unroll
-            for (int p = 0; p < G; ++p) {
-                const int x = (p0 + p) * C::RPP + xr;
-                if (lane_on && x < g.nx) {
-#pragma unroll
-                    for (int e = 0; e < C::VEC; ++e) sm[(y0 + e) * C::PITCH + x] = bv[p].e[e];
-                }
-            }
-        }
+    for (int p = 0; p < C::NPASS; ++p) {
+        av[p].raw = make_uint4(0, 0, 0, 0);
+        const int y = p * C::RPP + yr;
+        if (KIND >= K_AXPBY && x0 < g.nx && y < g.ny)
+            av[p] = load_rw(g.dst + static_cast<int64_t>(y) * g.dld + x0);
     }
-    __syncwarp();
-    {   // target runs (along x) <- sm[y][x], combined with A
-        const int c = lane % C::CPR, yr = lane / C::CPR, x0 = c * C::VEC;
-        const bool lane_on = x0 < g.nx;
-#pragma unroll
-        for (int p0 = 0; p0 < C::NPASS; p0 += G) {
-            Chunk<T> av[G];
-#pragma unroll
-            for (int p = 0; p < G; ++p) {
-                av[p].raw = make_uint4(0, 0, 0, 0);
-                const int y = (p0 + p) * C::RPP + yr;
-                if (READ_A && lane_on && y < g.ny) av[p] = load_rw(g.dst + y * g.dld + x0);
-            }
-#pragma unroll
-            for (int p = 0; p < G; ++p) {
-                const int y = (p0 + p) * C::RPP + yr;
-                if (lane_on && y < g.ny) {
-                    Chunk<T> o;
-#pragma unroll
-                    for (int e = 0; e < C::VEC; ++e)
-                        o.e[e] = combine<KIND>(sm[y * C::PITCH + x0 + e], av[p].e[e], s);
-                    store(g.dst + y * g.dld + x0, o);
-                }
-            }
-        }
-    }
-    __syncwarp();
 }
 
-// General path for ragged or misaligned tiles: element by element, lanes
-// strided along the contiguous axis of each phase.
+// Element-wise path for ragged or misaligned tiles, lanes strided along the
+// contiguous axis of each phase; uses a TS x (TS + 1) array in `buf`.
 template <typename T, int KIND>
-__device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, T *sm, int lane) {
+__device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
     using C = Cfg<T>;
     constexpr bool READ_A = KIND >= K_AXPBY;
+    T *sm = reinterpret_cast<T *>(buf);
     const int n = g.nx * g.ny;
     if (!g.transpose) {
         for (int k = lane; k < n; k += 32) {
             const int y = k / g.nx, x = k - y * g.nx;
-            T *d = g.dst + y * g.dld + x;
+            T *d = g.dst + static_cast<int64_t>(y) * g.dld + x;
             const T a = READ_A ? *d : T();
-            *d = combine<KIND>(__ldg(g.src + y * g.sld + x), a, s);
+            *d = combine<KIND>(__ldg(g.src + static_cast<int64_t>(y) * g.sld + x), a, s);
         }
         return;
     }
     for (int k = lane; k < n; k += 32) {
         const int x = k / g.ny, y = k - x * g.ny;
-        sm[y * C::PITCH + x] = __ldg(g.src + x * g.sld + y);
+        sm[y * C::PITCH + x] = __ldg(g.src + static_cast<int64_t>(x) * g.sld + y);
     }
     __syncwarp();
     for (int k = lane; k < n; k += 32) {
         const int y = k / g.nx, x = k - y * g.nx;
-        T *d = g.dst + y * g.dld + x;
+        T *d = g.dst + static_cast<int64_t>(y) * g.dld + x;
         const T a = READ_A ? *d : T();
         *d = combine<KIND>(sm[y * C::PITCH + x], a, s);
     }
-    __syncwarp();
-}
-
-template <typename T, int KIND>
-__device__ __forceinline__ void run_tile(const Geom<T> &g, const Sc &s, T *sm, int lane) {
-    using C = Cfg<T>;
-    // vector fast path: both sides 16-byte aligned and every run a whole
-    // number of chunks (the source runs along y when transposing)
-    const int vrun_src = g.transpose ? g.ny : g.nx;
-    const bool fast = g.dvec && g.svec && (g.nx % C::VEC) == 0 && (vrun_src % C::VEC) == 0;
-    if (!fast) tile_general<T, KIND>(g, s, sm, lane);
-    else if (g.transpose) tile_transpose_vec<T, KIND>(g, s, sm, lane);
-    else tile_copy_vec<T, KIND>(g, s, lane);
 }
 
 __device__ __forceinline__ bool aligned16(const void *p, int64_t ld_bytes) {
     return ((reinterpret_cast<uintptr_t>(p) | static_cast<uintptr_t>(ld_bytes)) & 15) == 0;
 }
 
+// The tile with linear id t (or the next one this launch covers), resolved
+// into its geometry and scalars.  Returns false when the warp has no tile
+// left.
 template <typename T, int MODE, int KIND>
-__global__ void __launch_bounds__(kWarps * 32, 2) remap_kernel(const RemapLaunch args) {
+__device__ __forceinline__ bool fetch_tile(const RemapLaunch &args, int64_t &t, int64_t stride,
+                                           Geom<T> &g, Sc &s) {
     using C = Cfg<T>;
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    T *sm = reinterpret_cast<T *>(smem_raw) + warp * C::SMEM_ELEMS;
-    const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kWarps;
-
-    for (int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + warp; t < args.total_tiles;
-         t += nwarps) {
+    for (; t < args.total_tiles; t += stride) {
         int k = 0;
         if (args.nprob > 1) {
             int lo = 0, hi = args.nprob;
@@ -317,12 +295,24 @@ __global__ void __launch_bounds__(kWarps * 32, 2) remap_kernel(const RemapLaunch
             if (MODE == KM_DIRECT_LOCAL ? soff >= 0 : soff < 0) continue;
             stld = P.stage_ld[tl];
         }
+        s.ar = 1.0; s.ai = 0.0; s.br = 0.0; s.bi = 0.0; s.conj_mask = 0u;
+        const int op = P.op;
+        if (MODE != KM_PACK) {
+            Scalars S;
+            if (args.per_problem) {
+                S = args.per_problem[k];
+                if (kind_of(S.flags) != KIND) continue;  // another launch covers it
+            } else {
+                S = args.s;
+            }
+            s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
+            s.conj_mask = (ET<T>::CPLX && op == COSTA_OP_C) ? 0x80000000u : 0u;
+        }
         const int u = static_cast<int>(tl / P.nv);
         const int v = static_cast<int>(tl - static_cast<int64_t>(u) * P.nv);
         const AxisTile rt = P.rows[u];
         const AxisTile ct = P.cols[v];
         const DevBlock dA = P.descA[static_cast<int64_t>(rt.a_blk) * P.nbcA + ct.a_blk];
-        const int op = P.op;
         const DevBlock dB = op == COSTA_OP_N
                                 ? P.descB[static_cast<int64_t>(rt.b_blk) * P.nbcB + ct.b_blk]
                                 : P.descB[static_cast<int64_t>(ct.b_blk) * P.nbcB + rt.b_blk];
@@ -351,8 +341,6 @@ __global__ void __launch_bounds__(kWarps * 32, 2) remap_kernel(const RemapLaunch
             src = reinterpret_cast<const T *>(args.staging) + soff;
             sld = stld;
         }
-
-        Geom<T> g;
         g.dst = dst;
         g.src = src;
         g.dld = dld;
@@ -360,23 +348,58 @@ __global__ void __launch_bounds__(kWarps * 32, 2) remap_kernel(const RemapLaunch
         g.nx = dst_fast_i ? rt.len : ct.len;
         g.ny = dst_fast_i ? ct.len : rt.len;
         g.transpose = dst_fast_i != src_fast_i;
-        g.dvec = aligned16(dst, dld * static_cast<int64_t>(sizeof(T)));
-        g.svec = aligned16(src, sld * static_cast<int64_t>(sizeof(T)));
-
-        Sc s{1.0, 0.0, 0.0, 0.0, 0u};
-        if (MODE != KM_PACK) {
-            Scalars S;
-            if (args.per_problem) {
-                S = args.per_problem[k];
-                if (kind_of(S.flags) != KIND) continue;  // another launch covers it
-            } else {
-                S = args.s;
-            }
-            s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
-            s.conj_mask = (ET<T>::CPLX && op == COSTA_OP_C) ? 0x80000000u : 0u;
-        }
-        run_tile<T, KIND>(g, s, sm, lane);
+        // vector fast path: both sides 16-byte aligned and every run a whole
+        // number of chunks (the source runs along y when transposing)
+        const int vrun_src = g.transpose ? g.ny : g.nx;
+        g.fast = aligned16(dst, dld * static_cast<int64_t>(sizeof(T))) &&
+                 aligned16(src, sld * static_cast<int64_t>(sizeof(T))) && (g.nx % C::VEC) == 0 &&
+                 (vrun_src % C::VEC) == 0;
+        return true;
     }
+    return false;
+}
+
+template <typename T, int MODE, int KIND>
+__global__ void __launch_bounds__(kWarps * 32, kMinBlocks) remap_kernel(const RemapLaunch args) {
+    using C = Cfg<T>;
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char *bufs = smem_raw + warp * 2 * C::BUF_BYTES;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * kWarps;
+
+    int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
+    Geom<T> g;
+    Sc s;
+    bool have = fetch_tile<T, MODE, KIND>(args, t, stride, g, s);
+    if (have && g.fast) stage_issue<T>(g, bufs, lane);
+    cp_async_commit();
+    int cur = 0;
+    while (have) {
+        // prefetch: resolve the next tile and start its copies
+        int64_t tn = t + stride;
+        Geom<T> gn;
+        Sc sn;
+        const bool have_n = fetch_tile<T, MODE, KIND>(args, tn, stride, gn, sn);
+        unsigned char *buf = bufs + cur * C::BUF_BYTES;
+        if (have_n && gn.fast) stage_issue<T>(gn, bufs + (cur ^ 1) * C::BUF_BYTES, lane);
+        cp_async_commit();
+        if (g.fast) {
+            Chunk<T> av[C::NPASS];
+            load_a<T, KIND>(g, av, lane);
+            cp_async_wait_1();  // this tile's copies (the next tile's may still fly)
+            __syncwarp();
+            stage_drain<T, KIND>(g, s, buf, av, lane);
+        } else {
+            tile_general<T, KIND>(g, s, buf, lane);
+        }
+        __syncwarp();  // the buffer is free before it is staged into again
+        g = gn;
+        s = sn;
+        t = tn;
+        have = have_n;
+        cur ^= 1;
+    }
+    cp_async_wait_0();
 }
 
 inline int sm_count() {
@@ -393,7 +416,7 @@ inline int sm_count() {
 template <typename T, int MODE, int KIND>
 cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     auto kern = remap_kernel<T, MODE, KIND>;
-    const size_t smem = static_cast<size_t>(kWarps) * Cfg<T>::SMEM_ELEMS * sizeof(T);
+    const size_t smem = static_cast<size_t>(kWarps) * 2 * Cfg<T>::BUF_BYTES;
     static int per_sm = 0;
     if (per_sm == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -423,7 +446,7 @@ cudaError_t launch_remap_t(const RemapLaunch &a, int mode, int kind, cudaStream_
     case K_SCALE: return launch_t<T, MODE, K_SCALE>(a, st);                       \
     case K_AXPBY: return launch_t<T, MODE, K_AXPBY>(a, st);                       \
     default:                                                                      \
-        if (ET<T>::CPLX) return launch_t<T, MODE, K_CPLX>(a, st);                 \
+        if constexpr (ET<T>::CPLX) return launch_t<T, MODE, K_CPLX>(a, st);       \
         return cudaErrorInvalidValue;                                             \
     }
     switch (mode) {
