@@ -59,6 +59,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--small", action="store_true",
+                    help="same layouts at about 1 GB (for profiler captures only)")
     return ap.parse_args()
 
 
@@ -152,8 +154,8 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm), "window": window}
 
 
-def problems(workload):
-    p = C.CONFIGS[workload]()
+def problems(workload, small=False):
+    p = (C.CONFIGS_SMALL if small else C.CONFIGS)[workload]()
     return p if isinstance(p, list) else [p]
 
 
@@ -171,7 +173,7 @@ def run_gpu(args, rank, world, local_rank):
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    probs = problems(args.workload)
+    probs = problems(args.workload, args.small)
     mats = []
     for p in probs:
         Bd = DeviceMatrix(p.B, p.dtype, dev).fill(p.b_kind, p.seed, p.src_stream)
@@ -328,7 +330,10 @@ def run_cpu_oracle(args, probs, seconds_target: float):
 def workload_config(args, probs, world):
     p = probs[0]
     nbytes = algorithmic_bytes(probs)
-    return {"workload": f"{args.workload}: {C.WORKLOAD_TEXT[args.workload]}",
+    text = C.WORKLOAD_TEXT[args.workload]
+    if args.small:
+        text = f"{args.workload} layouts at reduced size ({p.A.m}x{p.A.n} per instance)"
+    return {"workload": f"{args.workload}: {text}",
             "dtype": p.dtype, "op": p.op, "alpha": str(p.alpha), "beta": str(p.beta),
             "P": p.A.nranks, "instances": len(probs), "relabel": True, "mode": args.mode,
             "bytes_per_step_per_gpu": nbytes,
@@ -342,7 +347,7 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    probs = problems(args.workload)
+    probs = problems(args.workload, args.small)
 
     if args.impl == "reference":
         if rank != 0:

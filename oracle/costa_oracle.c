@@ -112,8 +112,13 @@ static double dot2(int n, const double *x, const double *y) {
     return p + s;
 }
 
-/* Sum of n products of doubles, the exact value rounded (nearly) once. */
+/* Sum of n products of doubles, the exact value rounded (nearly) once.
+   Non-finite inputs or an overflowing sum follow plain IEEE evaluation of
+   the expression (the error-free transformations would turn inf into NaN). */
 static double sum_products(int single, int n, const double *x, const double *y) {
+    double plain = 0.0;
+    for (int k = 0; k < n; k++) plain += x[k] * y[k];
+    if (!isfinite(plain)) return plain;
     if (single) {
         /* float data: products are exact in double, the double sum is within
            2^-53 relative, then one rounding to float by the caller */

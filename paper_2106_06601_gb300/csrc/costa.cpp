@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <atomic>
 #include <chrono>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -491,6 +492,12 @@ Scalars make_scalars(int dt, const void *alpha, const void *beta, int index) {
     if (s.beta[0] == 0.0 && s.beta[1] == 0.0) s.flags |= SF_BETA0;
     if (s.alpha[0] == 1.0 && s.alpha[1] == 0.0) s.flags |= SF_ALPHA1;
     if (s.alpha[1] != 0.0 || s.beta[1] != 0.0) s.flags |= SF_CPLX;
+    int e = 0;
+    const double fr = std::frexp(std::fabs(s.beta[0]), &e);
+    if (s.beta[1] == 0.0 && fr == 0.5 && e - 1 >= -1000 && e - 1 <= 1000) {
+        s.flags |= SF_BPOW2;  // |beta| = 2^(e-1)
+        s.beta_exp = e - 1;
+    }
     return s;
 }
 
@@ -550,10 +557,10 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         L.per_problem = plan->d_scalars;
     }
     // one launch per combine kind present in the batch
-    bool kinds[4] = {false, false, false, false};
+    bool kinds[K_NKINDS] = {};
     for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
     auto launch_all = [&](int km) -> cudaError_t {
-        for (int kind = 0; kind < 4; ++kind) {
+        for (int kind = 0; kind < K_NKINDS; ++kind) {
             if (!kinds[kind]) continue;
             cudaError_t e = launch_remap(L, km, kind, stream);
             if (e != cudaSuccess) return e;

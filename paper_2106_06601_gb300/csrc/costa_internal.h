@@ -84,9 +84,9 @@ struct Scalars {
     double alpha[2];
     double beta[2];
     int32_t flags;
-    int32_t pad;
+    int32_t beta_exp;  // k with |beta| = 2^k when SF_BPOW2 is set
 };
-enum : int32_t { SF_BETA0 = 1, SF_ALPHA1 = 2, SF_CPLX = 4 };
+enum : int32_t { SF_BETA0 = 1, SF_ALPHA1 = 2, SF_CPLX = 4, SF_BPOW2 = 8 };
 
 // Combine kinds: each kernel is compiled for one, so every path keeps only
 // the registers it needs.
@@ -94,11 +94,14 @@ enum : int32_t { SF_BETA0 = 1, SF_ALPHA1 = 2, SF_CPLX = 4 };
 //   K_SCALE real alpha, beta = 0       out = alpha * op(b)
 //   K_AXPBY real alpha, beta != 0      out = fma(alpha, op(b), beta * a)
 //   K_CPLX  complex alpha or beta      complex products as chains of fma
-enum : int { K_COPY = 0, K_SCALE = 1, K_AXPBY = 2, K_CPLX = 3 };
+//   K_AXPBY2 as K_AXPBY with beta = +-2^k: beta * a is formed exactly on the
+//            integer pipes (exponent add), saving one multiply on the scarce
+//            FP64 pipe; same bits as K_AXPBY
+enum : int { K_COPY = 0, K_SCALE = 1, K_AXPBY = 2, K_CPLX = 3, K_AXPBY2 = 4, K_NKINDS = 5 };
 
 COSTA_HD inline int kind_of(int32_t flags) {
     if (flags & SF_CPLX) return K_CPLX;
-    if (!(flags & SF_BETA0)) return K_AXPBY;
+    if (!(flags & SF_BETA0)) return (flags & SF_BPOW2) ? K_AXPBY2 : K_AXPBY;
     if (!(flags & SF_ALPHA1)) return K_SCALE;
     return K_COPY;
 }

@@ -104,14 +104,21 @@ __device__ __forceinline__ double fmar(double a, double b, double c) { return __
 struct Sc {
     double ar, ai, br, bi;
     uint32_t conj_mask;  // 0x80000000 flips the sign of b's imaginary part (op = C)
+    int32_t bexp;        // |beta| = 2^bexp (K_AXPBY2)
+    uint32_t bsign_hi;   // sign bit of beta in a high word (K_AXPBY2)
+    uint32_t p2_add;     // bexp << 20: exponent increment in a high word
+    uint32_t p2_lo;      // admissible biased exponents: p2_lo + [0, p2_span]
+    uint32_t p2_span;
 };
 
 // Combine of one element for a kind K_* (costa_internal.h); the kernel is
-// compiled per kind.  b arrives conjugated (op = C) via conj_mask.
+// compiled per kind.  b arrives conjugated (op = C) via conj_mask; for
+// K_AXPBY2, a arrives already multiplied by beta (exactly, see prescale).
 template <int KIND, typename R>
 __device__ __forceinline__ R comb_real(R b, R a, const Sc &s) {
     if (KIND == K_COPY) return b;
     if (KIND == K_SCALE) return mulr(R(s.ar), b);
+    if (KIND == K_AXPBY2) return fmar(R(s.ar), b, a);  // a arrives multiplied by beta
     return fmar(R(s.ar), b, mulr(R(s.br), a));
 }
 
@@ -180,17 +187,136 @@ __device__ __forceinline__ unsigned char *slot(unsigned char *buf, int r, int c)
     return buf + (r * Cfg<T>::CPR + (c ^ swz<T>(r))) * 16;
 }
 
+// Lane mapping for runs of `chunks` 16-byte chunks (1 <= chunks <= CPR):
+// lpr = the next power of two >= chunks lanes per run, 32 / lpr runs per warp
+// pass.  Narrow tiles thus keep all lanes busy instead of leaving the lanes
+// beyond the run idle.
+struct LaneMap {
+    int c;    // chunk of this lane within its run
+    int r0;   // run of this lane in pass 0
+    int rpp;  // runs per pass
+};
+__device__ __forceinline__ LaneMap lane_map(int chunks, int lane) {
+    const int sh = chunks <= 1 ? 0 : 32 - __clz(chunks - 1);
+    LaneMap m;
+    m.c = lane & ((1 << sh) - 1);
+    m.r0 = lane >> sh;
+    m.rpp = 32 >> sh;
+    return m;
+}
+
 // Issue the cp.async copies of a fast tile's source into `buf`.
 template <typename T>
 __device__ __forceinline__ void stage_issue(const Geom<T> &g, unsigned char *buf, int lane) {
     using C = Cfg<T>;
-    const int runs = g.transpose ? g.nx : g.ny;            // source runs
+    const int runs = g.transpose ? g.nx : g.ny;               // source runs
     const int chunks = (g.transpose ? g.ny : g.nx) / C::VEC;  // chunks per run
-    const int c = lane % C::CPR, r0 = lane / C::CPR;
-    if (c >= chunks) return;
+    const LaneMap m = lane_map(chunks, lane);
+    if (m.c >= chunks) return;
 #pragma unroll 4
-    for (int r = r0; r < runs; r += C::RPP)
-        cp_async16(slot<T>(buf, r, c), g.src + static_cast<int64_t>(r) * g.sld + c * C::VEC);
+    for (int r = m.r0; r < runs; r += m.rpp)
+        cp_async16(slot<T>(buf, r, m.c), g.src + static_cast<int64_t>(r) * g.sld + m.c * C::VEC);
+}
+
+// beta * a for beta = +-2^k without the FP64 pipe.  For a zero or a normal a
+// whose biased exponent e stays in [1, 2046] after adding k, the product is
+// exact: a's high word with k added to the exponent field (zeros unchanged)
+// and the sign flipped for negative beta.  Sc holds the admissible exponent
+// range as p2_lo + [0, p2_span].  `bad` collects the other cases
+// (subnormals, infinities, NaNs, products leaving the normal range), which
+// the multiply handles.
+__device__ __forceinline__ bool pow2_bad(double a, const Sc &s) {
+    const unsigned hi = static_cast<unsigned>(__double2hiint(a));
+    const unsigned lo = static_cast<unsigned>(__double2loint(a));
+    const unsigned e = (hi >> 20) & 0x7FFu;
+    const bool zero = ((hi & 0x7FFFFFFFu) | lo) == 0u;
+    return !zero && (e - s.p2_lo) > s.p2_span;
+}
+__device__ __forceinline__ double pow2_apply(double a, const Sc &s) {
+    const unsigned hi = static_cast<unsigned>(__double2hiint(a));
+    const unsigned lo = static_cast<unsigned>(__double2loint(a));
+    const unsigned nh = (hi & 0x7FF00000u) ? hi + s.p2_add : hi;  // zeros keep their exponent
+    return __hiloint2double(static_cast<int>(nh ^ s.bsign_hi), static_cast<int>(lo));
+}
+
+// Scales the loaded A chunks (the first `npass` passes) by beta in place for
+// kind K_AXPBY2.  Double data takes the exact integer path unless some lane
+// of the warp holds a value it does not cover; that choice is one warp vote,
+// so the scarce FP64 pipe never runs predicated-off multiplies.  beta = +-1
+// needs at most a sign flip.  Float data multiplies (the FP32 pipe is wide).
+template <typename T>
+__device__ __forceinline__ void prescale(Chunk<T> (&av)[Cfg<T>::NPASS], int npass, const Sc &s) {
+    using C = Cfg<T>;
+    using R = typename ET<T>::R;
+    constexpr int PER = 16 / static_cast<int>(sizeof(R));  // reals per chunk
+    if constexpr (sizeof(R) == 8) {
+        if (s.bexp == 0) {
+            if (s.bsign_hi) {
+#pragma unroll
+                for (int p = 0; p < C::NPASS; ++p) {
+                    if (p >= npass) break;
+                    av[p].raw.y ^= s.bsign_hi;
+                    av[p].raw.w ^= s.bsign_hi;
+                }
+            }
+            return;
+        }
+        bool bad = false;
+#pragma unroll
+        for (int p = 0; p < C::NPASS; ++p) {
+            if (p >= npass) break;
+            const double *v = reinterpret_cast<const double *>(&av[p]);
+#pragma unroll
+            for (int k = 0; k < PER; ++k) bad |= pow2_bad(v[k], s);
+        }
+        if (__any_sync(0xffffffffu, bad)) {
+#pragma unroll
+            for (int p = 0; p < C::NPASS; ++p) {
+                if (p >= npass) break;
+                double *v = reinterpret_cast<double *>(&av[p]);
+#pragma unroll
+                for (int k = 0; k < PER; ++k) v[k] = __dmul_rn(s.br, v[k]);
+            }
+        } else {
+#pragma unroll
+            for (int p = 0; p < C::NPASS; ++p) {
+                if (p >= npass) break;
+                double *v = reinterpret_cast<double *>(&av[p]);
+#pragma unroll
+                for (int k = 0; k < PER; ++k) v[k] = pow2_apply(v[k], s);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int p = 0; p < C::NPASS; ++p) {
+            if (p >= npass) break;
+            float *v = reinterpret_cast<float *>(&av[p]);
+#pragma unroll
+            for (int k = 0; k < PER; ++k) v[k] = __fmul_rn(float(s.br), v[k]);
+        }
+    }
+}
+
+// Loads the tile's A chunks (kinds that read A) in the drain's lane mapping.
+// Called by all 32 lanes (prescale votes).
+template <typename T, int KIND>
+__device__ __forceinline__ void load_a(const Geom<T> &g, const Sc &s, Chunk<T> (&av)[Cfg<T>::NPASS],
+                                       int lane) {
+    using C = Cfg<T>;
+    if (KIND == K_COPY || KIND == K_SCALE) return;
+    const int chunks = g.nx / C::VEC;
+    const LaneMap m = lane_map(chunks, lane);
+    const int x0 = m.c * C::VEC;
+    const bool on = m.c < chunks;
+    const int npass = (g.ny + m.rpp - 1) / m.rpp;
+#pragma unroll
+    for (int p = 0; p < C::NPASS; ++p) {
+        if (p >= npass) break;  // uniform across the warp
+        const int y = p * m.rpp + m.r0;
+        av[p].raw = make_uint4(0, 0, 0, 0);
+        if (on && y < g.ny) av[p] = load_rw(g.dst + static_cast<int64_t>(y) * g.dld + x0);
+    }
+    if (KIND == K_AXPBY2) prescale<T>(av, npass, s);
 }
 
 // Write a staged fast tile to A, combining with A when the kind reads it.
@@ -198,11 +324,15 @@ template <typename T, int KIND>
 __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsigned char *buf,
                                             const Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
     using C = Cfg<T>;
-    const int c = lane % C::CPR, yr = lane / C::CPR, x0 = c * C::VEC;
-    if (x0 >= g.nx) return;
+    const int chunks = g.nx / C::VEC;
+    const LaneMap m = lane_map(chunks, lane);
+    if (m.c >= chunks) return;
+    const int x0 = m.c * C::VEC;
+    const int npass = (g.ny + m.rpp - 1) / m.rpp;
 #pragma unroll
     for (int p = 0; p < C::NPASS; ++p) {
-        const int y = p * C::RPP + yr;
+        if (p >= npass) break;  // uniform across the warp
+        const int y = p * m.rpp + m.r0;
         if (y < g.ny) {
             Chunk<T> b;
             if (g.transpose) {
@@ -212,7 +342,7 @@ __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsig
                 for (int e = 0; e < C::VEC; ++e)
                     b.e[e] = reinterpret_cast<const T *>(slot<T>(buf, x0 + e, cy))[ey];
             } else {
-                b.raw = *reinterpret_cast<const uint4 *>(slot<T>(buf, y, c));
+                b.raw = *reinterpret_cast<const uint4 *>(slot<T>(buf, y, m.c));
             }
             Chunk<T> o;
 #pragma unroll
@@ -222,17 +352,19 @@ __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsig
     }
 }
 
-template <typename T, int KIND>
-__device__ __forceinline__ void load_a(const Geom<T> &g, Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
-    using C = Cfg<T>;
-    const int c = lane % C::CPR, yr = lane / C::CPR, x0 = c * C::VEC;
-#pragma unroll
-    for (int p = 0; p < C::NPASS; ++p) {
-        av[p].raw = make_uint4(0, 0, 0, 0);
-        const int y = p * C::RPP + yr;
-        if (KIND >= K_AXPBY && x0 < g.nx && y < g.ny)
-            av[p] = load_rw(g.dst + static_cast<int64_t>(y) * g.dld + x0);
-    }
+// K_AXPBY2 takes a multiplied by beta (a power of two: exact); other kinds
+// take a as it is.
+template <int KIND> __device__ __forceinline__ float premul(float a, const Sc &s) {
+    return KIND == K_AXPBY2 ? __fmul_rn(float(s.br), a) : a;
+}
+template <int KIND> __device__ __forceinline__ double premul(double a, const Sc &s) {
+    return KIND == K_AXPBY2 ? __dmul_rn(s.br, a) : a;
+}
+template <int KIND> __device__ __forceinline__ float2 premul(float2 a, const Sc &s) {
+    return KIND == K_AXPBY2 ? make_float2(__fmul_rn(float(s.br), a.x), __fmul_rn(float(s.br), a.y)) : a;
+}
+template <int KIND> __device__ __forceinline__ double2 premul(double2 a, const Sc &s) {
+    return KIND == K_AXPBY2 ? make_double2(__dmul_rn(s.br, a.x), __dmul_rn(s.br, a.y)) : a;
 }
 
 // Element-wise path for ragged or misaligned tiles, lanes strided along the
@@ -240,14 +372,14 @@ __device__ __forceinline__ void load_a(const Geom<T> &g, Chunk<T> (&av)[Cfg<T>::
 template <typename T, int KIND>
 __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
     using C = Cfg<T>;
-    constexpr bool READ_A = KIND >= K_AXPBY;
+    constexpr bool READ_A = KIND != K_COPY && KIND != K_SCALE;
     T *sm = reinterpret_cast<T *>(buf);
     const int n = g.nx * g.ny;
     if (!g.transpose) {
         for (int k = lane; k < n; k += 32) {
             const int y = k / g.nx, x = k - y * g.nx;
             T *d = g.dst + static_cast<int64_t>(y) * g.dld + x;
-            const T a = READ_A ? *d : T();
+            const T a = READ_A ? premul<KIND>(*d, s) : T();
             *d = combine<KIND>(__ldg(g.src + static_cast<int64_t>(y) * g.sld + x), a, s);
         }
         return;
@@ -260,7 +392,7 @@ __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsi
     for (int k = lane; k < n; k += 32) {
         const int y = k / g.nx, x = k - y * g.nx;
         T *d = g.dst + static_cast<int64_t>(y) * g.dld + x;
-        const T a = READ_A ? *d : T();
+        const T a = READ_A ? premul<KIND>(*d, s) : T();
         *d = combine<KIND>(sm[y * C::PITCH + x], a, s);
     }
 }
@@ -295,7 +427,8 @@ __device__ __forceinline__ bool fetch_tile(const RemapLaunch &args, int64_t &t, 
             if (MODE == KM_DIRECT_LOCAL ? soff >= 0 : soff < 0) continue;
             stld = P.stage_ld[tl];
         }
-        s.ar = 1.0; s.ai = 0.0; s.br = 0.0; s.bi = 0.0; s.conj_mask = 0u;
+        s.ar = 1.0; s.ai = 0.0; s.br = 0.0; s.bi = 0.0; s.conj_mask = 0u; s.bexp = 0; s.bsign_hi = 0u;
+        s.p2_add = 0u; s.p2_lo = 1u; s.p2_span = 0u;
         const int op = P.op;
         if (MODE != KM_PACK) {
             Scalars S;
@@ -306,6 +439,15 @@ __device__ __forceinline__ bool fetch_tile(const RemapLaunch &args, int64_t &t, 
                 S = args.s;
             }
             s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
+            s.bexp = S.beta_exp;
+            s.bsign_hi = static_cast<unsigned>(__double2hiint(S.beta[0])) & 0x80000000u;
+            s.p2_add = static_cast<unsigned>(S.beta_exp) << 20;
+            {   // e in [1, 2046] and e + k in [1, 2046]
+                const int lo = max(1, 1 - S.beta_exp), hi = min(2046, 2046 - S.beta_exp);
+                s.p2_lo = static_cast<unsigned>(lo);
+                s.p2_span = hi >= lo ? static_cast<unsigned>(hi - lo) : 0u;
+                if (hi < lo) s.p2_lo = 4096u;  // nothing admissible: always multiply
+            }
             s.conj_mask = (ET<T>::CPLX && op == COSTA_OP_C) ? 0x80000000u : 0u;
         }
         const int u = static_cast<int>(tl / P.nv);
@@ -385,7 +527,7 @@ __global__ void __launch_bounds__(kWarps * 32, kMinBlocks) remap_kernel(const Re
         cp_async_commit();
         if (g.fast) {
             Chunk<T> av[C::NPASS];
-            load_a<T, KIND>(g, av, lane);
+            load_a<T, KIND>(g, s, av, lane);
             cp_async_wait_1();  // this tile's copies (the next tile's may still fly)
             __syncwarp();
             stage_drain<T, KIND>(g, s, buf, av, lane);
@@ -445,6 +587,7 @@ cudaError_t launch_remap_t(const RemapLaunch &a, int mode, int kind, cudaStream_
     case K_COPY: return launch_t<T, MODE, K_COPY>(a, st);                         \
     case K_SCALE: return launch_t<T, MODE, K_SCALE>(a, st);                       \
     case K_AXPBY: return launch_t<T, MODE, K_AXPBY>(a, st);                       \
+    case K_AXPBY2: return launch_t<T, MODE, K_AXPBY2>(a, st);                     \
     default:                                                                      \
         if constexpr (ET<T>::CPLX) return launch_t<T, MODE, K_CPLX>(a, st);       \
         return cudaErrorInvalidValue;                                             \

@@ -183,3 +183,41 @@ def test_batched_matches_oracle(dev):
     finally:
         for g in gs:
             g.close()
+
+
+@pytest.mark.parametrize("dtype", ["f64", "c128", "f32"])
+@pytest.mark.parametrize("beta", [0.5, 2.0, -0.25, 1.0, 2.0 ** -1000])
+def test_special_values_power_of_two_beta(dtype, beta, dev):
+    """beta * a formed on the integer pipes must equal the multiply for zeros,
+    subnormals, infinities and NaNs, and when beta * a underflows below the
+    normal range.  (Values stay below max/4 so that alpha * b and beta * a do
+    not overflow: the kernel rounds beta * a before its fma, and an overflow
+    there is that formula's result, not the exact one.)"""
+    if dtype == "f32" and beta == 2.0 ** -1000:
+        pytest.skip("beta is not representable in float")
+    rng = np.random.default_rng(5)
+    B = L.block_cyclic(64, 48, 16, 16, 2, 2)
+    A = L.block_cyclic(48, 64, 8, 32, 2, 2, storage="C")
+    p = C.Problem("special", dtype, "T", 2.0, beta, A, B, "uniform", "uniform", C.SEED0)
+    g = OnDevice(p, dev)
+    try:
+        real = np.float64 if dtype in ("f64", "c128") else np.float32
+        fi = np.finfo(real)
+        specials = np.array([0.0, -0.0, fi.tiny, -fi.tiny, fi.tiny / 4, -fi.smallest_subnormal,
+                             fi.max / 4, -fi.max / 5, np.inf, -np.inf, np.nan, 1.5, -3.0,
+                             fi.tiny * 2, fi.max / 8, 1e-300 if real is np.float64 else 1e-30],
+                            dtype=real)
+        for h in (g.Ah, g.Bh):
+            v = h.arena.view(real) if dtype in ("c128",) else h.arena.view(real)
+            idx = rng.integers(0, v.size, v.size // 3)
+            v[idx] = specials[rng.integers(0, specials.size, idx.size)]
+        g.Bd.upload(g.Bh)
+        g.Ad.upload(g.Ah)
+        g.run(relabel=False)
+        got = g.Ad.download()
+        want = g.oracle_result()
+        if np.frexp(abs(beta))[0] == 0.5:
+            ok = (got.arena == want.arena) | (np.isnan(got.arena) & np.isnan(want.arena))
+            assert np.all(ok), (np.flatnonzero(~ok)[:5], got.arena[~ok][:5], want.arena[~ok][:5])
+    finally:
+        g.close()

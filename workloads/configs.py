@@ -119,6 +119,11 @@ def c5(rows: int = 131072, cols: int = 4096) -> Problem:
 
 CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5}
 
+# The same layouts and tile shapes at about 1 GB on the device, for profiler
+# captures (the workloads proper stay the ones above).
+CONFIGS_SMALL = {"c1": c1, "c2": lambda: c2(4096), "c3": lambda: c3(8192),
+                 "c4": lambda: c4(16), "c5": lambda: c5(rows=16384)}
+
 WORKLOAD_TEXT = {
     "c1": "256x256 f64 BC16 2x2R -> BC32 2x2C, N, alpha=1 beta=0, P=4",
     "c2": "8192x8192 f64 BC64 4x4 -> BC128 4x4 permuted owners, T, alpha=2 beta=0.5, P=16",
