@@ -240,6 +240,15 @@ costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op
 costa_status costa_volume_noalloc(costa_layout A, costa_layout B, costa_op op, int64_t *V,
                                   void *stream);
 
+/* Diagnostics (host only, no device work): the remap kernel's tile list for
+ * (A, B, op) in direct mode.  Each tile is 32 bytes: {source address, target
+ * address (uint64), source stride, target stride (int32), nx, ny, problem,
+ * flags (uint16)}, in the frame where x runs along A's contiguous axis
+ * (flags: 1 = transposed, 2 = vector path, 4 = conjugate).  Writes
+ * min(*count, cap) tiles to out (32 * cap bytes) and the total to *count. */
+costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void *out, int64_t cap,
+                               int64_t *count);
+
 /* Frees every cached plan (synchronizes the device). */
 costa_status costa_release_plans(void);
 

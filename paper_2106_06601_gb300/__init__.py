@@ -71,6 +71,7 @@ def _load():
         "costa_plan_stats_get": [I, P, P, P, I, P, P],
         "costa_release_plans": [],
         "costa_debug_axis_pieces": [P, P, I, I, P, I64, P],
+        "costa_debug_tiles": [P, P, I, P, I64, P],
     }
     for name, args in sigs.items():
         f = getattr(lib, name)
@@ -279,4 +280,19 @@ def costa_debug_axis_pieces(A: Layout, B: Layout, op: str, axis: int) -> np.ndar
     out = np.zeros((max(1, cnt.value), 6), dtype=np.int32)
     _check(_lib.costa_debug_axis_pieces(A.handle, B.handle, OPS[op], axis, _p(out), cnt.value,
                                         ctypes.byref(cnt)))
+    return out[:cnt.value]
+
+
+TILE_DTYPE = np.dtype([("src", np.uint64), ("dst", np.uint64), ("sld", np.int32),
+                       ("dld", np.int32), ("nx", np.uint16), ("ny", np.uint16),
+                       ("prob", np.uint16), ("flags", np.uint16)])
+
+
+def costa_debug_tiles(A: Layout, B: Layout, op: str) -> np.ndarray:
+    """The direct-mode tile list of (A, B, op) as a structured array."""
+    cnt = ctypes.c_int64()
+    _check(_lib.costa_debug_tiles(A.handle, B.handle, OPS[op], None, 0, ctypes.byref(cnt)))
+    out = np.zeros(max(1, cnt.value), dtype=TILE_DTYPE)
+    _check(_lib.costa_debug_tiles(A.handle, B.handle, OPS[op], out.ctypes.data, cnt.value,
+                                  ctypes.byref(cnt)))
     return out[:cnt.value]

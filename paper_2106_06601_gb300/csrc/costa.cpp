@@ -68,11 +68,13 @@ struct AxisCut {
     std::vector<AxisTile> tiles;
 };
 
-// Cuts one axis.  The pieces of an interval are aligned to `align_a` (true:
-// multiples of ts from the start of A's block, else of op(B)'s block), so
-// that the side whose contiguous axis this is gets 16-byte aligned runs.
+// Cuts one axis into pieces of at most ts elements.  When an interval starts
+// off a 16-byte boundary (vec elements) of the side chosen by `align_a`
+// (A's block if true, else op(B)'s), one short first piece reaches the
+// boundary, so that the remaining pieces start aligned and can use vector
+// accesses; otherwise the pieces are ts long from the interval's start.
 AxisCut cut_axis(const std::vector<int64_t> &SA, const std::vector<int64_t> &SB, int64_t extent,
-                 int ts, bool align_a) {
+                 int ts, int vec, bool align_a) {
     AxisCut out;
     const int nA = static_cast<int>(SA.size()) - 1, nB = static_cast<int>(SB.size()) - 1;
     int ka = 0, kb = 0;
@@ -86,9 +88,10 @@ AxisCut cut_axis(const std::vector<int64_t> &SA, const std::vector<int64_t> &SB,
         out.intervals.push_back(Interval{ka, kb, len});
         const int64_t a0 = pos - SA[ka], b0 = pos - SB[kb];
         int64_t q = 0;
+        const int64_t phase = (align_a ? a0 : b0) % vec;
         while (q < len) {
-            const int64_t phase = (align_a ? a0 + q : b0 + q) % ts;
-            const int64_t piece = std::min<int64_t>(ts - phase, len - q);
+            const int64_t want = (q == 0 && phase != 0) ? vec - phase : ts;
+            const int64_t piece = std::min<int64_t>(want, len - q);
             out.tiles.push_back(AxisTile{ka, kb, static_cast<int32_t>(a0 + q),
                                          static_cast<int32_t>(b0 + q),
                                          static_cast<int32_t>(piece), cell});
@@ -105,11 +108,12 @@ AxisCut cut_axis(const std::vector<int64_t> &SA, const std::vector<int64_t> &SB,
 // start on 16-byte boundaries.
 AxisCut cut_pair_axis(const costa_layout_s *A, const costa_layout_s *B, int op, int axis, int ts) {
     const bool tr = op != COSTA_OP_N;
+    const int vec = 16 / esize_of(A->dt);
     const bool a_rows_fast = A->blocks.empty() || A->blocks[0].order == COSTA_COL_MAJOR;
     const bool b_col = B->blocks.empty() || B->blocks[0].order == COSTA_COL_MAJOR;
     const bool b_rows_fast = tr ? !b_col : b_col;  // op(B)'s contiguous axis is rows
-    if (axis == 0) return cut_axis(A->R, tr ? B->C : B->R, A->m, ts, a_rows_fast || !b_rows_fast);
-    return cut_axis(A->C, tr ? B->R : B->C, A->n, ts, !a_rows_fast || b_rows_fast);
+    if (axis == 0) return cut_axis(A->R, tr ? B->C : B->R, A->m, ts, vec, a_rows_fast || !b_rows_fast);
+    return cut_axis(A->C, tr ? B->R : B->C, A->n, ts, vec, !a_rows_fast || b_rows_fast);
 }
 
 struct ProblemHost {
@@ -136,11 +140,11 @@ struct Arena {
 
 struct MessageData {
     bool built = false;
-    void *d_mem = nullptr;       // stage_off, stage_ld, ProblemDev[]
-    ProblemDev *d_probs = nullptr;
+    void *d_mem = nullptr;       // pack, local and unpack tile lists
+    const TileDesc *pack = nullptr, *local = nullptr, *unpack = nullptr;
+    int64_t n_pack = 0, n_local = 0, n_unpack = 0;
     void *d_staging = nullptr;
     int64_t staging_bytes = 0;
-    int64_t remote_tiles = 0;
 };
 
 struct Plan {
@@ -148,8 +152,7 @@ struct Plan {
     int dtype = 0, esize = 0, P = 0, ts = 32;
     std::vector<ProblemHost> probs;
     void *d_mem = nullptr;
-    ProblemDev *d_probs = nullptr;
-    std::vector<ProblemDev> h_probs;
+    const TileDesc *d_tiles = nullptr;  // the direct list
     Scalars *d_scalars = nullptr;
     std::vector<Scalars> cached_scalars;
     int64_t total_tiles = 0, total_cells = 0;
@@ -210,22 +213,80 @@ costa_status validate_pair(const costa_layout_s *A, const costa_layout_s *B, int
     return COSTA_OK;
 }
 
-// Builds the overlay, tiles and device tables, and runs the volume kernel.
+bool aligned16(uint64_t addr, int64_t ld_bytes) { return ((addr | static_cast<uint64_t>(ld_bytes)) & 15) == 0; }
+
+// The tile (rt, ct) of a problem in the kernel's canonical frame (x = A's
+// contiguous axis): source and target addresses of element (0, 0), strides,
+// extents, and whether source and target runs lie on different axes.
+TileDesc direct_tile(const ProblemHost &ph, const AxisTile &rt, const AxisTile &ct, int es, int prob) {
+    const DevBlock &dA = ph.A->blocks[static_cast<size_t>(rt.a_blk) * ph.A->nbc + ct.a_blk];
+    const bool tr = ph.op != COSTA_OP_N;
+    const DevBlock &dB = tr ? ph.B->blocks[static_cast<size_t>(ct.b_blk) * ph.B->nbc + rt.b_blk]
+                            : ph.B->blocks[static_cast<size_t>(rt.b_blk) * ph.B->nbc + ct.b_blk];
+    const bool b_col = dB.order == COSTA_COL_MAJOR;
+    const int64_t rb = tr ? ct.b_off : rt.b_off, cb = tr ? rt.b_off : ct.b_off;
+    const bool src_fast_i = tr ? !b_col : b_col;  // source runs along A's rows
+    const bool a_col = dA.order == COSTA_COL_MAJOR;
+    TileDesc d;
+    d.src = dB.ptr + static_cast<uint64_t>((b_col ? rb + cb * dB.ld : rb * dB.ld + cb) * es);
+    d.dst = dA.ptr + static_cast<uint64_t>(
+                         (a_col ? rt.a_off + static_cast<int64_t>(ct.a_off) * dA.ld
+                                : static_cast<int64_t>(rt.a_off) * dA.ld + ct.a_off) * es);
+    d.sld = dB.ld;
+    d.dld = dA.ld;
+    d.nx = static_cast<uint16_t>(a_col ? rt.len : ct.len);
+    d.ny = static_cast<uint16_t>(a_col ? ct.len : rt.len);
+    d.prob = static_cast<uint16_t>(prob);
+    d.flags = 0;
+    if (a_col != src_fast_i) d.flags |= TF_TRANSPOSE;
+    if (ph.op == COSTA_OP_C) d.flags |= TF_CONJ;
+    return d;
+}
+
+// Sets TF_FAST when every run is whole 16-byte chunks on both sides.
+void set_fast(TileDesc &d, int es) {
+    const int vec = 16 / es;
+    const bool tr = (d.flags & TF_TRANSPOSE) != 0;
+    const int src_run = tr ? d.ny : d.nx;
+    const bool fast = aligned16(d.dst, static_cast<int64_t>(d.dld) * es) &&
+                      aligned16(d.src, static_cast<int64_t>(d.sld) * es) && d.nx % vec == 0 &&
+                      src_run % vec == 0;
+    d.flags = static_cast<uint16_t>(fast ? (d.flags | TF_FAST) : (d.flags & ~TF_FAST));
+}
+
+// Visits the tiles of a problem in super-tiles of kSuper x kSuper pieces,
+// row pieces fastest inside each: the tiles that warps work on at the same
+// time then cover compact regions of A and of B (runs of kSuper tiles along
+// both axes) instead of one band of rows across every column.
+constexpr int kSuper = 8;
+
+template <typename F> void for_each_tile(const ProblemHost &ph, F &&f) {
+    const int nu = static_cast<int>(ph.rows.tiles.size()), nv = static_cast<int>(ph.cols.tiles.size());
+    for (int su = 0; su < nu; su += kSuper)
+        for (int sv = 0; sv < nv; sv += kSuper)
+            for (int v = sv; v < std::min(sv + kSuper, nv); ++v)
+                for (int u = su; u < std::min(su + kSuper, nu); ++u) f(ph.rows.tiles[u], ph.cols.tiles[v]);
+}
+
+// Builds the overlay, the tile list and the device tables, and runs the
+// volume kernel.
 costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, const costa_op *ops,
                         cudaStream_t stream, std::unique_ptr<Plan> &out) {
     auto t0 = std::chrono::steady_clock::now();
     auto plan = std::make_unique<Plan>();
     cudaError_t ce = cudaGetDevice(&plan->device);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaGetDevice");
+    if (n > 65535) return fail(COSTA_ERR_INVALID_ARG, "batch of %d exceeds 65535 pairs", n);
     plan->dtype = As[0]->dt;
     plan->esize = esize_of(plan->dtype);
     plan->P = As[0]->nranks;
     plan->ts = tile_extent(plan->esize);
-    const int P = plan->P, ts = plan->ts;
+    const int P = plan->P, ts = plan->ts, es = plan->esize;
 
     Arena arena;
-    struct Off { size_t rows, cols, descA, descB, irows, icols, ownA, ownB; };
+    struct Off { size_t irows, icols, ownA, ownB; };
     std::vector<Off> offs(n);
+    int64_t tiles = 0, cells = 0;
     for (int k = 0; k < n; ++k) {
         ProblemHost ph;
         ph.A = As[k];
@@ -234,19 +295,26 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
         ph.rows = cut_pair_axis(ph.A, ph.B, ph.op, 0, ts);
         ph.cols = cut_pair_axis(ph.A, ph.B, ph.op, 1, ts);
         Off &o = offs[k];
-        o.rows = arena.add_vec(ph.rows.tiles);
-        o.cols = arena.add_vec(ph.cols.tiles);
-        o.descA = arena.add_vec(ph.A->blocks);
-        o.descB = arena.add_vec(ph.B->blocks);
         o.irows = arena.add_vec(ph.rows.intervals);
         o.icols = arena.add_vec(ph.cols.intervals);
         o.ownA = arena.add_vec(ph.A->owner);
         o.ownB = arena.add_vec(ph.B->owner);
+        tiles += static_cast<int64_t>(ph.rows.tiles.size()) * static_cast<int64_t>(ph.cols.tiles.size());
+        cells += static_cast<int64_t>(ph.rows.intervals.size()) * static_cast<int64_t>(ph.cols.intervals.size());
         plan->probs.push_back(std::move(ph));
     }
-    std::vector<ProblemDev> pd(n);
+    // the direct tile list, in (problem, row piece, column piece) order
+    std::vector<TileDesc> list;
+    list.reserve(static_cast<size_t>(tiles));
+    for (int k = 0; k < n; ++k) {
+        for_each_tile(plan->probs[k], [&](const AxisTile &rt, const AxisTile &ct) {
+            TileDesc d = direct_tile(plan->probs[k], rt, ct, es, k);
+            set_fast(d, es);
+            list.push_back(d);
+        });
+    }
+    const size_t off_tiles = arena.add_vec(list);
     std::vector<VolumeProblemDev> vd(n);
-    const size_t off_pd = arena.add(pd.data(), sizeof(ProblemDev) * n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
     std::vector<Scalars> sc(n);
     const size_t off_sc = arena.add(sc.data(), sizeof(Scalars) * n);
@@ -259,46 +327,29 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
                                        cudaGetErrorString(ce));
     plan->d_mem = d;
     char *dbase = static_cast<char *>(d);
-    int64_t tiles = 0, cells = 0;
+    int64_t cell_begin = 0;
     for (int k = 0; k < n; ++k) {
         const ProblemHost &ph = plan->probs[k];
         const Off &o = offs[k];
-        ProblemDev &p = pd[k];
-        p.rows = reinterpret_cast<const AxisTile *>(dbase + o.rows);
-        p.cols = reinterpret_cast<const AxisTile *>(dbase + o.cols);
-        p.descA = reinterpret_cast<const DevBlock *>(dbase + o.descA);
-        p.descB = reinterpret_cast<const DevBlock *>(dbase + o.descB);
-        p.stage_off = nullptr;
-        p.stage_ld = nullptr;
-        p.tile_begin = tiles;
-        p.nu = static_cast<int32_t>(ph.rows.tiles.size());
-        p.nv = static_cast<int32_t>(ph.cols.tiles.size());
-        p.nbcA = ph.A->nbc;
-        p.nbcB = ph.B->nbc;
-        p.op = ph.op;
-        p.pad = 0;
-        tiles += static_cast<int64_t>(p.nu) * p.nv;
         VolumeProblemDev &v = vd[k];
         v.rows = reinterpret_cast<const Interval *>(dbase + o.irows);
         v.cols = reinterpret_cast<const Interval *>(dbase + o.icols);
         v.ownerA = reinterpret_cast<const int32_t *>(dbase + o.ownA);
         v.ownerB = reinterpret_cast<const int32_t *>(dbase + o.ownB);
-        v.cell_begin = cells;
+        v.cell_begin = cell_begin;
         v.nr = static_cast<int32_t>(ph.rows.intervals.size());
         v.nc = static_cast<int32_t>(ph.cols.intervals.size());
         v.nbcA = ph.A->nbc;
         v.nbcB = ph.B->nbc;
         v.op = ph.op;
         v.pad = 0;
-        cells += static_cast<int64_t>(v.nr) * v.nc;
+        cell_begin += static_cast<int64_t>(v.nr) * v.nc;
     }
-    std::memcpy(arena.host.data() + off_pd, pd.data(), sizeof(ProblemDev) * n);
     std::memcpy(arena.host.data() + off_vd, vd.data(), sizeof(VolumeProblemDev) * n);
     ce = cudaMemcpy(d, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(plan tables)");
-    plan->d_probs = reinterpret_cast<ProblemDev *>(dbase + off_pd);
+    plan->d_tiles = reinterpret_cast<const TileDesc *>(dbase + off_tiles);
     plan->d_scalars = reinterpret_cast<Scalars *>(dbase + off_sc);
-    plan->h_probs = pd;
     plan->total_tiles = tiles;
     plan->total_cells = cells;
 
@@ -354,11 +405,12 @@ costa_status ensure_sigma(Plan &plan) {
 // travels through the staging buffer.  Packages are ordered by (p, receiver)
 // at the exclusive-scan offsets of their sizes; inside a package the tiles
 // keep the tile order.  Each staged tile is dense in the source's element
-// order with its leading dimension rounded up to 16 bytes.
+// order with its leading dimension rounded up to 16 bytes.  Three tile lists
+// result: pack (B -> staging), local (B -> A) and unpack (staging -> A).
 costa_status ensure_message(Plan &plan, bool relabel) {
     MessageData &m = plan.msg[relabel ? 1 : 0];
     if (m.built) return COSTA_OK;
-    const int P = plan.P;
+    const int P = plan.P, es = plan.esize;
     std::vector<int> sig(P);
     if (relabel) {
         costa_status s = ensure_sigma(plan);
@@ -367,37 +419,37 @@ costa_status ensure_message(Plan &plan, bool relabel) {
     } else {
         for (int q = 0; q < P; ++q) sig[q] = q;
     }
-    const int vec = 16 / plan.esize;
-    const int64_t T = plan.total_tiles;
-    std::vector<int64_t> stage_off(static_cast<size_t>(std::max<int64_t>(T, 1)), -1);
-    std::vector<int32_t> stage_ld(static_cast<size_t>(std::max<int64_t>(T, 1)), 0);
-    std::vector<int32_t> pkg(static_cast<size_t>(std::max<int64_t>(T, 1)), -1);
+    const int vec = 16 / es;
+    struct Remote { TileDesc d; int32_t pkg; int32_t ld; int64_t size; };
+    std::vector<TileDesc> local;
+    std::vector<Remote> remote;
     std::vector<int64_t> size(static_cast<size_t>(P) * P, 0);
-    int64_t t = 0, remote = 0;
-    for (const ProblemHost &ph : plan.probs) {
+    for (size_t k = 0; k < plan.probs.size(); ++k) {
+        const ProblemHost &ph = plan.probs[k];
         const bool tr = ph.op != COSTA_OP_N;
-        for (const AxisTile &rt : ph.rows.tiles) {
-            for (const AxisTile &ct : ph.cols.tiles) {
+        for_each_tile(ph, [&](const AxisTile &rt, const AxisTile &ct) {
+            {
+                TileDesc d = direct_tile(ph, rt, ct, es, static_cast<int>(k));
                 const int q = ph.A->owner[static_cast<size_t>(rt.a_blk) * ph.A->nbc + ct.a_blk];
                 const size_t bidx = tr ? static_cast<size_t>(ct.b_blk) * ph.B->nbc + rt.b_blk
                                        : static_cast<size_t>(rt.b_blk) * ph.B->nbc + ct.b_blk;
                 const int p = ph.B->owner[bidx];
-                const int r = sig[q];
-                if (p != r) {
-                    const bool b_col = ph.B->blocks[bidx].order == COSTA_COL_MAJOR;
-                    const bool src_fast_i = tr ? !b_col : b_col;
-                    const int fast = src_fast_i ? rt.len : ct.len;
-                    const int other = src_fast_i ? ct.len : rt.len;
-                    const int ld = (fast + vec - 1) / vec * vec;
-                    stage_ld[t] = ld;
-                    pkg[t] = p * P + r;
-                    stage_off[t] = static_cast<int64_t>(ld) * other;  // size for now
-                    size[static_cast<size_t>(p) * P + r] += stage_off[t];
-                    ++remote;
+                if (p == sig[q]) {
+                    set_fast(d, es);
+                    local.push_back(d);
+                    return;
                 }
-                ++t;
+                const bool t = (d.flags & TF_TRANSPOSE) != 0;
+                const int fast = t ? d.ny : d.nx, other = t ? d.nx : d.ny;  // source frame
+                Remote r;
+                r.d = d;
+                r.pkg = p * P + sig[q];
+                r.ld = (fast + vec - 1) / vec * vec;
+                r.size = static_cast<int64_t>(r.ld) * other;
+                size[static_cast<size_t>(r.pkg)] += r.size;
+                remote.push_back(r);
             }
-        }
+        });
     }
     std::vector<int64_t> base(static_cast<size_t>(P) * P, 0);
     int64_t acc = 0;
@@ -405,37 +457,53 @@ costa_status ensure_message(Plan &plan, bool relabel) {
         base[k] = acc;
         acc += size[k];
     }
-    for (int64_t i = 0; i < T; ++i) {
-        if (pkg[i] < 0) continue;
-        const int64_t sz = stage_off[i];
-        stage_off[i] = base[pkg[i]];
-        base[pkg[i]] += sz;
-    }
-    const int n = static_cast<int>(plan.probs.size());
-    Arena arena;
-    const size_t o_off = arena.add_vec(stage_off);
-    const size_t o_ld = arena.add_vec(stage_ld);
-    std::vector<ProblemDev> pd = plan.h_probs;
-    const size_t o_pd = arena.add(pd.data(), sizeof(ProblemDev) * n);
-    cudaError_t ce = cudaMalloc(&m.d_mem, arena.host.size());
-    if (ce != cudaSuccess) return fail(COSTA_ERR_ALLOC, "cudaMalloc(message tables): %s", cudaGetErrorString(ce));
-    char *db = static_cast<char *>(m.d_mem);
-    for (int k = 0; k < n; ++k) {
-        pd[k].stage_off = reinterpret_cast<const int64_t *>(db + o_off) + pd[k].tile_begin;
-        pd[k].stage_ld = reinterpret_cast<const int32_t *>(db + o_ld) + pd[k].tile_begin;
-    }
-    std::memcpy(arena.host.data() + o_pd, pd.data(), sizeof(ProblemDev) * n);
-    ce = cudaMemcpy(m.d_mem, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
-    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(message tables)");
-    m.d_probs = reinterpret_cast<ProblemDev *>(db + o_pd);
-    m.staging_bytes = acc * plan.esize;
+    m.staging_bytes = acc * es;
     if (m.staging_bytes > 0) {
-        ce = cudaMalloc(&m.d_staging, static_cast<size_t>(m.staging_bytes));
+        cudaError_t ce = cudaMalloc(&m.d_staging, static_cast<size_t>(m.staging_bytes));
         if (ce != cudaSuccess)
             return fail(COSTA_ERR_ALLOC, "cudaMalloc(staging %lld B): %s", (long long)m.staging_bytes,
                         cudaGetErrorString(ce));
     }
-    m.remote_tiles = remote;
+    const uint64_t stage = reinterpret_cast<uint64_t>(m.d_staging);
+    std::vector<TileDesc> pack, unpack;
+    pack.reserve(remote.size());
+    unpack.reserve(remote.size());
+    for (const Remote &r : remote) {
+        const int64_t off = base[static_cast<size_t>(r.pkg)];
+        base[static_cast<size_t>(r.pkg)] += r.size;
+        const uint64_t addr = stage + static_cast<uint64_t>(off * es);
+        // pack: an exact copy in the source's frame (x = the source's contiguous axis)
+        TileDesc pk = r.d;
+        const bool t = (r.d.flags & TF_TRANSPOSE) != 0;
+        pk.nx = t ? r.d.ny : r.d.nx;
+        pk.ny = t ? r.d.nx : r.d.ny;
+        pk.dst = addr;
+        pk.dld = r.ld;
+        pk.flags = 0;
+        set_fast(pk, es);
+        pack.push_back(pk);
+        // unpack: the direct tile reading the staged copy
+        TileDesc up = r.d;
+        up.src = addr;
+        up.sld = r.ld;
+        set_fast(up, es);
+        unpack.push_back(up);
+    }
+    Arena arena;
+    const size_t o_pack = arena.add_vec(pack);
+    const size_t o_local = arena.add_vec(local);
+    const size_t o_unpack = arena.add_vec(unpack);
+    cudaError_t ce = cudaMalloc(&m.d_mem, arena.host.size());
+    if (ce != cudaSuccess) return fail(COSTA_ERR_ALLOC, "cudaMalloc(message tables): %s", cudaGetErrorString(ce));
+    ce = cudaMemcpy(m.d_mem, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(message tables)");
+    char *db = static_cast<char *>(m.d_mem);
+    m.pack = reinterpret_cast<const TileDesc *>(db + o_pack);
+    m.local = reinterpret_cast<const TileDesc *>(db + o_local);
+    m.unpack = reinterpret_cast<const TileDesc *>(db + o_unpack);
+    m.n_pack = static_cast<int64_t>(pack.size());
+    m.n_local = static_cast<int64_t>(local.size());
+    m.n_unpack = static_cast<int64_t>(unpack.size());
     m.built = true;
     plan.stats.staging_bytes = m.staging_bytes;
     return COSTA_OK;
@@ -531,10 +599,9 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     if (plan->total_tiles == 0) return COSTA_OK;
 
     RemapLaunch L{};
-    L.probs = plan->d_probs;
-    L.nprob = n;
+    L.tiles = plan->d_tiles;
+    L.ntiles = plan->total_tiles;
     L.dtype = plan->dtype;
-    L.total_tiles = plan->total_tiles;
     L.s = make_scalars(plan->dtype, alphas, betas, 0);
     L.per_problem = nullptr;
     bool uniform = true;
@@ -559,30 +626,41 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     // one launch per combine kind present in the batch
     bool kinds[K_NKINDS] = {};
     for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
-    auto launch_all = [&](int km) -> cudaError_t {
+    auto launch_list = [&](const TileDesc *list, int64_t count) -> cudaError_t {
+        RemapLaunch l = L;
+        l.tiles = list;
+        l.ntiles = count;
         for (int kind = 0; kind < K_NKINDS; ++kind) {
             if (!kinds[kind]) continue;
-            cudaError_t e = launch_remap(L, km, kind, stream);
+            cudaError_t e = launch_remap(l, kind, stream);
             if (e != cudaSuccess) return e;
         }
         return cudaSuccess;
     };
     cudaError_t ce;
     if (mode == COSTA_MODE_DIRECT) {
-        ce = launch_all(KM_DIRECT_ALL);
+        ce = launch_list(plan->d_tiles, plan->total_tiles);
         if (ce != cudaSuccess) return cuda_fail(ce, "remap kernel launch");
         return COSTA_OK;
     }
     s = ensure_message(*plan, relabel != 0);
     if (s != COSTA_OK) return s;
-    MessageData &m = plan->msg[relabel ? 1 : 0];
-    L.probs = m.d_probs;
-    L.staging = m.d_staging;
-    ce = launch_remap(L, KM_PACK, K_COPY, stream);
+    const MessageData &m = plan->msg[relabel ? 1 : 0];
+    RemapLaunch lp{};
+    lp.tiles = m.pack;
+    lp.ntiles = m.n_pack;
+    lp.dtype = plan->dtype;
+    lp.per_problem = nullptr;
+    const float one_f[2] = {1.0f, 0.0f}, zero_f[2] = {0.0f, 0.0f};
+    const double one_d[2] = {1.0, 0.0}, zero_d[2] = {0.0, 0.0};
+    const bool single = plan->dtype == COSTA_F32 || plan->dtype == COSTA_C64;
+    lp.s = make_scalars(plan->dtype, single ? static_cast<const void *>(one_f) : one_d,
+                        single ? static_cast<const void *>(zero_f) : zero_d, 0);
+    ce = launch_remap(lp, K_COPY, stream);
     if (ce != cudaSuccess) return cuda_fail(ce, "pack kernel launch");
-    ce = launch_all(KM_DIRECT_LOCAL);
+    ce = launch_list(m.local, m.n_local);
     if (ce != cudaSuccess) return cuda_fail(ce, "local remap kernel launch");
-    ce = launch_all(KM_UNPACK);
+    ce = launch_list(m.unpack, m.n_unpack);
     if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
     return COSTA_OK;
 }
@@ -839,6 +917,30 @@ costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op
         const int32_t v[6] = {t.a_blk, t.b_blk, t.a_off, t.b_off, t.len, t.cell};
         std::memcpy(out + 6 * k, v, sizeof v);
     }
+    return COSTA_OK;
+}
+
+costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void *out, int64_t cap,
+                               int64_t *count) {
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    if (!count || (cap > 0 && !out)) return fail(COSTA_ERR_INVALID_ARG, "bad arguments");
+    const int es = esize_of(A->dt), ts = tile_extent(es);
+    ProblemHost ph;
+    ph.A = A;
+    ph.B = B;
+    ph.op = op;
+    ph.rows = cut_pair_axis(A, B, op, 0, ts);
+    ph.cols = cut_pair_axis(A, B, op, 1, ts);
+    *count = static_cast<int64_t>(ph.rows.tiles.size()) * static_cast<int64_t>(ph.cols.tiles.size());
+    int64_t k = 0;
+    TileDesc *o = static_cast<TileDesc *>(out);
+    for_each_tile(ph, [&](const AxisTile &rt, const AxisTile &ct) {
+        if (k >= cap) return;
+        TileDesc d = direct_tile(ph, rt, ct, es, 0);
+        set_fast(d, es);
+        o[k++] = d;
+    });
     return COSTA_OK;
 }
 

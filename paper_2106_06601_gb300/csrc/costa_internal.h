@@ -63,20 +63,23 @@ struct Interval {
     int64_t len;
 };
 
-// One (A, B, op) pair as the kernels see it.
-struct ProblemDev {
-    const AxisTile *rows;
-    const AxisTile *cols;
-    const DevBlock *descA;      // nbrA * nbcA
-    const DevBlock *descB;      // nbrB * nbcB
-    const int64_t *stage_off;   // per tile (MESSAGE mode): element offset in staging, -1 = local
-    const int32_t *stage_ld;    // per tile (MESSAGE mode): leading dimension of the staged tile
-    int64_t tile_begin;         // first tile id of this problem in the launch
-    int32_t nu, nv;             // row pieces, column pieces
-    int32_t nbcA, nbcB;         // block columns of A and of B (descriptor indexing)
-    int32_t op;                 // costa_op
-    int32_t pad;
+// One tile of the remap kernel, resolved on the host at plan time: a
+// rectangle inside one block of A and one block of B (or a staging region),
+// in its canonical frame x = the target's contiguous axis:
+//   target element (x, y) at dst + (x + y * dld) elements
+//   source element (x, y) at src + (x + y * sld) elements (copy tile)
+//                         or src + (x * sld + y) elements (transposed tile)
+struct TileDesc {
+    uint64_t src;    // device address of source element (0, 0)
+    uint64_t dst;    // device address of target element (0, 0)
+    int32_t sld;     // source stride (elements)
+    int32_t dld;     // target stride (elements)
+    uint16_t nx, ny; // extents, at most the tile extent
+    uint16_t prob;   // problem index within the launch
+    uint16_t flags;  // TF_*
 };
+static_assert(sizeof(TileDesc) == 32, "TileDesc layout");
+enum : uint16_t { TF_TRANSPOSE = 1, TF_FAST = 2, TF_CONJ = 4 };
 
 // Scalars of one problem, as doubles ({re, im}); float data carries values
 // that are exactly representable in float.
@@ -106,16 +109,14 @@ COSTA_HD inline int kind_of(int32_t flags) {
     return K_COPY;
 }
 
-enum KernelMode : int { KM_DIRECT_ALL = 0, KM_DIRECT_LOCAL = 1, KM_PACK = 2, KM_UNPACK = 3 };
 
 struct RemapLaunch {
-    const ProblemDev *probs;
-    int32_t nprob;
+    const TileDesc *tiles;
+    int64_t ntiles;
     int32_t dtype;
-    int64_t total_tiles;
-    const Scalars *per_problem;  // device array of nprob, or nullptr: use `s`
+    int32_t pad;
+    const Scalars *per_problem;  // device array indexed by TileDesc::prob, or nullptr: use `s`
     Scalars s;
-    void *staging;
 };
 
 struct VolumeProblemDev {
@@ -141,13 +142,13 @@ struct VolumeLaunch {
 // Tile extent (elements along each axis of A) for an element size.
 inline int tile_extent(int esize) { return esize == 16 ? 16 : 32; }
 
-// Launches the remap kernel for (args.dtype, mode, kind).  With
+// Launches the remap kernel for (args.dtype, kind) over a tile list.  With
 // args.per_problem set, the kernel skips the tiles of problems of another kind.
-cudaError_t launch_remap(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
-cudaError_t launch_remap_f32(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
-cudaError_t launch_remap_f64(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
-cudaError_t launch_remap_c64(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
-cudaError_t launch_remap_c128(const RemapLaunch &args, int mode, int kind, cudaStream_t stream);
+cudaError_t launch_remap(const RemapLaunch &args, int kind, cudaStream_t stream);
+cudaError_t launch_remap_f32(const RemapLaunch &args, int kind, cudaStream_t stream);
+cudaError_t launch_remap_f64(const RemapLaunch &args, int kind, cudaStream_t stream);
+cudaError_t launch_remap_c64(const RemapLaunch &args, int kind, cudaStream_t stream);
+cudaError_t launch_remap_c128(const RemapLaunch &args, int kind, cudaStream_t stream);
 cudaError_t launch_volume(const VolumeLaunch &args, cudaStream_t stream);
 void count_launch();
 int64_t launches_so_far();

@@ -3,8 +3,8 @@
 
 namespace costa {
 
-cudaError_t launch_remap_c128(const RemapLaunch &a, int mode, int kind, cudaStream_t st) {
-    return remap::launch_remap_t<double2>(a, mode, kind, st);
+cudaError_t launch_remap_c128(const RemapLaunch &a, int kind, cudaStream_t st) {
+    return remap::launch_remap_t<double2>(a, kind, st);
 }
 
 }  // namespace costa

@@ -24,10 +24,12 @@
 // "cache-friendly ... kernel for matrix transposition").  Ragged or
 // misaligned tiles take an element-wise path.
 //
-// Modes: DIRECT_ALL (B -> A for every tile), and the message path of Alg. 3 /
-// Sec. 6: PACK (remote tiles: B -> staging, an exact copy), DIRECT_LOCAL
-// (tiles local after relabeling: B -> A), UNPACK (remote tiles: staging -> A
-// with the transform).
+// The kernel walks a list of tile descriptors (TileDesc) resolved on the host:
+// the direct list (every tile: B -> A), or the message path of Alg. 3 /
+// Sec. 6 as three lists: pack (remote tiles: B -> staging, an exact copy,
+// launched as K_COPY), local (tiles local after relabeling: B -> A) and
+// unpack (remote tiles: staging -> A with the transform).  Each warp takes
+// every (gridDim.x * warps)-th tile and reads the descriptors 32 at a time.
 //
 // No kernel here waits on another block or on a flag.  cp.async.wait_group
 // waits only for this thread's own copies, which always complete.
@@ -63,6 +65,9 @@ template <typename T> struct Cfg {
     static constexpr int PITCH = TS + 1;
     static constexpr int BUF_BYTES_RAW = TS * PITCH * static_cast<int>(sizeof(T));
     static constexpr int BUF_BYTES = (BUF_BYTES_RAW + 127) / 128 * 128;
+    // shared-memory buffers per warp: the warp keeps NBUF - 1 tiles' copies
+    // in flight ahead of the tile it writes (deeper for the 4 KB tiles)
+    static constexpr int NBUF = BUF_BYTES <= 4608 ? 3 : 2;
 };
 constexpr int kWarps = 4;
 constexpr int kMinBlocks = 3;
@@ -80,8 +85,9 @@ __device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;\n" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
+template <int N> __device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
 
 template <typename T>
 __device__ __forceinline__ Chunk<T> load_rw(const T *p) {
@@ -173,7 +179,8 @@ template <typename T> struct Geom {
     const T *src;
     int64_t dld, sld;
     int nx, ny;
-    bool transpose, fast;
+    int prob;
+    bool transpose, fast, conj;
 };
 
 // Chunk c of staged row r lives in slot c ^ swz(r): across the VEC rows that
@@ -397,151 +404,174 @@ __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsi
     }
 }
 
-__device__ __forceinline__ bool aligned16(const void *p, int64_t ld_bytes) {
-    return ((reinterpret_cast<uintptr_t>(p) | static_cast<uintptr_t>(ld_bytes)) & 15) == 0;
+// Scalars of a problem in the kernel's form.
+__device__ __forceinline__ void make_sc(const Scalars &S, Sc &s) {
+    s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
+    s.conj_mask = 0u;
+    s.bexp = S.beta_exp;
+    s.bsign_hi = static_cast<unsigned>(__double2hiint(S.beta[0])) & 0x80000000u;
+    s.p2_add = static_cast<unsigned>(S.beta_exp) << 20;
+    // admissible biased exponents e: e in [1, 2046] and e + k in [1, 2046]
+    const int lo = max(1, 1 - S.beta_exp), hi = min(2046, 2046 - S.beta_exp);
+    s.p2_lo = hi >= lo ? static_cast<unsigned>(lo) : 4096u;  // 4096: nothing admissible
+    s.p2_span = hi >= lo ? static_cast<unsigned>(hi - lo) : 0u;
 }
 
-// The tile with linear id t (or the next one this launch covers), resolved
-// into its geometry and scalars.  Returns false when the warp has no tile
-// left.
-template <typename T, int MODE, int KIND>
-__device__ __forceinline__ bool fetch_tile(const RemapLaunch &args, int64_t &t, int64_t stride,
-                                           Geom<T> &g, Sc &s) {
-    using C = Cfg<T>;
-    for (; t < args.total_tiles; t += stride) {
-        int k = 0;
-        if (args.nprob > 1) {
-            int lo = 0, hi = args.nprob;
-            while (hi - lo > 1) {
-                const int mid = (lo + hi) >> 1;
-                if (args.probs[mid].tile_begin <= t) lo = mid; else hi = mid;
-            }
-            k = lo;
-        }
-        const ProblemDev &P = args.probs[k];
-        const int64_t tl = t - P.tile_begin;
-        int64_t soff = -1;
-        int64_t stld = 0;
-        if (MODE != KM_DIRECT_ALL) {
-            soff = P.stage_off[tl];
-            if (MODE == KM_DIRECT_LOCAL ? soff >= 0 : soff < 0) continue;
-            stld = P.stage_ld[tl];
-        }
-        s.ar = 1.0; s.ai = 0.0; s.br = 0.0; s.bi = 0.0; s.conj_mask = 0u; s.bexp = 0; s.bsign_hi = 0u;
-        s.p2_add = 0u; s.p2_lo = 1u; s.p2_span = 0u;
-        const int op = P.op;
-        if (MODE != KM_PACK) {
-            Scalars S;
-            if (args.per_problem) {
-                S = args.per_problem[k];
-                if (kind_of(S.flags) != KIND) continue;  // another launch covers it
-            } else {
-                S = args.s;
-            }
-            s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
-            s.bexp = S.beta_exp;
-            s.bsign_hi = static_cast<unsigned>(__double2hiint(S.beta[0])) & 0x80000000u;
-            s.p2_add = static_cast<unsigned>(S.beta_exp) << 20;
-            {   // e in [1, 2046] and e + k in [1, 2046]
-                const int lo = max(1, 1 - S.beta_exp), hi = min(2046, 2046 - S.beta_exp);
-                s.p2_lo = static_cast<unsigned>(lo);
-                s.p2_span = hi >= lo ? static_cast<unsigned>(hi - lo) : 0u;
-                if (hi < lo) s.p2_lo = 4096u;  // nothing admissible: always multiply
-            }
-            s.conj_mask = (ET<T>::CPLX && op == COSTA_OP_C) ? 0x80000000u : 0u;
-        }
-        const int u = static_cast<int>(tl / P.nv);
-        const int v = static_cast<int>(tl - static_cast<int64_t>(u) * P.nv);
-        const AxisTile rt = P.rows[u];
-        const AxisTile ct = P.cols[v];
-        const DevBlock dA = P.descA[static_cast<int64_t>(rt.a_blk) * P.nbcA + ct.a_blk];
-        const DevBlock dB = op == COSTA_OP_N
-                                ? P.descB[static_cast<int64_t>(rt.b_blk) * P.nbcB + ct.b_blk]
-                                : P.descB[static_cast<int64_t>(ct.b_blk) * P.nbcB + rt.b_blk];
+// The tile descriptors of one warp come in batches of 32: lane k holds the
+// descriptor of the warp's tile 32 * b + k, loaded one batch ahead, and tile
+// j is shuffled out of lane j % 32 of the current batch.
+struct DescRegs {
+    uint4 lo, hi;
+};
 
-        // source block element (rb, cb) of tile element (i, j)
-        const bool b_col = dB.order == COSTA_COL_MAJOR;
-        int64_t rb, cb;
-        bool src_fast_i;
-        if (op == COSTA_OP_N) { rb = rt.b_off; cb = ct.b_off; src_fast_i = b_col; }
-        else                  { rb = ct.b_off; cb = rt.b_off; src_fast_i = !b_col; }
-        const T *src = reinterpret_cast<const T *>(dB.ptr) + (b_col ? rb + cb * dB.ld : rb * dB.ld + cb);
-        int64_t sld = dB.ld;
+__device__ __forceinline__ DescRegs load_batch(const RemapLaunch &a, int64_t first, int64_t stride,
+                                               int64_t b, int lane) {
+    DescRegs r;
+    const int64_t t = first + (b * 32 + lane) * stride;
+    if (t < a.ntiles) {
+        const uint4 *p = reinterpret_cast<const uint4 *>(a.tiles + t);
+        r.lo = __ldg(p);
+        r.hi = __ldg(p + 1);
+    } else {
+        r.lo = make_uint4(0, 0, 0, 0);
+        r.hi = make_uint4(0, 0, 0, 0);
+    }
+    return r;
+}
 
-        const bool a_col = dA.order == COSTA_COL_MAJOR;
-        T *dst = reinterpret_cast<T *>(dA.ptr) +
-                 (a_col ? rt.a_off + static_cast<int64_t>(ct.a_off) * dA.ld
-                        : static_cast<int64_t>(rt.a_off) * dA.ld + ct.a_off);
-        int64_t dld = dA.ld;
-        bool dst_fast_i = a_col;
+__device__ __forceinline__ TileDesc shfl_desc(const DescRegs &r, int src) {
+    uint4 lo, hi;
+    lo.x = __shfl_sync(0xffffffffu, r.lo.x, src);
+    lo.y = __shfl_sync(0xffffffffu, r.lo.y, src);
+    lo.z = __shfl_sync(0xffffffffu, r.lo.z, src);
+    lo.w = __shfl_sync(0xffffffffu, r.lo.w, src);
+    hi.x = __shfl_sync(0xffffffffu, r.hi.x, src);
+    hi.y = __shfl_sync(0xffffffffu, r.hi.y, src);
+    hi.z = __shfl_sync(0xffffffffu, r.hi.z, src);
+    hi.w = __shfl_sync(0xffffffffu, r.hi.w, src);
+    TileDesc d;
+    d.src = (static_cast<uint64_t>(lo.y) << 32) | lo.x;
+    d.dst = (static_cast<uint64_t>(lo.w) << 32) | lo.z;
+    d.sld = static_cast<int32_t>(hi.x);
+    d.dld = static_cast<int32_t>(hi.y);
+    d.nx = static_cast<uint16_t>(hi.z & 0xFFFFu);
+    d.ny = static_cast<uint16_t>(hi.z >> 16);
+    d.prob = static_cast<uint16_t>(hi.w & 0xFFFFu);
+    d.flags = static_cast<uint16_t>(hi.w >> 16);
+    return d;
+}
 
-        if (MODE == KM_PACK) {
-            dst = reinterpret_cast<T *>(args.staging) + soff;
-            dld = stld;
-            dst_fast_i = src_fast_i;
-        } else if (MODE == KM_UNPACK) {
-            src = reinterpret_cast<const T *>(args.staging) + soff;
-            sld = stld;
+template <typename T> __device__ __forceinline__ Geom<T> geom_of(const TileDesc &d) {
+    Geom<T> g;
+    g.src = reinterpret_cast<const T *>(d.src);
+    g.dst = reinterpret_cast<T *>(d.dst);
+    g.sld = d.sld;
+    g.dld = d.dld;
+    g.nx = d.nx;
+    g.ny = d.ny;
+    g.prob = d.prob;
+    g.transpose = (d.flags & TF_TRANSPOSE) != 0;
+    g.fast = (d.flags & TF_FAST) != 0;
+    g.conj = ET<T>::CPLX && (d.flags & TF_CONJ) != 0;
+    return g;
+}
+
+// Walks the warp's tile sequence j = 0, 1, ... (tile first + j * stride).
+struct TileStream {
+    DescRegs cur, nxt;
+    int64_t j;
+};
+
+// Next tile of the warp; false when none is left.  With per-problem scalars,
+// tiles of problems of another kind are skipped (another launch covers
+// them).  Called by all 32 lanes with the same state.
+template <typename T, int KIND>
+__device__ __forceinline__ bool next_tile(const RemapLaunch &a, int64_t first, int64_t stride,
+                                          TileStream &ts, Geom<T> &g, int lane) {
+    for (;;) {
+        const int64_t t = first + ts.j * stride;
+        if (t >= a.ntiles) return false;
+        const int k = static_cast<int>(ts.j & 31);
+        if (k == 0 && ts.j > 0) {
+            ts.cur = ts.nxt;
+            ts.nxt = load_batch(a, first, stride, (ts.j >> 5) + 1, lane);
         }
-        g.dst = dst;
-        g.src = src;
-        g.dld = dld;
-        g.sld = sld;
-        g.nx = dst_fast_i ? rt.len : ct.len;
-        g.ny = dst_fast_i ? ct.len : rt.len;
-        g.transpose = dst_fast_i != src_fast_i;
-        // vector fast path: both sides 16-byte aligned and every run a whole
-        // number of chunks (the source runs along y when transposing)
-        const int vrun_src = g.transpose ? g.ny : g.nx;
-        g.fast = aligned16(dst, dld * static_cast<int64_t>(sizeof(T))) &&
-                 aligned16(src, sld * static_cast<int64_t>(sizeof(T))) && (g.nx % C::VEC) == 0 &&
-                 (vrun_src % C::VEC) == 0;
+        const TileDesc d = shfl_desc(ts.cur, k);
+        ++ts.j;
+        if (a.per_problem && kind_of(a.per_problem[d.prob].flags) != KIND) continue;
+        g = geom_of<T>(d);
         return true;
     }
-    return false;
 }
 
-template <typename T, int MODE, int KIND>
+// Writes one tile (staged in `buf` if it is a fast tile).  `cached` holds
+// the problem whose scalars are in `s`.
+template <typename T, int KIND, int NB>
+__device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &g, Sc &s, int &cached,
+                                           unsigned char *buf, int lane) {
+    using C = Cfg<T>;
+    if (a.per_problem && g.prob != cached) {
+        make_sc(a.per_problem[g.prob], s);
+        cached = g.prob;
+    }
+    s.conj_mask = g.conj ? 0x80000000u : 0u;
+    if (g.fast) {
+        Chunk<T> av[C::NPASS];
+        load_a<T, KIND>(g, s, av, lane);
+        cp_async_wait<NB - 1>();  // this tile's copies (later tiles' may still fly)
+        __syncwarp();
+        stage_drain<T, KIND>(g, s, buf, av, lane);
+    } else {
+        tile_general<T, KIND>(g, s, buf, lane);
+    }
+    __syncwarp();  // the buffer is free before it is staged into again
+}
+
+template <typename T, int KIND>
 __global__ void __launch_bounds__(kWarps * 32, kMinBlocks) remap_kernel(const RemapLaunch args) {
     using C = Cfg<T>;
+    constexpr int NB = C::NBUF;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    unsigned char *bufs = smem_raw + warp * 2 * C::BUF_BYTES;
+    unsigned char *bufs = smem_raw + warp * NB * C::BUF_BYTES;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * kWarps;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
 
-    int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
-    Geom<T> g;
     Sc s;
-    bool have = fetch_tile<T, MODE, KIND>(args, t, stride, g, s);
-    if (have && g.fast) stage_issue<T>(g, bufs, lane);
-    cp_async_commit();
-    int cur = 0;
-    while (have) {
-        // prefetch: resolve the next tile and start its copies
-        int64_t tn = t + stride;
-        Geom<T> gn;
-        Sc sn;
-        const bool have_n = fetch_tile<T, MODE, KIND>(args, tn, stride, gn, sn);
-        unsigned char *buf = bufs + cur * C::BUF_BYTES;
-        if (have_n && gn.fast) stage_issue<T>(gn, bufs + (cur ^ 1) * C::BUF_BYTES, lane);
+    int cached = -1;
+    if (!args.per_problem) make_sc(args.s, s);
+    TileStream ts;
+    ts.j = 0;
+    ts.cur = load_batch(args, first, stride, 0, lane);
+    ts.nxt = load_batch(args, first, stride, 1, lane);
+
+    // ring[0] is the tile being written, ring[k] the tile k ahead, staged in
+    // buffer (cur + k) % NB
+    Geom<T> ring[NB];
+    bool have[NB];
+#pragma unroll
+    for (int k = 0; k < NB - 1; ++k) {
+        have[k] = (k == 0 || have[k - 1]) && next_tile<T, KIND>(args, first, stride, ts, ring[k], lane);
+        if (have[k] && ring[k].fast) stage_issue<T>(ring[k], bufs + k * C::BUF_BYTES, lane);
         cp_async_commit();
-        if (g.fast) {
-            Chunk<T> av[C::NPASS];
-            load_a<T, KIND>(g, s, av, lane);
-            cp_async_wait_1();  // this tile's copies (the next tile's may still fly)
-            __syncwarp();
-            stage_drain<T, KIND>(g, s, buf, av, lane);
-        } else {
-            tile_general<T, KIND>(g, s, buf, lane);
-        }
-        __syncwarp();  // the buffer is free before it is staged into again
-        g = gn;
-        s = sn;
-        t = tn;
-        have = have_n;
-        cur ^= 1;
     }
-    cp_async_wait_0();
+    int cur = 0;
+    while (have[0]) {
+        have[NB - 1] = have[NB - 2] && next_tile<T, KIND>(args, first, stride, ts, ring[NB - 1], lane);
+        int ahead = cur + NB - 1;
+        if (ahead >= NB) ahead -= NB;
+        if (have[NB - 1] && ring[NB - 1].fast)
+            stage_issue<T>(ring[NB - 1], bufs + ahead * C::BUF_BYTES, lane);
+        cp_async_commit();
+        write_tile<T, KIND, NB>(args, ring[0], s, cached, bufs + cur * C::BUF_BYTES, lane);
+#pragma unroll
+        for (int k = 0; k < NB - 1; ++k) {
+            ring[k] = ring[k + 1];
+            have[k] = have[k + 1];
+        }
+        cur = cur + 1 == NB ? 0 : cur + 1;
+    }
+    cp_async_wait<0>();
 }
 
 inline int sm_count() {
@@ -555,10 +585,10 @@ inline int sm_count() {
     return cached;
 }
 
-template <typename T, int MODE, int KIND>
+template <typename T, int KIND>
 cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
-    auto kern = remap_kernel<T, MODE, KIND>;
-    const size_t smem = static_cast<size_t>(kWarps) * 2 * Cfg<T>::BUF_BYTES;
+    auto kern = remap_kernel<T, KIND>;
+    const size_t smem = static_cast<size_t>(kWarps) * Cfg<T>::NBUF * Cfg<T>::BUF_BYTES;
     static int per_sm = 0;
     if (per_sm == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -568,7 +598,7 @@ cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         if (per_sm < 1) per_sm = 1;
     }
-    const int64_t want = (a.total_tiles + kWarps - 1) / kWarps;
+    const int64_t want = (a.ntiles + kWarps - 1) / kWarps;
     const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;
     const int blocks = static_cast<int>(want < cap ? want : cap);
     if (blocks <= 0) return cudaSuccess;
@@ -577,28 +607,18 @@ cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-// Kernel for (element type, mode, combine kind).  Real types never take
-// K_CPLX; PACK is always a plain copy.
+// Kernel for (element type, combine kind).  Real types never take K_CPLX.
 template <typename T>
-cudaError_t launch_remap_t(const RemapLaunch &a, int mode, int kind, cudaStream_t st) {
-    if (mode == KM_PACK) return launch_t<T, KM_PACK, K_COPY>(a, st);
-#define COSTA_KINDS(MODE)                                                         \
-    switch (kind) {                                                               \
-    case K_COPY: return launch_t<T, MODE, K_COPY>(a, st);                         \
-    case K_SCALE: return launch_t<T, MODE, K_SCALE>(a, st);                       \
-    case K_AXPBY: return launch_t<T, MODE, K_AXPBY>(a, st);                       \
-    case K_AXPBY2: return launch_t<T, MODE, K_AXPBY2>(a, st);                     \
-    default:                                                                      \
-        if constexpr (ET<T>::CPLX) return launch_t<T, MODE, K_CPLX>(a, st);       \
-        return cudaErrorInvalidValue;                                             \
+cudaError_t launch_remap_t(const RemapLaunch &a, int kind, cudaStream_t st) {
+    switch (kind) {
+    case K_COPY: return launch_t<T, K_COPY>(a, st);
+    case K_SCALE: return launch_t<T, K_SCALE>(a, st);
+    case K_AXPBY: return launch_t<T, K_AXPBY>(a, st);
+    case K_AXPBY2: return launch_t<T, K_AXPBY2>(a, st);
+    default:
+        if constexpr (ET<T>::CPLX) return launch_t<T, K_CPLX>(a, st);
+        return cudaErrorInvalidValue;
     }
-    switch (mode) {
-    case KM_DIRECT_ALL: COSTA_KINDS(KM_DIRECT_ALL)
-    case KM_DIRECT_LOCAL: COSTA_KINDS(KM_DIRECT_LOCAL)
-    case KM_UNPACK: COSTA_KINDS(KM_UNPACK)
-    default: return cudaErrorInvalidValue;
-    }
-#undef COSTA_KINDS
 }
 
 }  // namespace remap

@@ -62,13 +62,13 @@ void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int64_t launches_so_far() { return g_launches.load(std::memory_order_relaxed); }
 
-cudaError_t launch_remap(const RemapLaunch &a, int mode, int kind, cudaStream_t stream) {
-    if (a.total_tiles <= 0) return cudaSuccess;
+cudaError_t launch_remap(const RemapLaunch &a, int kind, cudaStream_t stream) {
+    if (a.ntiles <= 0) return cudaSuccess;
     switch (a.dtype) {
-    case COSTA_F32: return launch_remap_f32(a, mode, kind, stream);
-    case COSTA_F64: return launch_remap_f64(a, mode, kind, stream);
-    case COSTA_C64: return launch_remap_c64(a, mode, kind, stream);
-    case COSTA_C128: return launch_remap_c128(a, mode, kind, stream);
+    case COSTA_F32: return launch_remap_f32(a, kind, stream);
+    case COSTA_F64: return launch_remap_f64(a, kind, stream);
+    case COSTA_C64: return launch_remap_c64(a, kind, stream);
+    case COSTA_C128: return launch_remap_c128(a, kind, stream);
     default: return cudaErrorInvalidValue;
     }
 }

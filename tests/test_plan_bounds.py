@@ -16,7 +16,7 @@ FAKE = 1 << 40
 
 def _layout(spec, dtype):
     es = {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[dtype]
-    ptrs = FAKE + (spec.off + spec.buf.astype(np.int64) * (1 << 32)) * es
+    ptrs = FAKE + spec.buf.astype(np.int64) * (1 << 32) + spec.off * es
     return costa.costa_layout_from_spec(spec, dtype, ptrs)
 
 
@@ -50,16 +50,62 @@ def check_pair(p):
         LB.destroy()
 
 
+def check_tiles(p):
+    """Every tile's four corners (the tile is affine, so all its addresses lie
+    between them) fall inside the source and target rank buffers, the tiles
+    cover m * n elements, and the vector flag implies 16-byte alignment."""
+    es = {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[p.dtype]
+    LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+    try:
+        t = costa.costa_debug_tiles(LA, LB, p.op)
+    finally:
+        LA.destroy()
+        LB.destroy()
+    nx, ny = t["nx"].astype(np.int64), t["ny"].astype(np.int64)
+    assert (nx * ny).sum() == p.A.m * p.A.n
+    assert np.all(nx >= 1) and np.all(ny >= 1)
+    tr = (t["flags"] & 1) != 0
+    for name, base, ld, spec, xs, ys in (
+            ("dst", t["dst"], t["dld"], p.A, 1, None),
+            ("src", t["src"], t["sld"], p.B, None, None)):
+        base = base.astype(np.int64)
+        ld = ld.astype(np.int64)
+        if name == "dst":
+            sx, sy = np.ones_like(ld), ld
+        else:
+            sx = np.where(tr, ld, 1)
+            sy = np.where(tr, 1, ld)
+        for cx in (0, 1):
+            for cy in (0, 1):
+                addr = base + ((nx - 1) * cx * sx + (ny - 1) * cy * sy) * es
+                rel = addr - FAKE
+                buf = rel >> 32
+                off = rel - (buf << 32)
+                assert np.all(buf >= 0) and np.all(buf < spec.nbuf), name
+                assert np.all(off >= 0) and np.all(off < spec.bufsize[buf] * es), name
+                assert np.all(off % es == 0), name
+    fast = (t["flags"] & 2) != 0
+    vec = 16 // es
+    assert np.all(t["dst"][fast] % 16 == 0) and np.all(t["src"][fast] % 16 == 0)
+    assert np.all((t["dld"][fast].astype(np.int64) * es) % 16 == 0)
+    assert np.all((t["sld"][fast].astype(np.int64) * es) % 16 == 0)
+    assert np.all(nx[fast] % vec == 0)
+    assert np.all(np.where(tr, ny, nx)[fast] % vec == 0)
+
+
 @pytest.mark.parametrize("name", ["c1", "c2", "c3", "c5"])
 def test_config_pieces_in_bounds(name):
     check_pair(C.CONFIGS[name]())
+    check_tiles(C.CONFIGS[name]())
 
 
 def test_c4_pieces_in_bounds():
     for p in C.c4():
         check_pair(p)
+        check_tiles(p)
 
 
 def test_fuzz_pieces_in_bounds():
     for case in range(400):
         check_pair(C.fuzz_problem(case))
+        check_tiles(C.fuzz_problem(case))
