@@ -9,6 +9,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <memory>
@@ -254,13 +255,24 @@ void set_fast(TileDesc &d, int es) {
     d.flags = static_cast<uint16_t>(fast ? (d.flags | TF_FAST) : (d.flags & ~TF_FAST));
 }
 
-// Visits the tiles of a problem in super-tiles of kSuper x kSuper pieces,
+// Visits the tiles of a problem in super-tiles of k x k pieces,
 // row pieces fastest inside each: the tiles that warps work on at the same
 // time then cover compact regions of A and of B (runs of kSuper tiles along
 // both axes) instead of one band of rows across every column.
-constexpr int kSuper = 8;
+// Default k: 16 for 16-byte elements (16 x 16 tiles), 8 otherwise (measured
+// on GB300).  The environment variable COSTA_SUPER_TILE (1..64) overrides it,
+// for tuning.
+int super_tile(int esize) {
+    static const int env = [] {
+        const char *e = std::getenv("COSTA_SUPER_TILE");
+        const int v = e ? std::atoi(e) : 0;
+        return v >= 1 && v <= 64 ? v : 0;
+    }();
+    return env ? env : (esize == 16 ? 16 : 8);
+}
 
 template <typename F> void for_each_tile(const ProblemHost &ph, F &&f) {
+    const int kSuper = super_tile(esize_of(ph.A->dt));
     const int nu = static_cast<int>(ph.rows.tiles.size()), nv = static_cast<int>(ph.cols.tiles.size());
     for (int su = 0; su < nu; su += kSuper)
         for (int sv = 0; sv < nv; sv += kSuper)

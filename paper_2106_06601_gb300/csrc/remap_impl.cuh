@@ -51,6 +51,34 @@ template <> struct ET<double>  { enum { VEC = 2, CPLX = 0 }; typedef double R; }
 template <> struct ET<float2>  { enum { VEC = 2, CPLX = 1 }; typedef float R; };
 template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; };
 
+#ifndef COSTA_WARPS_4
+#define COSTA_WARPS_4 8
+#endif
+#ifndef COSTA_MINB_4
+#define COSTA_MINB_4 2
+#endif
+#ifndef COSTA_NBUF_4
+#define COSTA_NBUF_4 2
+#endif
+#ifndef COSTA_WARPS_8
+#define COSTA_WARPS_8 4
+#endif
+#ifndef COSTA_MINB_8
+#define COSTA_MINB_8 3
+#endif
+#ifndef COSTA_NBUF_8
+#define COSTA_NBUF_8 2
+#endif
+#ifndef COSTA_WARPS_16
+#define COSTA_WARPS_16 8
+#endif
+#ifndef COSTA_MINB_16
+#define COSTA_MINB_16 1
+#endif
+#ifndef COSTA_NBUF_16
+#define COSTA_NBUF_16 3
+#endif
+
 // Per element type: tile extent TS, 16-byte chunk width VEC (elements), and
 // the lane mapping: CPR chunks cover one run of TS elements, a warp pass
 // covers RPP runs, NPASS passes cover TS runs.  A staged tile is TS rows of
@@ -65,12 +93,14 @@ template <typename T> struct Cfg {
     static constexpr int PITCH = TS + 1;
     static constexpr int BUF_BYTES_RAW = TS * PITCH * static_cast<int>(sizeof(T));
     static constexpr int BUF_BYTES = (BUF_BYTES_RAW + 127) / 128 * 128;
-    // shared-memory buffers per warp: the warp keeps NBUF - 1 tiles' copies
-    // in flight ahead of the tile it writes (deeper for the 4 KB tiles)
-    static constexpr int NBUF = BUF_BYTES <= 4608 ? 3 : 2;
+    // Launch shape per element type (measured on GB300): warps per block,
+    // resident blocks per SM the registers must allow, and shared-memory
+    // buffers per warp (the warp keeps NBUF - 1 tiles' copies in flight ahead
+    // of the tile it writes).  Overridable at build time for tuning.
+    static constexpr int WARPS = sizeof(T) == 4 ? COSTA_WARPS_4 : sizeof(T) == 16 ? COSTA_WARPS_16 : COSTA_WARPS_8;
+    static constexpr int MINB = sizeof(T) == 4 ? COSTA_MINB_4 : sizeof(T) == 16 ? COSTA_MINB_16 : COSTA_MINB_8;
+    static constexpr int NBUF = sizeof(T) == 4 ? COSTA_NBUF_4 : sizeof(T) == 16 ? COSTA_NBUF_16 : COSTA_NBUF_8;
 };
-constexpr int kWarps = 4;
-constexpr int kMinBlocks = 3;
 
 template <typename T> struct Chunk {
     union {
@@ -528,14 +558,14 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
 }
 
 template <typename T, int KIND>
-__global__ void __launch_bounds__(kWarps * 32, kMinBlocks) remap_kernel(const RemapLaunch args) {
+__global__ void __launch_bounds__(Cfg<T>::WARPS * 32, Cfg<T>::MINB) remap_kernel(const RemapLaunch args) {
     using C = Cfg<T>;
     constexpr int NB = C::NBUF;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     unsigned char *bufs = smem_raw + warp * NB * C::BUF_BYTES;
-    const int64_t stride = static_cast<int64_t>(gridDim.x) * kWarps;
-    const int64_t first = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * C::WARPS;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * C::WARPS + warp;
 
     Sc s;
     int cached = -1;
@@ -588,6 +618,7 @@ inline int sm_count() {
 template <typename T, int KIND>
 cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     auto kern = remap_kernel<T, KIND>;
+    constexpr int kWarps = Cfg<T>::WARPS;
     const size_t smem = static_cast<size_t>(kWarps) * Cfg<T>::NBUF * Cfg<T>::BUF_BYTES;
     static int per_sm = 0;
     if (per_sm == 0) {
