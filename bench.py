@@ -317,13 +317,21 @@ def run_cpu_oracle(args, probs, seconds_target: float):
                      rows=(0, rows), threads=threads)
     dt = max(time.perf_counter() - t0, 1e-6)
     rows2 = int(min(p.A.m, max(rows, rows * seconds_target / dt)))
+    # when the whole instance takes less than the target, repeat it
+    reps, done = 0, 0.0
     t0 = time.perf_counter()
-    oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B, Bh.buffers(),
-                     rows=(0, rows2), threads=threads)
-    dt2 = time.perf_counter() - t0
+    while True:
+        oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B, Bh.buffers(),
+                         rows=(0, rows2), threads=threads)
+        reps += 1
+        done = time.perf_counter() - t0
+        if rows2 < p.A.m or done >= seconds_target:
+            break
+    dt2 = done / reps
     gbs = rows2 * per_row_bytes / dt2 / 1e9
     desc = (f"rows 0..{rows2} of A ({rows2 * p.A.n} of {p.A.m * p.A.n} elements"
-            f"{' of instance 0 of ' + str(len(probs)) if len(probs) > 1 else ''}), {dt2:.1f} s")
+            f"{' of instance 0 of ' + str(len(probs)) if len(probs) > 1 else ''}), "
+            f"{reps} pass(es), {done:.1f} s")
     return gbs, threads, desc, rows2, dt2
 
 
