@@ -154,6 +154,23 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm), "window": window}
 
 
+def max_over_ranks(x: float, device=None) -> float:
+    """The maximum of x over all ranks (identity without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(bytes_per_rank: int, world: int, steps: int, max_ms: float) -> float:
+    """Whole-job GB/s: the bytes every rank moved in `steps` steps over the
+    slowest rank's time."""
+    return bytes_per_rank * world * steps / (max_ms * 1e-3) / 1e9
+
+
 def problems(workload, small=False):
     p = (C.CONFIGS_SMALL if small else C.CONFIGS)[workload]()
     return p if isinstance(p, list) else [p]
@@ -237,12 +254,9 @@ def run_gpu(args, rank, world, local_rank):
     clocks.stop()
     clk = clocks.summary(t_wall0, t_wall1)
 
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = t.item()
+    total_ms = max_over_ranks(total_ms, dev)
     ms_per_step = total_ms / args.steps
-    value = nbytes * world * args.steps / (total_ms * 1e-3) / 1e9
+    value = job_throughput(nbytes, world, args.steps, total_ms)
 
     # ---- end to end: pinned host inputs, copies inside the timed region ----
     e2e = None
@@ -279,12 +293,8 @@ def run_gpu(args, rank, world, local_rank):
             e2e_step()
         e2.record(stream)
         torch.cuda.synchronize(dev)
-        e2e_ms = s2.elapsed_time(e2)
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e2e_ms = t.item()
-        e2e = {"value": round(nbytes * world * args.e2e_steps / (e2e_ms * 1e-3) / 1e9, 3),
+        e2e_ms = max_over_ranks(s2.elapsed_time(e2), dev)
+        e2e = {"value": round(job_throughput(nbytes, world, args.e2e_steps, e2e_ms), 3),
                "unit": "GB/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "ms_per_step": round(e2e_ms / args.e2e_steps, 4), "steps": args.e2e_steps}
 
