@@ -204,6 +204,40 @@ costa_status costa_plan_stats_get(int n, const costa_layout *A, const costa_layo
                                   const costa_op *ops, int relabel,
                                   costa_plan_stats *stats, void *stream);
 
+/* A process-grid layout described without per-block arrays (for the
+ * relabeling study of Sec. 7.2, where blocks can be 1 x 1): block (bi, bj)
+ * covers rows [row_splits[bi], row_splits[bi+1]) x columns
+ * [col_splits[bj], col_splits[bj+1]) and is owned by rank
+ * grid[row_procs[bi] * pc + col_procs[bj]].  Block-cyclic layouts are the
+ * case row_procs[bi] = bi mod pr, col_procs[bj] = bj mod pc.  All arrays are
+ * host arrays: row_splits nbr + 1, row_procs nbr, col_splits nbc + 1,
+ * col_procs nbc, grid pr * pc. */
+typedef struct {
+    int nbr, nbc;
+    const int64_t *row_splits;
+    const int *row_procs;
+    const int64_t *col_splits;
+    const int *col_procs;
+    int pr, pc;
+    const int *grid;
+} costa_grid_desc;
+
+/* Volumes V[p * P + q] of the reshuffle of B into A's layout (as
+ * costa_volume, Alg. 2) for process-grid layouts, computed from the 1-D
+ * overlaps of the row and column splits: O(blocks per axis + P^2), no
+ * overlay cells, no device work.  Errors: INVALID_ARG, LAYOUT, SHAPE. */
+costa_status costa_volume_grid(const costa_grid_desc *A, const costa_grid_desc *B, costa_op op, int P,
+                               int64_t *V);
+
+/* The greedy relabeling of Sec. 6 ("a simple greedy algorithm, which is a
+ * 2-approximation" of the maximum-weight perfect matching): pairs (p, q) by
+ * decreasing V[p * P + q] (ties: smaller p, then smaller q), each kept when p
+ * and q are both unmatched; leftover target labels take leftover processes in
+ * increasing order.  sigma[q] = p as in costa_relabel; local_volume
+ * (nullable) receives sum_q V[sigma[q] * P + q], at least half the optimum.
+ * Host only.  Errors: INVALID_ARG. */
+costa_status costa_relabel_greedy(int P, const int64_t *V, int *sigma, int64_t *local_volume);
+
 /* Diagnostics (host only, no device work): the pieces into which the plan
  * cuts one axis of A (axis 0 = rows, 1 = columns) for the pair (A, B, op).
  * Each piece is 6 int32: {A block index, op(B) block index, offset in A's

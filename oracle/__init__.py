@@ -68,6 +68,8 @@ def lib():
             _lib.oracle_lap_bruteforce.restype = ctypes.c_int64
             _lib.oracle_lap_subset_dp.argtypes = [ctypes.c_int, P, P]
             _lib.oracle_lap_subset_dp.restype = ctypes.c_int64
+            _lib.oracle_lap_greedy.argtypes = [ctypes.c_int, P, P]
+            _lib.oracle_lap_greedy.restype = ctypes.c_int64
         return _lib
 
 
@@ -187,6 +189,17 @@ def lap_subset_dp(V: np.ndarray):
     sigma = np.zeros(P, dtype=np.int32)
     best = lib().oracle_lap_subset_dp(P, _ptr(V), _ptr(sigma))
     return int(best), sigma
+
+
+def lap_greedy(V: np.ndarray):
+    """The greedy relabeling of Sec. 6 (a 2-approximation): pairs by
+    decreasing volume (ties: smaller p, then smaller q), each kept when both
+    ends are free; leftover labels take leftover processes in order."""
+    V = np.ascontiguousarray(V, dtype=np.int64)
+    P = V.shape[0]
+    sigma = np.zeros(P, dtype=np.int32)
+    total = lib().oracle_lap_greedy(P, _ptr(V), _ptr(sigma))
+    return int(total), sigma
 
 
 def lap_library(V: np.ndarray):

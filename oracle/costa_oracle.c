@@ -35,6 +35,13 @@
  *    the process that takes target label q).  Brute force over all P!
  *    permutations in lexicographic order, and an exact dynamic program over
  *    subsets of processes.
+ *
+ *  - greedy relabeling (Sec. 6, "Max Weight Bipartite Perfect Matching": a
+ *    simple greedy algorithm, a 2-approximation): take the pairs (p, q) in
+ *    order of decreasing V[p][q] (ties: smaller p first, then smaller q) and
+ *    keep a pair when neither p nor q is matched yet; then give the target
+ *    labels left over, in increasing order, the processes left over, in
+ *    increasing order.
  */
 #include <math.h>
 #include <stdint.h>
@@ -340,6 +347,43 @@ int64_t oracle_lap_subset_dp(int P, const int64_t *V, int *sigma) {
     free(best);
     free(last);
     return result;
+}
+
+/* Greedy matching, as described in the header comment. */
+int64_t oracle_lap_greedy(int P, const int64_t *V, int *sigma) {
+    int64_t n = (int64_t)P * P;
+    int64_t *idx = (int64_t *)malloc(sizeof(int64_t) * (size_t)n);
+    char *used_p = (char *)calloc((size_t)P, 1), *used_q = (char *)calloc((size_t)P, 1);
+    if (!idx || !used_p || !used_q) { free(idx); free(used_p); free(used_q); return INT64_MIN; }
+    for (int64_t k = 0; k < n; k++) idx[k] = k;  /* k = p * P + q */
+    /* insertion of each pair into the sorted prefix (plain, O(n^2)) */
+    for (int64_t i = 1; i < n; i++) {
+        int64_t key = idx[i], j = i - 1;
+        while (j >= 0) {
+            int64_t a = idx[j];
+            int before = V[key] > V[a] || (V[key] == V[a] && key < a);
+            if (!before) break;
+            idx[j + 1] = a;
+            j--;
+        }
+        idx[j + 1] = key;
+    }
+    for (int q = 0; q < P; q++) sigma[q] = -1;
+    for (int64_t i = 0; i < n; i++) {
+        int p = (int)(idx[i] / P), q = (int)(idx[i] % P);
+        if (!used_p[p] && !used_q[q]) { used_p[p] = used_q[q] = 1; sigma[q] = p; }
+    }
+    int next_p = 0;
+    for (int q = 0; q < P; q++) {
+        if (sigma[q] >= 0) continue;
+        while (used_p[next_p]) next_p++;
+        sigma[q] = next_p;
+        used_p[next_p] = 1;
+    }
+    int64_t total = 0;
+    for (int q = 0; q < P; q++) total += V[(int64_t)sigma[q] * P + q];
+    free(idx); free(used_p); free(used_q);
+    return total;
 }
 
 int oracle_abi_version(void) { return 1; }

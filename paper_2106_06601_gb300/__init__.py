@@ -71,6 +71,8 @@ def _load():
         "costa_plan_stats_get": [I, P, P, P, I, P, P],
         "costa_release_plans": [],
         "costa_debug_axis_pieces": [P, P, I, I, P, I64, P],
+        "costa_volume_grid": [P, P, I, I, P],
+        "costa_relabel_greedy": [I, P, P, P],
         "costa_debug_tiles": [P, P, I, P, I64, P],
     }
     for name, args in sigs.items():
@@ -203,6 +205,53 @@ def costa_relabel(V):
     lv = ctypes.c_int64()
     _check(_lib.costa_relabel(P, _p(V), _p(sigma), ctypes.byref(lv)))
     return sigma, lv.value
+
+
+def costa_relabel_greedy(V):
+    """(sigma, local_volume) from the greedy 2-approximation (Sec. 6)."""
+    V = _i64(V)
+    P = V.shape[0]
+    sigma = np.zeros(P, dtype=np.int32)
+    lv = ctypes.c_int64()
+    _check(_lib.costa_relabel_greedy(P, _p(V), _p(sigma), ctypes.byref(lv)))
+    return sigma, lv.value
+
+
+class _GridDesc(ctypes.Structure):
+    _fields_ = [("nbr", ctypes.c_int), ("nbc", ctypes.c_int), ("row_splits", ctypes.c_void_p),
+                ("row_procs", ctypes.c_void_p), ("col_splits", ctypes.c_void_p),
+                ("col_procs", ctypes.c_void_p), ("pr", ctypes.c_int), ("pc", ctypes.c_int),
+                ("grid", ctypes.c_void_p)]
+
+
+class GridLayout:
+    """A process-grid layout without per-block arrays (costa_grid_desc)."""
+
+    def __init__(self, row_splits, row_procs, col_splits, col_procs, grid):
+        self.rs, self.cs = _i64(row_splits), _i64(col_splits)
+        self.rp, self.cp = _i32(row_procs), _i32(col_procs)
+        self.grid = _i32(grid)
+        assert self.grid.ndim == 2
+        self.desc = _GridDesc(len(self.rs) - 1, len(self.cs) - 1, self.rs.ctypes.data,
+                              self.rp.ctypes.data, self.cs.ctypes.data, self.cp.ctypes.data,
+                              self.grid.shape[0], self.grid.shape[1], self.grid.ctypes.data)
+
+    @staticmethod
+    def block_cyclic(m, n, mb, nb, pr, pc, grid_order="R", rank_perm=None):
+        rs = np.append(np.arange(0, m, mb, dtype=np.int64), m)
+        cs = np.append(np.arange(0, n, nb, dtype=np.int64), n)
+        ranks = np.arange(pr * pc).reshape(pr, pc) if grid_order == "R" else \
+            np.arange(pr * pc).reshape(pc, pr).T
+        if rank_perm is not None:
+            ranks = np.asarray(rank_perm)[ranks]
+        return GridLayout(rs, np.arange(len(rs) - 1) % pr, cs, np.arange(len(cs) - 1) % pc, ranks)
+
+
+def costa_volume_grid(A: GridLayout, B: GridLayout, op: str, P: int) -> np.ndarray:
+    """V[p, q] for process-grid layouts from 1-D overlaps (no device work)."""
+    V = np.zeros((P, P), dtype=np.int64)
+    _check(_lib.costa_volume_grid(ctypes.byref(A.desc), ctypes.byref(B.desc), OPS[op], P, _p(V)))
+    return V
 
 
 def _scalars(dtype: str, values) -> np.ndarray:

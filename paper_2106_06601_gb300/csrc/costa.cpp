@@ -25,6 +25,7 @@ namespace costa {
 
 int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
                    std::vector<int64_t> *u_out, std::vector<int64_t> *v_out);
+int64_t greedy_max(int P, const int64_t *V, std::vector<int> &sigma);
 
 namespace {
 
@@ -869,6 +870,18 @@ costa_status costa_relabel(int P, const int64_t *V, int *sigma, int64_t *local_v
     solve_relabel(P, V, sig, best);
     std::copy(sig.begin(), sig.end(), sigma);
     if (local_volume) *local_volume = best;
+    return COSTA_OK;
+}
+
+costa_status costa_relabel_greedy(int P, const int64_t *V, int *sigma, int64_t *local_volume) {
+    if (P < 1) return fail(COSTA_ERR_INVALID_ARG, "P %d < 1", P);
+    if (!V || !sigma) return fail(COSTA_ERR_INVALID_ARG, "null argument");
+    for (int64_t k = 0; k < static_cast<int64_t>(P) * P; ++k)
+        if (V[k] < 0) return fail(COSTA_ERR_INVALID_ARG, "negative volume at %lld", (long long)k);
+    std::vector<int> sig;
+    const int64_t total = greedy_max(P, V, sig);
+    std::copy(sig.begin(), sig.end(), sigma);
+    if (local_volume) *local_volume = total;
     return COSTA_OK;
 }
 

@@ -9,6 +9,7 @@
 // the alternating path.  After n insertions the matching is a minimum-cost
 // perfect assignment and (u, v) is a feasible dual solution whose objective
 // equals its cost (LP duality, the certificate of optimality).
+#include <algorithm>
 #include <cstdint>
 #include <limits>
 #include <vector>
@@ -73,6 +74,40 @@ int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &ro
     }
     if (u_out) u_out->assign(u.begin() + 1, u.end());
     if (v_out) v_out->assign(v.begin() + 1, v.end());
+    return total;
+}
+
+}  // namespace costa
+
+namespace costa {
+
+// Greedy maximum-weight matching (Sec. 6: "a simple greedy algorithm, which
+// is a 2-approximation"): pairs (p, q) by decreasing V[p][q], ties broken by
+// smaller p then smaller q; a pair is kept when p and q are both unmatched.
+// Target labels left unmatched take the unmatched processes, both in
+// increasing order.  sigma[q] = p.  Returns sum_q V[sigma[q]][q].
+int64_t greedy_max(int P, const int64_t *V, std::vector<int> &sigma) {
+    const int64_t n = static_cast<int64_t>(P) * P;
+    std::vector<int64_t> order(static_cast<size_t>(n));
+    for (int64_t k = 0; k < n; ++k) order[static_cast<size_t>(k)] = k;
+    std::stable_sort(order.begin(), order.end(), [V](int64_t a, int64_t b) { return V[a] > V[b]; });
+    std::vector<char> used_p(P, 0), used_q(P, 0);
+    sigma.assign(P, -1);
+    for (int64_t k : order) {
+        const int p = static_cast<int>(k / P), q = static_cast<int>(k % P);
+        if (used_p[p] || used_q[q]) continue;
+        used_p[p] = used_q[q] = 1;
+        sigma[q] = p;
+    }
+    int next = 0;
+    for (int q = 0; q < P; ++q) {
+        if (sigma[q] >= 0) continue;
+        while (used_p[next]) ++next;
+        sigma[q] = next;
+        used_p[next] = 1;
+    }
+    int64_t total = 0;
+    for (int q = 0; q < P; ++q) total += V[static_cast<int64_t>(sigma[q]) * P + q];
     return total;
 }
 
