@@ -238,6 +238,21 @@ costa_status costa_volume_grid(const costa_grid_desc *A, const costa_grid_desc *
  * Host only.  Errors: INVALID_ARG. */
 costa_status costa_relabel_greedy(int P, const int64_t *V, int *sigma, int64_t *local_volume);
 
+/* Relabeling under a general communication cost (Sec. 3): sending a package
+ * of volume v from process i to process j != i costs lat[i * P + j] +
+ * bw[i * P + j] * v (network topology: latency and bandwidth cost per element);
+ * local packages and empty packages cost nothing.  sigma (sigma[q] = process
+ * that takes target label q) minimizes the total cost W(G_sigma) of the
+ * relabeled communication graph (Def. COPR, Eq. WG).  Following Alg. 1 it is
+ * found as the assignment maximizing the total relabeling gain (Eq. delta,
+ * Thm. 1), solved exactly (Hungarian method on doubles, O(P^3)); the identity
+ * is kept when it is optimal.  cost_identity / cost_relabeled (nullable)
+ * receive W(G) and W(G_sigma).  With lat = 0 and bw = 1 off the diagonal this
+ * is costa_relabel's objective.  Host only.  Errors: INVALID_ARG (P < 1,
+ * null, negative V, non-finite costs). */
+costa_status costa_relabel_cost(int P, const int64_t *V, const double *lat, const double *bw, int *sigma,
+                                double *cost_identity, double *cost_relabeled);
+
 /* Diagnostics (host only, no device work): the pieces into which the plan
  * cuts one axis of A (axis 0 = rows, 1 = columns) for the pair (A, B, op).
  * Each piece is 6 int32: {A block index, op(B) block index, offset in A's

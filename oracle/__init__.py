@@ -70,6 +70,10 @@ def lib():
             _lib.oracle_lap_subset_dp.restype = ctypes.c_int64
             _lib.oracle_lap_greedy.argtypes = [ctypes.c_int, P, P]
             _lib.oracle_lap_greedy.restype = ctypes.c_int64
+            _lib.oracle_cost_W.argtypes = [ctypes.c_int, P, P, P, P]
+            _lib.oracle_cost_W.restype = ctypes.c_double
+            _lib.oracle_copr_bruteforce_cost.argtypes = [ctypes.c_int, P, P, P, P]
+            _lib.oracle_copr_bruteforce_cost.restype = ctypes.c_double
         return _lib
 
 
@@ -200,6 +204,27 @@ def lap_greedy(V: np.ndarray):
     sigma = np.zeros(P, dtype=np.int32)
     total = lib().oracle_lap_greedy(P, _ptr(V), _ptr(sigma))
     return int(total), sigma
+
+
+def cost_W(V, lat, bw, sigma) -> float:
+    """W(G_sigma) under w = lat + bw * volume for remote non-empty packages
+    (Def. RG, Eq. WG)."""
+    V = np.ascontiguousarray(V, dtype=np.int64)
+    lat = np.ascontiguousarray(lat, dtype=np.float64)
+    bw = np.ascontiguousarray(bw, dtype=np.float64)
+    sig = np.ascontiguousarray(sigma, dtype=np.int32)
+    return float(lib().oracle_cost_W(V.shape[0], _ptr(V), _ptr(lat), _ptr(bw), _ptr(sig)))
+
+
+def copr_bruteforce_cost(V, lat, bw):
+    """(min W(G_sigma), sigma) over all permutations (P <= 10), Def. COPR."""
+    V = np.ascontiguousarray(V, dtype=np.int64)
+    lat = np.ascontiguousarray(lat, dtype=np.float64)
+    bw = np.ascontiguousarray(bw, dtype=np.float64)
+    P = V.shape[0]
+    sigma = np.zeros(P, dtype=np.int32)
+    best = lib().oracle_copr_bruteforce_cost(P, _ptr(V), _ptr(lat), _ptr(bw), _ptr(sigma))
+    return float(best), sigma
 
 
 def lap_library(V: np.ndarray):

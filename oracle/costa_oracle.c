@@ -386,4 +386,41 @@ int64_t oracle_lap_greedy(int P, const int64_t *V, int *sigma) {
     return total;
 }
 
+/* Total cost W(G_sigma) of the relabeled communication graph (Def. RG,
+   Eq. WG) under the topology cost of Sec. 3: every non-empty package S_ij
+   (V[i][j] > 0) is sent from p_i to p_sigma(j) at cost
+   w = lat[i][k] + bw[i][k] * V[i][j] with k = sigma(j), or 0 when i == k. */
+double oracle_cost_W(int P, const int64_t *V, const double *lat, const double *bw, const int *sigma) {
+    double W = 0.0;
+    for (int i = 0; i < P; i++)
+        for (int j = 0; j < P; j++) {
+            int64_t v = V[(int64_t)i * P + j];
+            if (v == 0) continue;
+            int k = sigma[j];
+            if (k == i) continue;
+            W += lat[(int64_t)i * P + k] + bw[(int64_t)i * P + k] * (double)v;
+        }
+    return W;
+}
+
+/* COPR by definition (Def. COPR): the permutation of least W(G_sigma), over
+   all P! permutations in lexicographic order (the first minimum is kept). */
+double oracle_copr_bruteforce_cost(int P, const int64_t *V, const double *lat, const double *bw,
+                                   int *sigma) {
+    int perm[16];
+    if (P < 1 || P > 10) return -1.0;
+    for (int k = 0; k < P; k++) perm[k] = k;
+    double best = 0.0;
+    int first = 1;
+    do {
+        double W = oracle_cost_W(P, V, lat, bw, perm);
+        if (first || W < best) {
+            best = W;
+            memcpy(sigma, perm, sizeof(int) * (size_t)P);
+            first = 0;
+        }
+    } while (next_permutation(perm, P));
+    return best;
+}
+
 int oracle_abi_version(void) { return 1; }

@@ -73,6 +73,7 @@ def _load():
         "costa_debug_axis_pieces": [P, P, I, I, P, I64, P],
         "costa_volume_grid": [P, P, I, I, P],
         "costa_relabel_greedy": [I, P, P, P],
+        "costa_relabel_cost": [I, P, P, P, P, P, P],
         "costa_debug_tiles": [P, P, I, P, I64, P],
     }
     for name, args in sigs.items():
@@ -215,6 +216,20 @@ def costa_relabel_greedy(V):
     lv = ctypes.c_int64()
     _check(_lib.costa_relabel_greedy(P, _p(V), _p(sigma), ctypes.byref(lv)))
     return sigma, lv.value
+
+
+def costa_relabel_cost(V, lat, bw):
+    """(sigma, W(G), W(G_sigma)) under w = lat + bw * volume for remote packages."""
+    V = _i64(V)
+    P = V.shape[0]
+    lat = np.ascontiguousarray(lat, dtype=np.float64)
+    bw = np.ascontiguousarray(bw, dtype=np.float64)
+    assert lat.shape == (P, P) and bw.shape == (P, P)
+    sigma = np.zeros(P, dtype=np.int32)
+    c0, c1 = ctypes.c_double(), ctypes.c_double()
+    _check(_lib.costa_relabel_cost(P, _p(V), _p(lat), _p(bw), _p(sigma), ctypes.byref(c0),
+                                   ctypes.byref(c1)))
+    return sigma, c0.value, c1.value
 
 
 class _GridDesc(ctypes.Structure):

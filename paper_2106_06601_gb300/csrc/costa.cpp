@@ -26,6 +26,7 @@ namespace costa {
 int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
                    std::vector<int64_t> *u_out, std::vector<int64_t> *v_out);
 int64_t greedy_max(int P, const int64_t *V, std::vector<int> &sigma);
+double assign_min_f(int n, const std::vector<double> &cost, std::vector<int> &row_to_col);
 
 namespace {
 
@@ -870,6 +871,55 @@ costa_status costa_relabel(int P, const int64_t *V, int *sigma, int64_t *local_v
     solve_relabel(P, V, sig, best);
     std::copy(sig.begin(), sig.end(), sigma);
     if (local_volume) *local_volume = best;
+    return COSTA_OK;
+}
+
+// Relabeling under the topology cost of Sec. 3: w(i, j, s) = lat[i][j] +
+// bw[i][j] * V(s) for i != j, 0 for i == j, and nothing for empty packages.
+// As in Alg. 1 the weights are the gains of Eq. 3,
+//   delta(x, y) = sum over senders i of package S_ix of w(i, x, S_ix) - w(i, y, S_ix),
+// and sigma maximizes sum_x delta(x, sigma(x)) (Thm. 1), solved exactly as an
+// assignment on doubles.  By Lemma 1 this minimizes W(G_sigma).
+costa_status costa_relabel_cost(int P, const int64_t *V, const double *lat, const double *bw, int *sigma,
+                                double *cost_identity, double *cost_relabeled) {
+    if (P < 1) return fail(COSTA_ERR_INVALID_ARG, "P %d < 1", P);
+    if (!V || !lat || !bw || !sigma) return fail(COSTA_ERR_INVALID_ARG, "null argument");
+    const size_t PP = static_cast<size_t>(P) * P;
+    for (size_t k = 0; k < PP; ++k) {
+        if (V[k] < 0) return fail(COSTA_ERR_INVALID_ARG, "negative volume at %zu", k);
+        if (!std::isfinite(lat[k]) || !std::isfinite(bw[k]))
+            return fail(COSTA_ERR_INVALID_ARG, "non-finite cost at %zu", k);
+    }
+    auto w = [&](int i, int j, int64_t v) -> double {
+        if (v == 0 || i == j) return 0.0;
+        return lat[static_cast<size_t>(i) * P + j] + bw[static_cast<size_t>(i) * P + j] * static_cast<double>(v);
+    };
+    // C[x][y]: cost of the packages of target label x when process y takes it
+    std::vector<double> C(PP, 0.0);
+    for (int x = 0; x < P; ++x)
+        for (int y = 0; y < P; ++y) {
+            double c = 0.0;
+            for (int i = 0; i < P; ++i) c += w(i, y, V[static_cast<size_t>(i) * P + x]);
+            C[static_cast<size_t>(x) * P + y] = c;
+        }
+    // maximize sum delta(x, sigma(x)) with delta(x, y) = C[x][x] - C[x][y]:
+    // the same assignment as minimizing sum C[x][sigma(x)]
+    std::vector<double> cost(PP);
+    for (int x = 0; x < P; ++x)
+        for (int y = 0; y < P; ++y)
+            cost[static_cast<size_t>(x) * P + y] =
+                -(C[static_cast<size_t>(x) * P + x] - C[static_cast<size_t>(x) * P + y]);
+    std::vector<int> row_to_col;
+    assign_min_f(P, cost, row_to_col);
+    double ident = 0.0, best = 0.0;
+    for (int x = 0; x < P; ++x) {
+        ident += C[static_cast<size_t>(x) * P + x];
+        best += C[static_cast<size_t>(x) * P + row_to_col[x]];
+    }
+    const bool keep = ident <= best;  // tie rule: the identity when it is optimal
+    for (int x = 0; x < P; ++x) sigma[x] = keep ? x : row_to_col[x];
+    if (cost_identity) *cost_identity = ident;
+    if (cost_relabeled) *cost_relabeled = keep ? ident : best;
     return COSTA_OK;
 }
 

@@ -16,15 +16,17 @@
 
 namespace costa {
 
-// cost: row-major n x n.  row_to_col[i] receives the column assigned to row i.
+// cost: row-major n x n (integer or floating-point weights).  row_to_col[i]
+// receives the column assigned to row i.
 // Returns the minimum total cost.  u (n rows) and v (n columns) receive the
 // dual potentials when non-null: u[i] + v[j] <= cost[i][j] for all (i, j),
 // with equality on the assignment.
-int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
-                   std::vector<int64_t> *u_out, std::vector<int64_t> *v_out) {
-    const int64_t INF = std::numeric_limits<int64_t>::max() / 4;
+template <typename W>
+W assign_min_t(int n, const std::vector<W> &cost, std::vector<int> &row_to_col, std::vector<W> *u_out,
+               std::vector<W> *v_out) {
+    const W INF = std::numeric_limits<W>::max() / 4;
     // 1-based internally; column 0 is a virtual source column.
-    std::vector<int64_t> u(n + 1, 0), v(n + 1, 0), dist(n + 1);
+    std::vector<W> u(n + 1, 0), v(n + 1, 0), dist(n + 1);
     std::vector<int> col_row(n + 1, 0), prev(n + 1, 0);
     std::vector<char> done(n + 1);
     for (int i = 1; i <= n; ++i) {
@@ -35,12 +37,12 @@ int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &ro
         do {
             done[j0] = 1;
             const int i0 = col_row[j0];
-            int64_t delta = INF;
+            W delta = INF;
             int j1 = 0;
-            const int64_t *crow = cost.data() + static_cast<size_t>(i0 - 1) * n;
+            const W *crow = cost.data() + static_cast<size_t>(i0 - 1) * n;
             for (int j = 1; j <= n; ++j) {
                 if (done[j]) continue;
-                const int64_t red = crow[j - 1] - u[i0] - v[j];
+                const W red = crow[j - 1] - u[i0] - v[j];
                 if (red < dist[j]) {
                     dist[j] = red;
                     prev[j] = j0;
@@ -67,7 +69,7 @@ int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &ro
         } while (j0 != 0);
     }
     row_to_col.assign(n, -1);
-    int64_t total = 0;
+    W total = 0;
     for (int j = 1; j <= n; ++j) {
         row_to_col[col_row[j] - 1] = j - 1;
         total += cost[static_cast<size_t>(col_row[j] - 1) * n + (j - 1)];
@@ -75,6 +77,15 @@ int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &ro
     if (u_out) u_out->assign(u.begin() + 1, u.end());
     if (v_out) v_out->assign(v.begin() + 1, v.end());
     return total;
+}
+
+int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &row_to_col,
+                   std::vector<int64_t> *u_out, std::vector<int64_t> *v_out) {
+    return assign_min_t<int64_t>(n, cost, row_to_col, u_out, v_out);
+}
+
+double assign_min_f(int n, const std::vector<double> &cost, std::vector<int> &row_to_col) {
+    return assign_min_t<double>(n, cost, row_to_col, nullptr, nullptr);
 }
 
 }  // namespace costa
