@@ -253,6 +253,53 @@ costa_status costa_relabel_greedy(int P, const int64_t *V, int *sigma, int64_t *
 costa_status costa_relabel_cost(int P, const int64_t *V, const double *lat, const double *bw, int *sigma,
                                 double *cost_identity, double *cost_relabeled);
 
+/* ---- ScaLAPACK-style interface (Sec. 6: pxgemr2d and pxtran wrappers) ----
+ *
+ * A BLACS-like process grid of virtual ranks: nprow x npcol processes,
+ * numbered row-major ('R': rank = prow * npcol + pcol) or column-major
+ * ('C': rank = prow + pcol * nprow).  local[rank] is the device address of
+ * that rank's local matrix, column-major with leading dimension lld[rank]
+ * (lld NULL: every rank uses the descriptor's LLD). */
+typedef struct {
+    int nprow, npcol;
+    char order;
+    void *const *local;
+    const int64_t *lld;
+} costa_blacs_grid;
+
+/* Layout of the submatrix rows i..i+m-1, columns j..j+n-1 (1-based, as in
+ * ScaLAPACK) of a block-cyclic matrix with array descriptor
+ * desc = {DTYPE_ = 1, CTXT_ (ignored), M_, N_, MB_, NB_, RSRC_, CSRC_, LLD_}
+ * distributed over grid g: the global block grid truncated to the submatrix
+ * (Sec. 5), each block pointing into its owner's local matrix at the
+ * ScaLAPACK local indices (INDXG2L).  Host only; the layout borrows the local
+ * pointers.  Errors: INVALID_ARG, SHAPE (submatrix outside M_ x N_), LAYOUT
+ * (LLD below NUMROC rows, null local pointer), DTYPE. */
+costa_status costa_layout_create_scalapack(costa_layout *out, costa_dtype dt, const costa_blacs_grid *g,
+                                           int64_t i, int64_t j, int64_t m, int64_t n,
+                                           const int64_t *desc);
+
+/* sub(B) := sub(A), the m x n submatrices A(ia.., ja..) and B(ib.., jb..)
+ * (ScaLAPACK PxGEMR2D).  The two grids must have the same number of ranks.
+ * Asynchronous on stream like costa_transform; the first call with a given
+ * argument set builds and caches its layouts and plan (32 entries, least
+ * recently used evicted). */
+costa_status costa_pxgemr2d(costa_dtype dt, int64_t m, int64_t n, const costa_blacs_grid *ga, int64_t ia,
+                            int64_t ja, const int64_t *desca, const costa_blacs_grid *gb, int64_t ib,
+                            int64_t jb, const int64_t *descb, void *stream);
+
+/* sub(C) := beta * sub(C) + alpha * op(sub(A)), sub(C) m x n, sub(A) n x m,
+ * op = transpose (conjugate = 0: PxTRAN / PxTRANU) or conjugate transpose
+ * (conjugate != 0: PxTRANC).  alpha, beta: host scalars of dt.  Caching as
+ * costa_pxgemr2d. */
+costa_status costa_pxtran(costa_dtype dt, int conjugate, int64_t m, int64_t n, const void *alpha,
+                          const costa_blacs_grid *ga, int64_t ia, int64_t ja, const int64_t *desca,
+                          const void *beta, const costa_blacs_grid *gc, int64_t ic, int64_t jc,
+                          const int64_t *descc, void *stream);
+
+/* Frees the layouts (and plans) cached by costa_pxgemr2d / costa_pxtran. */
+costa_status costa_scalapack_release(void);
+
 /* Diagnostics (host only, no device work): the pieces into which the plan
  * cuts one axis of A (axis 0 = rows, 1 = columns) for the pair (A, B, op).
  * Each piece is 6 int32: {A block index, op(B) block index, offset in A's

@@ -74,6 +74,10 @@ def _load():
         "costa_volume_grid": [P, P, I, I, P],
         "costa_relabel_greedy": [I, P, P, P],
         "costa_relabel_cost": [I, P, P, P, P, P, P],
+        "costa_layout_create_scalapack": [P, I, P, I64, I64, I64, I64, P],
+        "costa_pxgemr2d": [I, I64, I64, P, I64, I64, P, P, I64, I64, P, P],
+        "costa_pxtran": [I, I, I64, I64, P, P, I64, I64, P, P, P, I64, I64, P, P],
+        "costa_scalapack_release": [],
         "costa_debug_tiles": [P, P, I, P, I64, P],
     }
     for name, args in sigs.items():
@@ -230,6 +234,57 @@ def costa_relabel_cost(V, lat, bw):
     _check(_lib.costa_relabel_cost(P, _p(V), _p(lat), _p(bw), _p(sigma), ctypes.byref(c0),
                                    ctypes.byref(c1)))
     return sigma, c0.value, c1.value
+
+
+class _BlacsGrid(ctypes.Structure):
+    _fields_ = [("nprow", ctypes.c_int), ("npcol", ctypes.c_int), ("order", ctypes.c_char),
+                ("local", ctypes.c_void_p), ("lld", ctypes.c_void_p)]
+
+
+class BlacsGrid:
+    """A grid of virtual ranks with one column-major local matrix each
+    (costa_blacs_grid): device addresses and leading dimensions per rank."""
+
+    def __init__(self, nprow: int, npcol: int, order: str, local_ptrs, lld=None):
+        P = nprow * npcol
+        self.ptrs = (ctypes.c_void_p * P)(*[int(x) for x in local_ptrs])
+        self.lld = None if lld is None else _i64(lld)
+        self.s = _BlacsGrid(nprow, npcol, order.encode(), ctypes.cast(self.ptrs, ctypes.c_void_p),
+                            None if self.lld is None else self.lld.ctypes.data)
+
+    def ref(self):
+        return ctypes.byref(self.s)
+
+
+def costa_layout_create_scalapack(dtype: str, grid: BlacsGrid, i: int, j: int, m: int, n: int,
+                                  desc) -> Layout:
+    d = _i64(desc)
+    out = ctypes.c_void_p()
+    _check(_lib.costa_layout_create_scalapack(ctypes.byref(out), DTYPES[dtype], grid.ref(), i, j,
+                                              m, n, _p(d)))
+    return Layout(out.value, dtype)
+
+
+def costa_pxgemr2d(dtype: str, m: int, n: int, ga: BlacsGrid, ia: int, ja: int, desca,
+                   gb: BlacsGrid, ib: int, jb: int, descb, stream: int = 0) -> None:
+    """sub(B) := sub(A) (ScaLAPACK PxGEMR2D; 1-based ia, ja, ib, jb)."""
+    da, db = _i64(desca), _i64(descb)
+    _check(_lib.costa_pxgemr2d(DTYPES[dtype], m, n, ga.ref(), ia, ja, _p(da), gb.ref(), ib, jb,
+                               _p(db), ctypes.c_void_p(stream)))
+
+
+def costa_pxtran(dtype: str, m: int, n: int, alpha, ga: BlacsGrid, ia: int, ja: int, desca, beta,
+                 gc: BlacsGrid, ic: int, jc: int, descc, conjugate: bool = False,
+                 stream: int = 0) -> None:
+    """sub(C) := beta sub(C) + alpha op(sub(A)), op = T (PxTRAN) or C (PxTRANC)."""
+    da, dc = _i64(desca), _i64(descc)
+    al, be = _scalars(dtype, [alpha]), _scalars(dtype, [beta])
+    _check(_lib.costa_pxtran(DTYPES[dtype], int(conjugate), m, n, _p(al), ga.ref(), ia, ja,
+                             _p(da), _p(be), gc.ref(), ic, jc, _p(dc), ctypes.c_void_p(stream)))
+
+
+def costa_scalapack_release() -> None:
+    _check(_lib.costa_scalapack_release())
 
 
 class _GridDesc(ctypes.Structure):

@@ -222,3 +222,57 @@ def random_splits(extent: int, nblocks: int, lo: int, hi: int, rng) -> np.ndarra
         if lo <= last <= hi:
             sizes.append(last)
             return _arr(np.concatenate([[0], np.cumsum(sizes)]), np.int64)
+
+
+def scalapack_full(M: int, N: int, MB: int, NB: int, RSRC: int, CSRC: int, pr: int, pc: int,
+                   order: str = "R", ld_pad: int = 0):
+    """Per-rank local matrix sizes (rows, cols, lld) of a ScaLAPACK
+    block-cyclic matrix whose first block sits on process (RSRC, CSRC);
+    ranks numbered row-major ("R") or column-major ("C")."""
+    out = []
+    for rank in range(pr * pc):
+        prow, pcol = (rank // pc, rank % pc) if order == "R" else (rank % pr, rank // pr)
+        rows = numroc(M, MB, prow, pr, RSRC)
+        cols = numroc(N, NB, pcol, pc, CSRC)
+        out.append((rows, cols, max(1, rows) + ld_pad))
+    return out
+
+
+def scalapack_sub(M: int, N: int, MB: int, NB: int, RSRC: int, CSRC: int, pr: int, pc: int,
+                  order: str, i: int, j: int, m: int, n: int, lld) -> LayoutSpec:
+    """The m x n submatrix at 1-based (i, j) of a ScaLAPACK block-cyclic
+    matrix as a LayoutSpec over the ranks' local matrices (buffer r = rank
+    r's column-major local matrix with leading dimension lld[r]).  Built
+    element-wise from the ScaLAPACK index maps: global row g lives on process
+    row (g div MB + RSRC) mod pr at local row MB (g div (MB pr)) + g mod MB."""
+    g_rows = np.arange(i - 1, i - 1 + m)
+    g_cols = np.arange(j - 1, j - 1 + n)
+    # blocks of the submatrix: maximal runs of rows (columns) in one global block
+    def runs(g, b):
+        if len(g) == 0:
+            return np.array([0], np.int64)
+        blk = g // b
+        cut = np.flatnonzero(np.diff(blk)) + 1
+        return np.concatenate([[0], cut, [len(g)]]).astype(np.int64)
+    R, C = runs(g_rows, MB), runs(g_cols, NB)
+    nbr, nbc = len(R) - 1, len(C) - 1
+    owner = np.zeros((nbr, nbc), np.int32)
+    off = np.zeros((nbr, nbc), np.int64)
+    ldm = np.zeros((nbr, nbc), np.int64)
+    for bi in range(nbr):
+        g = g_rows[R[bi]]
+        prow = (g // MB + RSRC) % pr
+        lr = MB * (g // (MB * pr)) + g % MB
+        for bj in range(nbc):
+            h = g_cols[C[bj]]
+            pcol = (h // NB + CSRC) % pc
+            lc = NB * (h // (NB * pc)) + h % NB
+            rank = prow * pc + pcol if order == "R" else prow + pcol * pr
+            owner[bi, bj] = rank
+            off[bi, bj] = lr + lc * lld[rank]
+            ldm[bi, bj] = lld[rank]
+    full = scalapack_full(M, N, MB, NB, RSRC, CSRC, pr, pc, order)
+    bufsize = np.array([max(1, lld[r]) * max(1, full[r][1]) for r in range(pr * pc)], np.int64)
+    return LayoutSpec(m, n, R, C, owner, pr * pc, owner.copy(), off, ldm,
+                      np.zeros((nbr, nbc), np.int32), bufsize, name="scalapack_sub",
+                      meta=dict(kind="scalapack_sub"))
