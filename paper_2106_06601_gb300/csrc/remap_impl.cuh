@@ -64,10 +64,16 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #define COSTA_WARPS_8 4
 #endif
 #ifndef COSTA_MINB_8
-#define COSTA_MINB_8 3
+#define COSTA_MINB_8 5
 #endif
 #ifndef COSTA_NBUF_8
-#define COSTA_NBUF_8 2
+#define COSTA_NBUF_8 1
+#endif
+#ifndef COSTA_MINB_8H
+#define COSTA_MINB_8H 3
+#endif
+#ifndef COSTA_NBUF_8H
+#define COSTA_NBUF_8H 2
 #endif
 #ifndef COSTA_WARPS_16
 #define COSTA_WARPS_16 8
@@ -93,13 +99,25 @@ template <typename T> struct Cfg {
     static constexpr int PITCH = TS + 1;
     static constexpr int BUF_BYTES_RAW = TS * PITCH * static_cast<int>(sizeof(T));
     static constexpr int BUF_BYTES = (BUF_BYTES_RAW + 127) / 128 * 128;
-    // Launch shape per element type (measured on GB300): warps per block,
-    // resident blocks per SM the registers must allow, and shared-memory
-    // buffers per warp (the warp keeps NBUF - 1 tiles' copies in flight ahead
-    // of the tile it writes).  Overridable at build time for tuning.
     static constexpr int WARPS = sizeof(T) == 4 ? COSTA_WARPS_4 : sizeof(T) == 16 ? COSTA_WARPS_16 : COSTA_WARPS_8;
-    static constexpr int MINB = sizeof(T) == 4 ? COSTA_MINB_4 : sizeof(T) == 16 ? COSTA_MINB_16 : COSTA_MINB_8;
-    static constexpr int NBUF = sizeof(T) == 4 ? COSTA_NBUF_4 : sizeof(T) == 16 ? COSTA_NBUF_16 : COSTA_NBUF_8;
+};
+
+// Launch shape per element type and combine kind (measured on GB300): warps
+// per block, resident blocks per SM the registers must allow, and
+// shared-memory buffers per warp (the warp keeps NBUF - 1 tiles' copies in
+// flight ahead of the tile it writes).  8-byte types with the light kinds
+// run more warps without look-ahead; the general kinds (non-power-of-two
+// beta, complex scalars) need the registers of 3 blocks and use a 2-deep
+// ring.  Overridable at build time for tuning.
+template <typename T, int KIND> struct KCfg {
+    static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX;
+    static constexpr int WARPS = Cfg<T>::WARPS;
+    static constexpr int MINB = sizeof(T) == 4 ? COSTA_MINB_4
+                              : sizeof(T) == 16 ? COSTA_MINB_16
+                              : HEAVY ? COSTA_MINB_8H : COSTA_MINB_8;
+    static constexpr int NBUF = sizeof(T) == 4 ? COSTA_NBUF_4
+                              : sizeof(T) == 16 ? COSTA_NBUF_16
+                              : HEAVY ? COSTA_NBUF_8H : COSTA_NBUF_8;
 };
 
 template <typename T> struct Chunk {
@@ -558,9 +576,10 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
 }
 
 template <typename T, int KIND>
-__global__ void __launch_bounds__(Cfg<T>::WARPS * 32, Cfg<T>::MINB) remap_kernel(const RemapLaunch args) {
+__global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB)
+    remap_kernel(const RemapLaunch args) {
     using C = Cfg<T>;
-    constexpr int NB = C::NBUF;
+    constexpr int NB = KCfg<T, KIND>::NBUF;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     unsigned char *bufs = smem_raw + warp * NB * C::BUF_BYTES;
@@ -577,8 +596,17 @@ __global__ void __launch_bounds__(Cfg<T>::WARPS * 32, Cfg<T>::MINB) remap_kernel
 
     // ring[0] is the tile being written, ring[k] the tile k ahead, staged in
     // buffer (cur + k) % NB
-    Geom<T> ring[NB];
-    bool have[NB];
+    if constexpr (NB == 1) {  // no look-ahead: copy, wait, write, one tile at a time
+        Geom<T> g;
+        while (next_tile<T, KIND>(args, first, stride, ts, g, lane)) {
+            if (g.fast) stage_issue<T>(g, bufs, lane);
+            cp_async_commit();
+            write_tile<T, KIND, 1>(args, g, s, cached, bufs, lane);
+        }
+        return;
+    }
+    Geom<T> ring[NB > 1 ? NB : 2];
+    bool have[NB > 1 ? NB : 2];
 #pragma unroll
     for (int k = 0; k < NB - 1; ++k) {
         have[k] = (k == 0 || have[k - 1]) && next_tile<T, KIND>(args, first, stride, ts, ring[k], lane);
@@ -586,16 +614,16 @@ __global__ void __launch_bounds__(Cfg<T>::WARPS * 32, Cfg<T>::MINB) remap_kernel
         cp_async_commit();
     }
     int cur = 0;
+    constexpr int LA = NB > 1 ? NB - 1 : 1;  // index of the look-ahead slot
     while (have[0]) {
-        have[NB - 1] = have[NB - 2] && next_tile<T, KIND>(args, first, stride, ts, ring[NB - 1], lane);
+        have[LA] = have[LA - 1] && next_tile<T, KIND>(args, first, stride, ts, ring[LA], lane);
         int ahead = cur + NB - 1;
         if (ahead >= NB) ahead -= NB;
-        if (have[NB - 1] && ring[NB - 1].fast)
-            stage_issue<T>(ring[NB - 1], bufs + ahead * C::BUF_BYTES, lane);
+        if (have[LA] && ring[LA].fast) stage_issue<T>(ring[LA], bufs + ahead * C::BUF_BYTES, lane);
         cp_async_commit();
         write_tile<T, KIND, NB>(args, ring[0], s, cached, bufs + cur * C::BUF_BYTES, lane);
 #pragma unroll
-        for (int k = 0; k < NB - 1; ++k) {
+        for (int k = 0; k < LA; ++k) {
             ring[k] = ring[k + 1];
             have[k] = have[k + 1];
         }
@@ -619,7 +647,7 @@ template <typename T, int KIND>
 cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     auto kern = remap_kernel<T, KIND>;
     constexpr int kWarps = Cfg<T>::WARPS;
-    const size_t smem = static_cast<size_t>(kWarps) * Cfg<T>::NBUF * Cfg<T>::BUF_BYTES;
+    const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND>::NBUF * Cfg<T>::BUF_BYTES;
     static int per_sm = 0;
     if (per_sm == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
