@@ -45,7 +45,9 @@ def _stale(objs_and_srcs) -> bool:
     return any(os.path.getmtime(s) > t for s in objs_and_srcs)
 
 
-def build(force: bool = False, verbose: bool = False, extra_nvcc=()) -> str:
+def build(force: bool = False, verbose: bool = False, extra_nvcc=(), defines=()) -> str:
+    """Compiles every translation unit and links the library.  `defines`
+    (-DNAME=VALUE) go to both compilers (tuning overrides)."""
     os.makedirs(BUILD, exist_ok=True)
     cu, cpp, hdr = sources()
     deps = [os.path.join(CSRC, f) for f in cu + cpp + hdr] + [os.path.join(INCLUDE, "costa_gb300.h"),
@@ -59,14 +61,14 @@ def build(force: bool = False, verbose: bool = False, extra_nvcc=()) -> str:
     for f in cu:
         obj = os.path.join(BUILD, f + ".o")
         cmd = [nvcc, *ARCH, "-lineinfo", "-O3", "-std=c++17", "-Xcompiler", "-fPIC",
-               "-Xptxas", "-v" if verbose else "-O3", *extra_nvcc, *incs,
+               "-Xptxas", "-v" if verbose else "-O3", *extra_nvcc, *defines, *incs,
                "-c", os.path.join(CSRC, f), "-o", obj]
         jobs.append((cmd, f))
         objs.append(obj)
     for f in cpp:
         obj = os.path.join(BUILD, f + ".o")
         cmd = ["g++", "-O2", "-std=c++17", "-fPIC", "-Wall", "-Wextra", "-Wno-unused-parameter",
-               *incs, "-I", os.path.join(cuda, "include"), "-c", os.path.join(CSRC, f), "-o", obj]
+               *defines, *incs, "-I", os.path.join(cuda, "include"), "-c", os.path.join(CSRC, f), "-o", obj]
         jobs.append((cmd, f))
         objs.append(obj)
     procs = [(subprocess.Popen(c, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True), f)

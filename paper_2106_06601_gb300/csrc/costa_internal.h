@@ -139,8 +139,12 @@ struct VolumeLaunch {
     unsigned long long *V;      // P * P, zeroed by the caller
 };
 
-// Tile extent (elements along each axis of A) for an element size.
-inline int tile_extent(int esize) { return esize == 16 ? 16 : 32; }
+// Tile extent (elements along each axis of A) for an element size; shared
+// by the planner and the kernels.
+#ifndef COSTA_TS_16
+#define COSTA_TS_16 32
+#endif
+COSTA_HD constexpr int tile_extent(int esize) { return esize == 16 ? COSTA_TS_16 : 32; }
 
 // Launches the remap kernel for (args.dtype, kind) over a tile list.  With
 // args.per_problem set, the kernel skips the tiles of problems of another kind.

@@ -76,13 +76,13 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #define COSTA_NBUF_8H 2
 #endif
 #ifndef COSTA_WARPS_16
-#define COSTA_WARPS_16 8
+#define COSTA_WARPS_16 4
 #endif
 #ifndef COSTA_MINB_16
 #define COSTA_MINB_16 1
 #endif
 #ifndef COSTA_NBUF_16
-#define COSTA_NBUF_16 3
+#define COSTA_NBUF_16 2
 #endif
 
 // Per element type: tile extent TS, 16-byte chunk width VEC (elements), and
@@ -91,7 +91,7 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 // CPR chunks (TS * TS elements); the element-wise path uses a TS x (TS + 1)
 // array in the same buffer.
 template <typename T> struct Cfg {
-    static constexpr int TS = sizeof(T) == 16 ? 16 : 32;
+    static constexpr int TS = tile_extent(static_cast<int>(sizeof(T)));
     static constexpr int VEC = ET<T>::VEC;
     static constexpr int CPR = TS / VEC;
     static constexpr int RPP = 32 / CPR;

@@ -22,7 +22,7 @@ def _layout(spec, dtype):
 
 def check_pair(p):
     LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
-    ts = 16 if p.dtype == "c128" else 32
+    ts = 32  # tile extent of every element type
     try:
         for axis in (0, 1):
             pc = costa.costa_debug_axis_pieces(LA, LB, p.op, axis).astype(np.int64)
