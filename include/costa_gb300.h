@@ -354,6 +354,21 @@ const char *costa_last_error(void);
 /* Number of kernels this library has launched in this process. */
 int64_t costa_kernel_launch_count(void);
 
+/* Per-phase device time of transform calls (diagnostic).  While enabled
+ * (enable != 0; process-wide, off at load), every costa_transform* call
+ * records CUDA events on its stream around its phases: the remap launches in
+ * direct mode (1 phase); pack, local remap and unpack in message mode (3
+ * phases: Alg. 3 and Sec. 6, packing, the blocks that stay local, unpacking
+ * with the transform).  The events add no synchronization to the call. */
+costa_status costa_phase_timing(int enable);
+
+/* Waits for the events of the last timed transform call on the calling
+ * host thread's current device and writes its phase durations in
+ * milliseconds to ms[0 .. *nphases - 1] (ms: host array of 3 doubles).
+ * COSTA_ERR_INVALID_ARG if no call has been timed since timing was enabled,
+ * or if the last timed call had no tiles. */
+costa_status costa_phase_times(double *ms, int *nphases);
+
 /* ABI version of this header (1). */
 int costa_abi_version(void);
 

@@ -79,6 +79,8 @@ def _load():
         "costa_pxtran": [I, I, I64, I64, P, P, I64, I64, P, P, P, I64, I64, P, P],
         "costa_scalapack_release": [],
         "costa_debug_tiles": [P, P, I, P, I64, P],
+        "costa_phase_timing": [I],
+        "costa_phase_times": [P, P],
     }
     for name, args in sigs.items():
         f = getattr(lib, name)
@@ -381,6 +383,21 @@ def costa_kernel_launch_count() -> int:
 
 def costa_abi_version() -> int:
     return _lib.costa_abi_version()
+
+
+def costa_phase_timing(enable: bool) -> None:
+    """Turns per-phase CUDA-event timing of transform calls on or off."""
+    _check(_lib.costa_phase_timing(int(bool(enable))))
+
+
+def costa_phase_times() -> list:
+    """Device milliseconds of the phases of the last timed transform call on
+    the current device: [remap] (direct mode) or [pack, local, unpack]
+    (message mode).  Waits for that call's events."""
+    ms = (ctypes.c_double * 3)()
+    n = ctypes.c_int(0)
+    _check(_lib.costa_phase_times(ms, ctypes.byref(n)))
+    return [ms[k] for k in range(n.value)]
 
 
 def costa_layout_from_spec(spec, dtype: str, block_ptrs) -> Layout:

@@ -177,6 +177,36 @@ struct Plan {
 std::mutex g_mu;
 std::map<std::vector<uint64_t>, std::unique_ptr<Plan>> g_plans;
 
+// Phase timing (costa_phase_timing): CUDA events per device, recorded by
+// transform calls around their phases.  Guarded by g_mu.
+struct PhaseTimer {
+    cudaEvent_t ev[4] = {};
+    int nphases = 0;  // phases of the last timed call (0: none yet)
+};
+std::atomic<bool> g_phase_on{false};
+std::map<int, PhaseTimer> g_timers;
+
+// The timer of the current device with its events created, or null.
+PhaseTimer *phase_timer(costa_status &st) {
+    st = COSTA_OK;
+    int dev = 0;
+    cudaError_t ce = cudaGetDevice(&dev);
+    if (ce != cudaSuccess) {
+        st = cuda_fail(ce, "cudaGetDevice");
+        return nullptr;
+    }
+    PhaseTimer &t = g_timers[dev];
+    for (cudaEvent_t &e : t.ev) {
+        if (e) continue;
+        ce = cudaEventCreate(&e);
+        if (ce != cudaSuccess) {
+            st = cuda_fail(ce, "cudaEventCreate");
+            return nullptr;
+        }
+    }
+    return &t;
+}
+
 bool plan_uses(const std::vector<uint64_t> &key, uint64_t id) {
     // key = [device, n, (A.id, B.id, op) x n]
     for (size_t i = 2; i + 1 < key.size(); i += 3)
@@ -610,7 +640,15 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     }
     if (sigma_out)
         for (int q = 0; q < P; ++q) sigma_out[q] = relabel ? plan->sigma[q] : q;
+    PhaseTimer *timer = nullptr;
+    if (g_phase_on.load()) {
+        timer = phase_timer(s);
+        if (!timer) return s;
+        timer->nphases = 0;
+    }
     if (plan->total_tiles == 0) return COSTA_OK;
+    // event k marks the end of phase k (event 0: the start)
+    auto mark = [&](int k) -> cudaError_t { return timer ? cudaEventRecord(timer->ev[k], stream) : cudaSuccess; };
 
     RemapLaunch L{};
     L.tiles = plan->d_tiles;
@@ -653,8 +691,11 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     };
     cudaError_t ce;
     if (mode == COSTA_MODE_DIRECT) {
-        ce = launch_list(plan->d_tiles, plan->total_tiles);
+        ce = mark(0);
+        if (ce == cudaSuccess) ce = launch_list(plan->d_tiles, plan->total_tiles);
+        if (ce == cudaSuccess) ce = mark(1);
         if (ce != cudaSuccess) return cuda_fail(ce, "remap kernel launch");
+        if (timer) timer->nphases = 1;
         return COSTA_OK;
     }
     s = ensure_message(*plan, relabel != 0);
@@ -670,12 +711,17 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     const bool single = plan->dtype == COSTA_F32 || plan->dtype == COSTA_C64;
     lp.s = make_scalars(plan->dtype, single ? static_cast<const void *>(one_f) : one_d,
                         single ? static_cast<const void *>(zero_f) : zero_d, 0);
-    ce = launch_remap(lp, K_COPY, stream);
+    ce = mark(0);
+    if (ce == cudaSuccess) ce = launch_remap(lp, K_COPY, stream);
+    if (ce == cudaSuccess) ce = mark(1);
     if (ce != cudaSuccess) return cuda_fail(ce, "pack kernel launch");
     ce = launch_list(m.local, m.n_local);
+    if (ce == cudaSuccess) ce = mark(2);
     if (ce != cudaSuccess) return cuda_fail(ce, "local remap kernel launch");
     ce = launch_list(m.unpack, m.n_unpack);
+    if (ce == cudaSuccess) ce = mark(3);
     if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
+    if (timer) timer->nphases = 3;
     return COSTA_OK;
 }
 
@@ -1028,6 +1074,30 @@ costa_status costa_release_plans(void) {
 const char *costa_last_error(void) { return g_err.c_str(); }
 
 int64_t costa_kernel_launch_count(void) { return launches_so_far(); }
+
+costa_status costa_phase_timing(int enable) {
+    g_phase_on.store(enable != 0);
+    return COSTA_OK;
+}
+
+costa_status costa_phase_times(double *ms, int *nphases) {
+    if (!ms || !nphases) return fail(COSTA_ERR_INVALID_ARG, "null argument");
+    std::lock_guard<std::mutex> lock(g_mu);
+    costa_status st;
+    PhaseTimer *t = phase_timer(st);
+    if (!t) return st;
+    if (t->nphases == 0) return fail(COSTA_ERR_INVALID_ARG, "no timed transform call with tiles on this device");
+    cudaError_t ce = cudaEventSynchronize(t->ev[t->nphases]);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaEventSynchronize");
+    for (int k = 0; k < t->nphases; ++k) {
+        float f = 0.0f;
+        ce = cudaEventElapsedTime(&f, t->ev[k], t->ev[k + 1]);
+        if (ce != cudaSuccess) return cuda_fail(ce, "cudaEventElapsedTime");
+        ms[k] = f;
+    }
+    *nphases = t->nphases;
+    return COSTA_OK;
+}
 
 int costa_abi_version(void) { return 1; }
 

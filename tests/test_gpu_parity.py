@@ -221,3 +221,39 @@ def test_special_values_power_of_two_beta(dtype, beta, dev):
             assert np.all(ok), (np.flatnonzero(~ok)[:5], got.arena[~ok][:5], want.arena[~ok][:5])
     finally:
         g.close()
+
+
+def test_phase_timing(dev):
+    """Phase events: one phase in direct mode, pack/local/unpack in message
+    mode; results are unchanged by the timing; a call with no tiles leaves
+    nothing to read."""
+    import paper_2106_06601_gb300 as costa
+    p = C.fuzz_problem(11, dtype="f64", P=4)
+    g = OnDevice(p, dev)
+    costa.costa_phase_timing(True)
+    try:
+        g.run(mode="direct")
+        d = costa.costa_phase_times()
+        assert len(d) == 1 and d[0] > 0
+        want = g.oracle_result()
+        compare(p, g.Ad.download(), want, g.Ah, g.Bh)
+        g.reset_A()
+        g.run(mode="message")
+        m = costa.costa_phase_times()
+        assert len(m) == 3 and min(m) >= 0 and sum(m) > 0
+        compare(p, g.Ad.download(), want, g.Ah, g.Bh)
+        # an empty matrix records no phases
+        A = L.packed_blocks([0], [0, 5], np.zeros((0, 1), np.int32), 2)
+        B = L.packed_blocks([0, 5], [0], np.zeros((1, 0), np.int32), 2)
+        LA = costa.costa_layout_create("f64", 2, A.rsplit, A.csplit, A.owner, np.zeros((0, 1)),
+                                       A.ld, A.order)
+        LB = costa.costa_layout_create("f64", 2, B.rsplit, B.csplit, B.owner, np.zeros((1, 0)),
+                                       B.ld, B.order)
+        costa.costa_transform(LA, LB, "T", 1.0, 0.0)
+        with pytest.raises(costa.CostaError):
+            costa.costa_phase_times()
+        LA.destroy()
+        LB.destroy()
+    finally:
+        costa.costa_phase_timing(False)
+        g.close()
