@@ -337,7 +337,7 @@ costa_status costa_volume_noalloc(costa_layout A, costa_layout B, costa_op op, i
                                   void *stream);
 
 /* Diagnostics (host only, no device work): the remap kernel's tile list for
- * (A, B, op) in direct mode.  Each tile is 32 bytes: {source address, target
+ * (A, B, op) in direct mode, in the order the kernel's warps take the tiles.  Each tile is 32 bytes: {source address, target
  * address (uint64), source stride, target stride (int32), nx, ny, problem,
  * flags (uint16)}, in the frame where x runs along A's contiguous axis
  * (flags: 1 = transposed, 2 = vector path, 4 = conjugate).  Writes

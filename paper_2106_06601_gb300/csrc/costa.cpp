@@ -312,6 +312,124 @@ template <typename F> void for_each_tile(const ProblemHost &ph, F &&f) {
                 for (int u = su; u < std::min(su + kSuper, nu); ++u) f(ph.rows.tiles[u], ph.cols.tiles[v]);
 }
 
+// Tile order in the target's own storage.  For a transposed problem (op = T
+// or C) the source tiles that warps read at the same time are scattered
+// across the source whatever the order, so the order serves the target,
+// which is read and written: each target buffer is walked in strips of
+// kLocalStrip tiles across its non-contiguous axis, each strip down the
+// buffer's contiguous axis, so that concurrent tiles form long contiguous
+// runs of target memory.  Measured on GB300: +6.6% on 16384^2 c128 (C) and
+// +2% on 8192^2 f64 (T); no gain for 4-byte elements (32 x 32 f32 tiles) and
+// a loss for op = N, whose source runs the global order keeps.  The
+// environment variable COSTA_TILE_ORDER (global | local) overrides the rule,
+// for tuning.
+constexpr int kLocalStrip = 2;
+
+bool use_local_order(const ProblemHost &ph) {
+    static const int env = [] {
+        const char *e = std::getenv("COSTA_TILE_ORDER");
+        if (!e) return -1;
+        if (std::strcmp(e, "global") == 0) return 0;
+        if (std::strcmp(e, "local") == 0) return 1;
+        return -1;
+    }();
+    if (env >= 0) return env == 1;
+    return ph.op != COSTA_OP_N && esize_of(ph.A->dt) >= 8;
+}
+
+// Stable LSD radix sort of (key, index) pairs by key, 11 bits per pass (the
+// counts and the scatter targets stay in cache); passes stop at the highest
+// bit in which two keys differ, and a pass whose digit is equal for every
+// key is skipped.
+void radix_sort_pairs(std::vector<std::pair<uint64_t, uint32_t>> &v) {
+    constexpr int kBits = 11, kBuckets = 1 << kBits;
+    std::vector<std::pair<uint64_t, uint32_t>> tmp(v.size());
+    std::vector<size_t> count(kBuckets + 1);
+    uint64_t lo = ~uint64_t(0), hi = 0;
+    for (const auto &e : v) {
+        lo = std::min(lo, e.first);
+        hi = std::max(hi, e.first);
+    }
+    for (int shift = 0; shift < 64; shift += kBits) {
+        if (((lo ^ hi) >> shift) == 0) break;  // keys agree on every higher bit
+        std::fill(count.begin(), count.end(), size_t(0));
+        for (const auto &e : v) ++count[((e.first >> shift) & (kBuckets - 1)) + 1];
+        bool uniform = false;
+        for (int d = 1; d <= kBuckets; ++d)
+            if (count[d] == v.size()) uniform = true;
+        if (uniform) continue;
+        for (int d = 1; d <= kBuckets; ++d) count[d] += count[d - 1];
+        for (const auto &e : v) tmp[count[(e.first >> shift) & (kBuckets - 1)]++] = e;
+        v.swap(tmp);
+    }
+}
+
+// Reorders tiles [first, last) (one problem) into the target-local order.
+// Tiles are grouped by target stride; within a group an element's local
+// coordinates are taken from its offset to the group's lowest target
+// address: y = offset / stride (the non-contiguous axis), then strips of
+// kLocalStrip * ts along y, ordered by address inside each strip.
+void order_tiles_local(std::vector<TileDesc> &list, size_t first, size_t last, int es, int ts) {
+    const size_t n = last - first;
+    if (n < 2) return;
+    std::vector<std::pair<int32_t, uint64_t>> groups;  // (stride, lowest target address)
+    std::vector<uint32_t> gid(n);
+    for (size_t i = 0; i < n; ++i) {
+        const TileDesc &d = list[first + i];
+        size_t g = 0;
+        while (g < groups.size() && groups[g].first != d.dld) ++g;
+        if (g == groups.size()) groups.emplace_back(d.dld, d.dst);
+        else groups[g].second = std::min(groups[g].second, d.dst);
+        gid[i] = static_cast<uint32_t>(g);
+    }
+    const uint64_t strip_elems = static_cast<uint64_t>(kLocalStrip) * static_cast<uint64_t>(ts);
+    int es_shift = 0;
+    while ((1 << es_shift) < es) ++es_shift;
+    std::vector<std::pair<uint64_t, uint32_t>> keys(n);
+    std::vector<uint64_t> off(n);
+    uint64_t max_strip = 0;
+    for (size_t i = 0; i < n; ++i) {
+        const TileDesc &d = list[first + i];
+        off[i] = (d.dst - groups[gid[i]].second) >> es_shift;
+        keys[i] = {off[i] / (static_cast<uint64_t>(d.dld) * strip_elems), static_cast<uint32_t>(i)};
+        max_strip = std::max(max_strip, keys[i].first);
+    }
+    // key = group * (max_strip + 1) + strip, so that the sort needs only the
+    // bits the keys span
+    const uint64_t span = max_strip + 1;
+    if (groups.size() > 1 && span <= ~uint64_t(0) / groups.size())
+        for (size_t i = 0; i < n; ++i) keys[i].first += gid[keys[i].second] * span;
+    radix_sort_pairs(keys);
+    // inside each strip, by target address
+    for (size_t a = 0; a < n;) {
+        size_t b = a + 1;
+        while (b < n && keys[b].first == keys[a].first) ++b;
+        std::sort(keys.begin() + static_cast<std::ptrdiff_t>(a), keys.begin() + static_cast<std::ptrdiff_t>(b),
+                  [&](const std::pair<uint64_t, uint32_t> &x, const std::pair<uint64_t, uint32_t> &y) {
+                      return off[x.second] < off[y.second];
+                  });
+        a = b;
+    }
+    std::vector<TileDesc> tmp(n);
+    for (size_t k = 0; k < n; ++k) tmp[k] = list[first + keys[k].second];
+    std::copy(tmp.begin(), tmp.end(), list.begin() + static_cast<std::ptrdiff_t>(first));
+}
+
+// Appends the direct tiles of problem `prob` in the kernel's order.
+void append_direct_tiles(const ProblemHost &ph, int prob, int es, int ts, std::vector<TileDesc> &list) {
+    const size_t first = list.size();
+    for_each_tile(ph, [&](const AxisTile &rt, const AxisTile &ct) {
+        TileDesc d = direct_tile(ph, rt, ct, es, prob);
+        set_fast(d, es);
+        list.push_back(d);
+    });
+    if (!use_local_order(ph)) return;
+    // a target whose tiles are each one contiguous run gains nothing
+    bool contiguous = true;
+    for (size_t i = first; i < list.size() && contiguous; ++i) contiguous = list[i].nx == list[i].dld;
+    if (!contiguous) order_tiles_local(list, first, list.size(), es, ts);
+}
+
 // Builds the overlay, the tile list and the device tables, and runs the
 // volume kernel.
 costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, const costa_op *ops,
@@ -350,13 +468,7 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     // the direct tile list, in (problem, row piece, column piece) order
     std::vector<TileDesc> list;
     list.reserve(static_cast<size_t>(tiles));
-    for (int k = 0; k < n; ++k) {
-        for_each_tile(plan->probs[k], [&](const AxisTile &rt, const AxisTile &ct) {
-            TileDesc d = direct_tile(plan->probs[k], rt, ct, es, k);
-            set_fast(d, es);
-            list.push_back(d);
-        });
-    }
+    for (int k = 0; k < n; ++k) append_direct_tiles(plan->probs[k], k, es, ts, list);
     const size_t off_tiles = arena.add_vec(list);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
@@ -1054,14 +1166,11 @@ costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void
     ph.rows = cut_pair_axis(A, B, op, 0, ts);
     ph.cols = cut_pair_axis(A, B, op, 1, ts);
     *count = static_cast<int64_t>(ph.rows.tiles.size()) * static_cast<int64_t>(ph.cols.tiles.size());
-    int64_t k = 0;
-    TileDesc *o = static_cast<TileDesc *>(out);
-    for_each_tile(ph, [&](const AxisTile &rt, const AxisTile &ct) {
-        if (k >= cap) return;
-        TileDesc d = direct_tile(ph, rt, ct, es, 0);
-        set_fast(d, es);
-        o[k++] = d;
-    });
+    std::vector<TileDesc> list;
+    list.reserve(static_cast<size_t>(*count));
+    append_direct_tiles(ph, 0, es, ts, list);
+    const size_t k = static_cast<size_t>(std::min<int64_t>(cap, *count));
+    if (k) std::memcpy(out, list.data(), k * sizeof(TileDesc));
     return COSTA_OK;
 }
 

@@ -109,3 +109,76 @@ def test_fuzz_pieces_in_bounds():
     for case in range(400):
         check_pair(C.fuzz_problem(case))
         check_tiles(C.fuzz_problem(case))
+
+
+def _tile_dst(p, rows, cols, u, v):
+    """Target address of tile (row piece u, column piece v) from the layout
+    spec (independent of the library's tile construction)."""
+    es = {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[p.dtype]
+    bi, bj = rows[u, 0], cols[v, 0]
+    r, c = rows[u, 2].astype(np.int64), cols[v, 2].astype(np.int64)
+    A = p.A
+    ptr = FAKE + A.buf[bi, bj].astype(np.int64) * (1 << 32) + A.off[bi, bj] * es
+    ld = A.ld[bi, bj]
+    local = np.where(A.order[bi, bj] == 0, r + c * ld, r * ld + c)
+    return (ptr + local * es).astype(np.uint64)
+
+
+def check_order(p):
+    """The kernel's tile order.  Transposed problems of 8- and 16-byte
+    elements whose target tiles are not each one contiguous run walk each
+    target buffer in strips of 2 tiles (64 elements) across its
+    non-contiguous axis, by address inside a strip, one target stride group
+    after another; the others follow the global super-tile order
+    (k x k pieces, k = 16 for 16-byte elements and 8 otherwise, row pieces
+    fastest).  Either way the list is a permutation of the product of the
+    row and column pieces."""
+    es = {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[p.dtype]
+    LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+    try:
+        t = costa.costa_debug_tiles(LA, LB, p.op)
+        rows = costa.costa_debug_axis_pieces(LA, LB, p.op, 0)
+        cols = costa.costa_debug_axis_pieces(LA, LB, p.op, 1)
+    finally:
+        LA.destroy()
+        LB.destroy()
+    nu, nv = len(rows), len(cols)
+    if nu * nv == 0:
+        assert len(t) == 0
+        return
+    u, v = np.meshgrid(np.arange(nu), np.arange(nv), indexing="ij")
+    u, v = u.ravel(), v.ravel()
+    k = 16 if es == 16 else 8
+    glob = np.lexsort((u, v, v // k, u // k))  # last key is the primary one
+    want = _tile_dst(p, rows, cols, u[glob], v[glob])
+    dst = t["dst"].astype(np.uint64)
+    assert np.array_equal(np.sort(dst), np.sort(want))
+    assert len(np.unique(dst)) == len(dst)
+    contiguous = np.all(t["nx"].astype(np.int64) == t["dld"].astype(np.int64))
+    if p.op == "N" or es < 8 or contiguous:
+        assert np.array_equal(dst, want)
+        return
+    ld = t["dld"].astype(np.int64)
+    # stride groups are contiguous runs of the list
+    change = np.flatnonzero(ld[1:] != ld[:-1]) + 1
+    starts = np.concatenate(([0], change))
+    ends = np.concatenate((change, [len(ld)]))
+    assert len(np.unique(ld[starts])) == len(starts)
+    for a, b in zip(starts, ends):
+        d = dst[a:b]
+        off = ((d - d.min()) // np.uint64(es)).astype(np.int64)
+        strip = off // ld[a] // 64
+        ds, do = np.diff(strip), np.diff(off)
+        assert np.all((ds > 0) | ((ds == 0) & (do > 0)))
+
+
+@pytest.mark.parametrize("name", ["c1", "c2", "c3", "c5"])
+def test_config_tile_order(name):
+    check_order(C.CONFIGS[name]())
+
+
+def test_c4_and_fuzz_tile_order():
+    for p in C.c4()[:8]:
+        check_order(p)
+    for case in range(300):
+        check_order(C.fuzz_problem(case))
