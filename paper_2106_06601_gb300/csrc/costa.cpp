@@ -119,6 +119,16 @@ AxisCut cut_pair_axis(const costa_layout_s *A, const costa_layout_s *B, int op, 
     return cut_axis(A->C, tr ? B->R : B->C, A->n, ts, vec, !a_rows_fast || b_rows_fast);
 }
 
+// Every tile of a list fits the kernel's tile extent along both axes (the
+// kernel's shared-memory buffers and register passes are sized by it).
+costa_status check_extents(const std::vector<TileDesc> &list, int es, const char *what) {
+    const int ts = tile_extent(es);
+    for (const TileDesc &d : list)
+        if (d.nx < 1 || d.ny < 1 || d.nx > ts || d.ny > ts)
+            return fail(COSTA_ERR_INTERNAL, "%s tile %d x %d exceeds the tile extent %d", what, d.nx, d.ny, ts);
+    return COSTA_OK;
+}
+
 struct ProblemHost {
     const costa_layout_s *A;
     const costa_layout_s *B;
@@ -469,6 +479,10 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     std::vector<TileDesc> list;
     list.reserve(static_cast<size_t>(tiles));
     for (int k = 0; k < n; ++k) append_direct_tiles(plan->probs[k], k, es, ts, list);
+    {
+        costa_status st = check_extents(list, es, "direct");
+        if (st != COSTA_OK) return st;
+    }
     const size_t off_tiles = arena.add_vec(list);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
@@ -644,6 +658,11 @@ costa_status ensure_message(Plan &plan, bool relabel) {
         up.sld = r.ld;
         set_fast(up, es);
         unpack.push_back(up);
+    }
+    for (const auto &l : {std::make_pair(&pack, "pack"), std::make_pair(&local, "local"),
+                          std::make_pair(&unpack, "unpack")}) {
+        costa_status st = check_extents(*l.first, es, l.second);
+        if (st != COSTA_OK) return st;
     }
     Arena arena;
     const size_t o_pack = arena.add_vec(pack);
