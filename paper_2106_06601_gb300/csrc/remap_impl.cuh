@@ -84,6 +84,12 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_NBUF_16
 #define COSTA_NBUF_16 2
 #endif
+#ifndef COSTA_MINB_16A
+#define COSTA_MINB_16A 2
+#endif
+#ifndef COSTA_NBUF_16A
+#define COSTA_NBUF_16A 1
+#endif
 
 // Per element type: tile extent TS, 16-byte chunk width VEC (elements), and
 // the lane mapping: CPR chunks cover one run of TS elements, a warp pass
@@ -108,15 +114,18 @@ template <typename T> struct Cfg {
 // flight ahead of the tile it writes).  8-byte types with the light kinds
 // run more warps without look-ahead; the general kinds (non-power-of-two
 // beta, complex scalars) need the registers of 3 blocks and use a 2-deep
-// ring.  Overridable at build time for tuning.
+// ring.  16-byte kinds that read A hold a whole 16 KB tile of A in
+// registers; they run two blocks without look-ahead.  Overridable at build
+// time for tuning.
 template <typename T, int KIND> struct KCfg {
     static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX;
+    static constexpr bool READS_A = KIND != K_COPY && KIND != K_SCALE;
     static constexpr int WARPS = Cfg<T>::WARPS;
     static constexpr int MINB = sizeof(T) == 4 ? COSTA_MINB_4
-                              : sizeof(T) == 16 ? COSTA_MINB_16
+                              : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
                               : HEAVY ? COSTA_MINB_8H : COSTA_MINB_8;
     static constexpr int NBUF = sizeof(T) == 4 ? COSTA_NBUF_4
-                              : sizeof(T) == 16 ? COSTA_NBUF_16
+                              : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
                               : HEAVY ? COSTA_NBUF_8H : COSTA_NBUF_8;
 };
 
