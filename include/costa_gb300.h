@@ -345,6 +345,22 @@ costa_status costa_volume_noalloc(costa_layout A, costa_layout B, costa_op op, i
 costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void *out, int64_t cap,
                                int64_t *count);
 
+/* Diagnostics (host only, no device work): how the direct tile list of
+ * (A, B, op) is split between the two remap kernels.  Tiles needing fewer
+ * than half of a full tile's warp passes are cut into pieces of one warp
+ * pass each (at most 8 x 8 elements; 16 x 8 for 4-byte and 8 x 4 for
+ * 16-byte elements, x along A's contiguous axis), which the small-tile
+ * kernel moves in groups of up to a full tile's passes; the other tiles stay
+ * with the tile kernel.  Writes up to cap_tiles full-size tiles to `tiles`
+ * and up to cap_pieces pieces to `pieces` (32-byte descriptors as in
+ * costa_debug_tiles), and up to cap_groups group offsets to `groups` (group
+ * g covers pieces [groups[g], groups[g + 1]), so there are *ngroups + 1
+ * offsets when *ngroups > 0); the totals go to *ntiles, *npieces and
+ * *ngroups. */
+costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
+                               void *pieces, int64_t cap_pieces, uint32_t *groups, int64_t cap_groups,
+                               int64_t *ntiles, int64_t *npieces, int64_t *ngroups);
+
 /* Frees every cached plan (synchronizes the device). */
 costa_status costa_release_plans(void);
 

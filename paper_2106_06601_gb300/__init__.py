@@ -79,6 +79,7 @@ def _load():
         "costa_pxtran": [I, I, I64, I64, P, P, I64, I64, P, P, P, I64, I64, P, P],
         "costa_scalapack_release": [],
         "costa_debug_tiles": [P, P, I, P, I64, P],
+        "costa_debug_split": [P, P, I, P, I64, P, I64, P, I64, P, P, P],
         "costa_phase_timing": [I],
         "costa_phase_times": [P, P],
     }
@@ -422,6 +423,21 @@ def costa_debug_axis_pieces(A: Layout, B: Layout, op: str, axis: int) -> np.ndar
 TILE_DTYPE = np.dtype([("src", np.uint64), ("dst", np.uint64), ("sld", np.int32),
                        ("dld", np.int32), ("nx", np.uint16), ("ny", np.uint16),
                        ("prob", np.uint16), ("flags", np.uint16)])
+
+
+def costa_debug_split(A: Layout, B: Layout, op: str):
+    """(full-size tiles, one-pass pieces, group offsets) of the direct list."""
+    nt, npc, ng = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+    _check(_lib.costa_debug_split(A.handle, B.handle, OPS[op], None, 0, None, 0, None, 0,
+                                  ctypes.byref(nt), ctypes.byref(npc), ctypes.byref(ng)))
+    tiles = np.zeros(max(1, nt.value), dtype=TILE_DTYPE)
+    pieces = np.zeros(max(1, npc.value), dtype=TILE_DTYPE)
+    ngo = ng.value + 1 if ng.value > 0 else 0
+    groups = np.zeros(max(1, ngo), dtype=np.uint32)
+    _check(_lib.costa_debug_split(A.handle, B.handle, OPS[op], tiles.ctypes.data, nt.value,
+                                  pieces.ctypes.data, npc.value, groups.ctypes.data, ngo,
+                                  ctypes.byref(nt), ctypes.byref(npc), ctypes.byref(ng)))
+    return tiles[:nt.value], pieces[:npc.value], groups[:ngo]
 
 
 def costa_debug_tiles(A: Layout, B: Layout, op: str) -> np.ndarray:

@@ -129,6 +129,126 @@ costa_status check_extents(const std::vector<TileDesc> &list, int es, const char
     return COSTA_OK;
 }
 
+void set_fast(TileDesc &d, int es);
+
+int next_pow2(int v) {
+    int p = 1;
+    while (p < v) p <<= 1;
+    return p;
+}
+
+// Warp passes the tile kernel needs for a fast tile: the larger of its
+// staging and drain pass counts, with the kernel's lane maps (a run of c
+// chunks takes the next power of two >= c lanes; 32 lanes per pass).
+int fast_tile_passes(const TileDesc &d, int es) {
+    const int vec = 16 / es;
+    const bool tr = (d.flags & TF_TRANSPOSE) != 0;
+    const int runs = tr ? d.nx : d.ny;
+    const int rpp_s = 32 / next_pow2((tr ? d.ny : d.nx) / vec);
+    const int rpp_d = 32 / next_pow2(d.nx / vec);
+    return std::max((runs + rpp_s - 1) / rpp_s, (d.ny + rpp_d - 1) / rpp_d);
+}
+
+// A tile list split for the two remap kernels: full-size tiles for the tile
+// kernel, and the one-pass pieces of the small tiles with their groups for
+// the small-tile kernel.
+struct SplitList {
+    std::vector<TileDesc> big, pieces;
+    std::vector<uint32_t> groups;  // group g = pieces [groups[g], groups[g + 1])
+    int64_t ngroups() const { return groups.empty() ? 0 : static_cast<int64_t>(groups.size()) - 1; }
+};
+
+// A small tile is a fast tile needing fewer passes than small_limit: half
+// of a full tile's passes, a quarter for 8-byte elements (measured on
+// GB300: 16 x 16 tiles of 8-byte elements run faster in the tile kernel,
+// those of 4- and 16-byte elements in the small-tile kernel).
+int small_limit(int es) { return es == 8 ? tile_passes(es) / 4 : tile_passes(es) / 2; }
+
+bool is_small(const TileDesc &d, int es) {
+    // a pass moves at most 32 chunks: a larger tile cannot be small
+    const int64_t area = static_cast<int64_t>(d.nx) * d.ny;
+    if (area * es >= int64_t(512) * small_limit(es) || !(d.flags & TF_FAST)) return false;
+    return fast_tile_passes(d, es) < small_limit(es);
+}
+
+// Splits a list between the kernels.  Only a list whose small tiles hold at
+// least half of its elements uses the small-tile kernel: in a mixed list the
+// warps on small tiles wait on latency while the others keep DRAM busy, and
+// one launch over the whole list measured faster than two (c4: 6157 against
+// 5787 GB/s).  A small tile is cut into pieces of at most piece_x x piece_y
+// (x fastest, so that consecutive pieces continue the target's runs); piece
+// offsets are multiples of the 16-byte chunk, so the pieces stay on the
+// vector path.  Pieces are grouped in list order, at most group_pieces(es)
+// per group and one problem per group.
+SplitList split_small(std::vector<TileDesc> &&list, int es) {
+    SplitList out;
+    int64_t small_elems = 0, all_elems = 0;
+    for (const TileDesc &d : list) {
+        const int64_t e = static_cast<int64_t>(d.nx) * d.ny;
+        all_elems += e;
+        if (is_small(d, es)) small_elems += e;
+    }
+    if (2 * small_elems < all_elems) {
+        out.big = std::move(list);
+        return out;
+    }
+    const int px = piece_x(es), py = piece_y(es), cap = group_pieces(es);
+    int in_group = 0, group_prob = -1;
+    auto add_piece = [&](const TileDesc &pc) {
+        if (in_group == cap || pc.prob != group_prob || out.groups.empty()) {
+            out.groups.push_back(static_cast<uint32_t>(out.pieces.size()));
+            in_group = 0;
+            group_prob = pc.prob;
+        }
+        out.pieces.push_back(pc);
+        ++in_group;
+    };
+    std::vector<TileDesc> cut;
+    for (const TileDesc &d : list) {
+        if (!is_small(d, es)) {
+            out.big.push_back(d);
+            continue;
+        }
+        const bool tr = (d.flags & TF_TRANSPOSE) != 0;
+        cut.clear();
+        bool ok = true;
+        for (int y0 = 0; y0 < d.ny && ok; y0 += py)
+            for (int x0 = 0; x0 < d.nx && ok; x0 += px) {
+                TileDesc pc = d;
+                pc.nx = static_cast<uint16_t>(std::min(px, d.nx - x0));
+                pc.ny = static_cast<uint16_t>(std::min(py, d.ny - y0));
+                pc.dst = d.dst + static_cast<uint64_t>((x0 + static_cast<int64_t>(y0) * d.dld) * es);
+                pc.src = d.src + static_cast<uint64_t>(
+                                     (tr ? static_cast<int64_t>(x0) * d.sld + y0 : x0 + static_cast<int64_t>(y0) * d.sld) *
+                                     es);
+                set_fast(pc, es);
+                ok = (pc.flags & TF_FAST) != 0;
+                cut.push_back(pc);
+            }
+        if (!ok) {  // not expected for a fast tile; keep it whole
+            out.big.push_back(d);
+            continue;
+        }
+        for (const TileDesc &pc : cut) add_piece(pc);
+    }
+    if (!out.groups.empty()) out.groups.push_back(static_cast<uint32_t>(out.pieces.size()));
+    return out;
+}
+
+// Device copies of a split list inside a plan's arena.
+struct DevList {
+    const TileDesc *tiles = nullptr;
+    int64_t ntiles = 0;
+    const TileDesc *pieces = nullptr;
+    const uint32_t *groups = nullptr;
+    int64_t ngroups = 0;
+    bool empty() const { return ntiles == 0 && ngroups == 0; }
+};
+
+struct SplitOffsets {
+    size_t tiles, pieces, groups;
+};
+
 struct ProblemHost {
     const costa_layout_s *A;
     const costa_layout_s *B;
@@ -149,13 +269,23 @@ struct Arena {
     template <typename V> size_t add_vec(const std::vector<V> &v) {
         return add(v.data(), v.size() * sizeof(V));
     }
+    SplitOffsets add_split(const SplitList &l) { return {add_vec(l.big), add_vec(l.pieces), add_vec(l.groups)}; }
 };
+
+DevList resolve(const char *dbase, const SplitOffsets &o, const SplitList &l) {
+    DevList d;
+    d.tiles = reinterpret_cast<const TileDesc *>(dbase + o.tiles);
+    d.ntiles = static_cast<int64_t>(l.big.size());
+    d.pieces = reinterpret_cast<const TileDesc *>(dbase + o.pieces);
+    d.groups = reinterpret_cast<const uint32_t *>(dbase + o.groups);
+    d.ngroups = l.ngroups();
+    return d;
+}
 
 struct MessageData {
     bool built = false;
     void *d_mem = nullptr;       // pack, local and unpack tile lists
-    const TileDesc *pack = nullptr, *local = nullptr, *unpack = nullptr;
-    int64_t n_pack = 0, n_local = 0, n_unpack = 0;
+    DevList pack, local, unpack;
     void *d_staging = nullptr;
     int64_t staging_bytes = 0;
 };
@@ -165,7 +295,7 @@ struct Plan {
     int dtype = 0, esize = 0, P = 0, ts = 32;
     std::vector<ProblemHost> probs;
     void *d_mem = nullptr;
-    const TileDesc *d_tiles = nullptr;  // the direct list
+    DevList direct;                     // the direct list
     Scalars *d_scalars = nullptr;
     std::vector<Scalars> cached_scalars;
     int64_t total_tiles = 0, total_cells = 0;
@@ -483,7 +613,8 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
         costa_status st = check_extents(list, es, "direct");
         if (st != COSTA_OK) return st;
     }
-    const size_t off_tiles = arena.add_vec(list);
+    const SplitList split = split_small(std::move(list), es);
+    const SplitOffsets off_tiles = arena.add_split(split);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
     std::vector<Scalars> sc(n);
@@ -518,7 +649,7 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     std::memcpy(arena.host.data() + off_vd, vd.data(), sizeof(VolumeProblemDev) * n);
     ce = cudaMemcpy(d, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(plan tables)");
-    plan->d_tiles = reinterpret_cast<const TileDesc *>(dbase + off_tiles);
+    plan->direct = resolve(dbase, off_tiles, split);
     plan->d_scalars = reinterpret_cast<Scalars *>(dbase + off_sc);
     plan->total_tiles = tiles;
     plan->total_cells = cells;
@@ -664,21 +795,20 @@ costa_status ensure_message(Plan &plan, bool relabel) {
         costa_status st = check_extents(*l.first, es, l.second);
         if (st != COSTA_OK) return st;
     }
+    const SplitList s_pack = split_small(std::move(pack), es), s_local = split_small(std::move(local), es),
+                    s_unpack = split_small(std::move(unpack), es);
     Arena arena;
-    const size_t o_pack = arena.add_vec(pack);
-    const size_t o_local = arena.add_vec(local);
-    const size_t o_unpack = arena.add_vec(unpack);
+    const SplitOffsets o_pack = arena.add_split(s_pack);
+    const SplitOffsets o_local = arena.add_split(s_local);
+    const SplitOffsets o_unpack = arena.add_split(s_unpack);
     cudaError_t ce = cudaMalloc(&m.d_mem, arena.host.size());
     if (ce != cudaSuccess) return fail(COSTA_ERR_ALLOC, "cudaMalloc(message tables): %s", cudaGetErrorString(ce));
     ce = cudaMemcpy(m.d_mem, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(message tables)");
-    char *db = static_cast<char *>(m.d_mem);
-    m.pack = reinterpret_cast<const TileDesc *>(db + o_pack);
-    m.local = reinterpret_cast<const TileDesc *>(db + o_local);
-    m.unpack = reinterpret_cast<const TileDesc *>(db + o_unpack);
-    m.n_pack = static_cast<int64_t>(pack.size());
-    m.n_local = static_cast<int64_t>(local.size());
-    m.n_unpack = static_cast<int64_t>(unpack.size());
+    const char *db = static_cast<const char *>(m.d_mem);
+    m.pack = resolve(db, o_pack, s_pack);
+    m.local = resolve(db, o_local, s_local);
+    m.unpack = resolve(db, o_unpack, s_unpack);
     m.built = true;
     plan.stats.staging_bytes = m.staging_bytes;
     return COSTA_OK;
@@ -782,8 +912,6 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     auto mark = [&](int k) -> cudaError_t { return timer ? cudaEventRecord(timer->ev[k], stream) : cudaSuccess; };
 
     RemapLaunch L{};
-    L.tiles = plan->d_tiles;
-    L.ntiles = plan->total_tiles;
     L.dtype = plan->dtype;
     L.s = make_scalars(plan->dtype, alphas, betas, 0);
     L.per_problem = nullptr;
@@ -809,10 +937,13 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     // one launch per combine kind present in the batch
     bool kinds[K_NKINDS] = {};
     for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
-    auto launch_list = [&](const TileDesc *list, int64_t count) -> cudaError_t {
+    auto launch_list = [&](const DevList &list) -> cudaError_t {
         RemapLaunch l = L;
-        l.tiles = list;
-        l.ntiles = count;
+        l.tiles = list.tiles;
+        l.ntiles = list.ntiles;
+        l.pieces = list.pieces;
+        l.groups = list.groups;
+        l.ngroups = list.ngroups;
         for (int kind = 0; kind < K_NKINDS; ++kind) {
             if (!kinds[kind]) continue;
             cudaError_t e = launch_remap(l, kind, stream);
@@ -823,7 +954,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     cudaError_t ce;
     if (mode == COSTA_MODE_DIRECT) {
         ce = mark(0);
-        if (ce == cudaSuccess) ce = launch_list(plan->d_tiles, plan->total_tiles);
+        if (ce == cudaSuccess) ce = launch_list(plan->direct);
         if (ce == cudaSuccess) ce = mark(1);
         if (ce != cudaSuccess) return cuda_fail(ce, "remap kernel launch");
         if (timer) timer->nphases = 1;
@@ -833,8 +964,11 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     if (s != COSTA_OK) return s;
     const MessageData &m = plan->msg[relabel ? 1 : 0];
     RemapLaunch lp{};
-    lp.tiles = m.pack;
-    lp.ntiles = m.n_pack;
+    lp.tiles = m.pack.tiles;
+    lp.ntiles = m.pack.ntiles;
+    lp.pieces = m.pack.pieces;
+    lp.groups = m.pack.groups;
+    lp.ngroups = m.pack.ngroups;
     lp.dtype = plan->dtype;
     lp.per_problem = nullptr;
     const float one_f[2] = {1.0f, 0.0f}, zero_f[2] = {0.0f, 0.0f};
@@ -846,10 +980,10 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     if (ce == cudaSuccess) ce = launch_remap(lp, K_COPY, stream);
     if (ce == cudaSuccess) ce = mark(1);
     if (ce != cudaSuccess) return cuda_fail(ce, "pack kernel launch");
-    ce = launch_list(m.local, m.n_local);
+    ce = launch_list(m.local);
     if (ce == cudaSuccess) ce = mark(2);
     if (ce != cudaSuccess) return cuda_fail(ce, "local remap kernel launch");
-    ce = launch_list(m.unpack, m.n_unpack);
+    ce = launch_list(m.unpack);
     if (ce == cudaSuccess) ce = mark(3);
     if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
     if (timer) timer->nphases = 3;
@@ -1190,6 +1324,36 @@ costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void
     append_direct_tiles(ph, 0, es, ts, list);
     const size_t k = static_cast<size_t>(std::min<int64_t>(cap, *count));
     if (k) std::memcpy(out, list.data(), k * sizeof(TileDesc));
+    return COSTA_OK;
+}
+
+costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
+                               void *pieces, int64_t cap_pieces, uint32_t *groups, int64_t cap_groups,
+                               int64_t *ntiles, int64_t *npieces, int64_t *ngroups) {
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    if (!ntiles || !npieces || !ngroups || (cap_tiles > 0 && !tiles) || (cap_pieces > 0 && !pieces) ||
+        (cap_groups > 0 && !groups))
+        return fail(COSTA_ERR_INVALID_ARG, "bad arguments");
+    const int es = esize_of(A->dt), ts = tile_extent(es);
+    ProblemHost ph;
+    ph.A = A;
+    ph.B = B;
+    ph.op = op;
+    ph.rows = cut_pair_axis(A, B, op, 0, ts);
+    ph.cols = cut_pair_axis(A, B, op, 1, ts);
+    std::vector<TileDesc> list;
+    append_direct_tiles(ph, 0, es, ts, list);
+    const SplitList sp = split_small(std::move(list), es);
+    *ntiles = static_cast<int64_t>(sp.big.size());
+    *npieces = static_cast<int64_t>(sp.pieces.size());
+    *ngroups = sp.ngroups();
+    const size_t kt = static_cast<size_t>(std::min<int64_t>(cap_tiles, *ntiles));
+    const size_t kp = static_cast<size_t>(std::min<int64_t>(cap_pieces, *npieces));
+    const size_t kg = static_cast<size_t>(std::min<int64_t>(cap_groups, static_cast<int64_t>(sp.groups.size())));
+    if (kt) std::memcpy(tiles, sp.big.data(), kt * sizeof(TileDesc));
+    if (kp) std::memcpy(pieces, sp.pieces.data(), kp * sizeof(TileDesc));
+    if (kg) std::memcpy(groups, sp.groups.data(), kg * sizeof(uint32_t));
     return COSTA_OK;
 }
 

@@ -111,8 +111,11 @@ COSTA_HD inline int kind_of(int32_t flags) {
 
 
 struct RemapLaunch {
-    const TileDesc *tiles;
+    const TileDesc *tiles;       // full-size tiles (the tile kernel)
     int64_t ntiles;
+    const TileDesc *pieces;      // one-pass pieces of small tiles (the small-tile kernel)
+    const uint32_t *groups;      // group g = pieces [groups[g], groups[g + 1])
+    int64_t ngroups;
     int32_t dtype;
     int32_t pad;
     const Scalars *per_problem;  // device array indexed by TileDesc::prob, or nullptr: use `s`
@@ -145,6 +148,15 @@ struct VolumeLaunch {
 #define COSTA_TS_16 32
 #endif
 COSTA_HD constexpr int tile_extent(int esize) { return esize == 16 ? COSTA_TS_16 : 32; }
+
+// Small tiles are cut by the host into pieces of at most piece_x x piece_y
+// elements, each exactly one warp pass (32 lanes x 16 bytes at most), and
+// grouped at most group_pieces (a full tile's tile_passes) per group, one
+// problem per group; the small-tile kernel moves a group like one tile.
+COSTA_HD constexpr int piece_x(int esize) { return esize == 4 ? 16 : 8; }
+COSTA_HD constexpr int piece_y(int esize) { return esize == 16 ? 4 : 8; }
+COSTA_HD constexpr int tile_passes(int esize) { return tile_extent(esize) * tile_extent(esize) * esize / 512; }
+COSTA_HD constexpr int group_pieces(int esize) { return tile_passes(esize); }
 
 // Launches the remap kernel for (args.dtype, kind) over a tile list.  With
 // args.per_problem set, the kernel skips the tiles of problems of another kind.

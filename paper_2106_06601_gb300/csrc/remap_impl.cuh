@@ -308,16 +308,15 @@ __device__ __forceinline__ double pow2_apply(double a, const Sc &s) {
 // of the warp holds a value it does not cover; that choice is one warp vote,
 // so the scarce FP64 pipe never runs predicated-off multiplies.  beta = +-1
 // needs at most a sign flip.  Float data multiplies (the FP32 pipe is wide).
-template <typename T>
-__device__ __forceinline__ void prescale(Chunk<T> (&av)[Cfg<T>::NPASS], int npass, const Sc &s) {
-    using C = Cfg<T>;
+template <typename T, int N>
+__device__ __forceinline__ void prescale(Chunk<T> (&av)[N], int npass, const Sc &s) {
     using R = typename ET<T>::R;
     constexpr int PER = 16 / static_cast<int>(sizeof(R));  // reals per chunk
     if constexpr (sizeof(R) == 8) {
         if (s.bexp == 0) {
             if (s.bsign_hi) {
 #pragma unroll
-                for (int p = 0; p < C::NPASS; ++p) {
+                for (int p = 0; p < N; ++p) {
                     if (p >= npass) break;
                     av[p].raw.y ^= s.bsign_hi;
                     av[p].raw.w ^= s.bsign_hi;
@@ -327,7 +326,7 @@ __device__ __forceinline__ void prescale(Chunk<T> (&av)[Cfg<T>::NPASS], int npas
         }
         bool bad = false;
 #pragma unroll
-        for (int p = 0; p < C::NPASS; ++p) {
+        for (int p = 0; p < N; ++p) {
             if (p >= npass) break;
             const double *v = reinterpret_cast<const double *>(&av[p]);
 #pragma unroll
@@ -335,7 +334,7 @@ __device__ __forceinline__ void prescale(Chunk<T> (&av)[Cfg<T>::NPASS], int npas
         }
         if (__any_sync(0xffffffffu, bad)) {
 #pragma unroll
-            for (int p = 0; p < C::NPASS; ++p) {
+            for (int p = 0; p < N; ++p) {
                 if (p >= npass) break;
                 double *v = reinterpret_cast<double *>(&av[p]);
 #pragma unroll
@@ -343,7 +342,7 @@ __device__ __forceinline__ void prescale(Chunk<T> (&av)[Cfg<T>::NPASS], int npas
             }
         } else {
 #pragma unroll
-            for (int p = 0; p < C::NPASS; ++p) {
+            for (int p = 0; p < N; ++p) {
                 if (p >= npass) break;
                 double *v = reinterpret_cast<double *>(&av[p]);
 #pragma unroll
@@ -352,7 +351,7 @@ __device__ __forceinline__ void prescale(Chunk<T> (&av)[Cfg<T>::NPASS], int npas
         }
     } else {
 #pragma unroll
-        for (int p = 0; p < C::NPASS; ++p) {
+        for (int p = 0; p < N; ++p) {
             if (p >= npass) break;
             float *v = reinterpret_cast<float *>(&av[p]);
 #pragma unroll
@@ -561,6 +560,167 @@ __device__ __forceinline__ bool next_tile(const RemapLaunch &a, int64_t first, i
     }
 }
 
+// ---- the small-tile kernel ----
+//
+// Lists made mostly of small tiles (see split_small on the host) come as
+// one-pass pieces (at most 32 chunks; piece_x x piece_y) in groups of at
+// most group_pieces (a full tile's passes) of one problem.  A warp moves one
+// group like one tile: it stages every piece's source into its own 512-byte
+// slot, loads every piece's A chunk into its own register, waits once and
+// drains every piece.  A warp thus keeps a full tile's bytes in flight
+// instead of one small tile's.
+
+// Row width (chunks) of a staged piece: the lanes per run of its lane map.
+__device__ __forceinline__ int piece_width(int chunks) {
+    return 1 << (chunks <= 1 ? 0 : 32 - __clz(chunks - 1));
+}
+
+// Stages a piece's source into its slot (one pass: every run has its lanes).
+template <typename T>
+__device__ __forceinline__ void piece_issue(const Geom<T> &g, unsigned char *slot_base, int lane) {
+    using C = Cfg<T>;
+    const int runs = g.transpose ? g.nx : g.ny;
+    const int chunks = (g.transpose ? g.ny : g.nx) / C::VEC;
+    const LaneMap m = lane_map(chunks, lane);
+    const int W = piece_width(chunks);
+    if (m.c < chunks && m.r0 < runs)
+        cp_async16(slot_base + (m.r0 * W + (m.c ^ (swz<T>(m.r0) & (W - 1)))) * 16,
+                   g.src + static_cast<int64_t>(m.r0) * g.sld + m.c * C::VEC);
+}
+
+// This lane's A chunk of a piece (zero when the lane has none).
+template <typename T>
+__device__ __forceinline__ Chunk<T> piece_load_a(const Geom<T> &g, int lane) {
+    using C = Cfg<T>;
+    const int chunks = g.nx / C::VEC;
+    const LaneMap m = lane_map(chunks, lane);
+    Chunk<T> a;
+    a.raw = make_uint4(0, 0, 0, 0);
+    if (m.c < chunks && m.r0 < g.ny) a = load_rw(g.dst + static_cast<int64_t>(m.r0) * g.dld + m.c * C::VEC);
+    return a;
+}
+
+// Writes this lane's chunk of a staged piece to A.
+template <typename T, int KIND>
+__device__ __forceinline__ void piece_drain(const Geom<T> &g, const Sc &s, unsigned char *slot_base,
+                                            const Chunk<T> &a, int lane) {
+    using C = Cfg<T>;
+    const int chunks = g.nx / C::VEC;
+    const LaneMap m = lane_map(chunks, lane);
+    const int y = m.r0;
+    if (m.c >= chunks || y >= g.ny) return;
+    const int x0 = m.c * C::VEC;
+    Chunk<T> b;
+    if (g.transpose) {
+        // element (x0 + e, y): staged row x0 + e, chunk y / VEC, lane y % VEC
+        const int W = piece_width(g.ny / C::VEC);
+        if ((x0 + C::VEC - 1) * W >= 32) return;  // rows beyond one pass (never emitted by the host)
+        const int cy = y / C::VEC, ey = y % C::VEC;
+#pragma unroll
+        for (int e = 0; e < C::VEC; ++e) {
+            const int r = x0 + e;
+            b.e[e] = reinterpret_cast<const T *>(slot_base + (r * W + (cy ^ (swz<T>(r) & (W - 1)))) * 16)[ey];
+        }
+    } else {
+        const int W = piece_width(chunks);
+        b.raw = *reinterpret_cast<const uint4 *>(slot_base + (y * W + (m.c ^ (swz<T>(y) & (W - 1)))) * 16);
+    }
+    Chunk<T> o;
+#pragma unroll
+    for (int e = 0; e < C::VEC; ++e) o.e[e] = combine<KIND>(b.e[e], a.e[e], s);
+    store(g.dst + static_cast<int64_t>(y) * g.dld + x0, o);
+}
+
+#ifndef COSTA_SWARPS
+#define COSTA_SWARPS 4
+#endif
+#ifndef COSTA_SMINB_4
+#define COSTA_SMINB_4 5
+#endif
+#ifndef COSTA_SMINB_8
+#define COSTA_SMINB_8 4
+#endif
+#ifndef COSTA_SMINB_8H
+#define COSTA_SMINB_8H 3
+#endif
+#ifndef COSTA_SMINB_16
+#define COSTA_SMINB_16 3
+#endif
+#ifndef COSTA_SMINB_16A
+#define COSTA_SMINB_16A 2
+#endif
+
+// Launch shape of the small-tile kernel: warps per block and resident blocks
+// per SM; each warp has one buffer of NS 512-byte slots.
+template <typename T, int KIND> struct SCfg {
+    static constexpr int WARPS = COSTA_SWARPS;
+    static constexpr int MINB = sizeof(T) == 4 ? COSTA_SMINB_4
+                              : sizeof(T) == 16 ? (KCfg<T, KIND>::READS_A ? COSTA_SMINB_16A : COSTA_SMINB_16)
+                              : KCfg<T, KIND>::HEAVY ? COSTA_SMINB_8H : COSTA_SMINB_8;
+    static constexpr int NS = group_pieces(static_cast<int>(sizeof(T)));
+    static constexpr int BUF_BYTES = NS * 512;
+};
+
+template <typename T, int KIND>
+__global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB)
+    remap_small_kernel(const RemapLaunch args) {
+    using SC = SCfg<T, KIND>;
+    constexpr int NS = SC::NS;
+    constexpr bool READS_A = KCfg<T, KIND>::READS_A;
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char *buf = smem_raw + warp * SC::BUF_BYTES;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * SC::WARPS;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * SC::WARPS + warp;
+    Sc s;
+    int cached = -1;
+    if (!args.per_problem) make_sc(args.s, s);
+    for (int64_t gi = first; gi < args.ngroups; gi += stride) {
+        const uint32_t g0 = __ldg(args.groups + gi), g1 = __ldg(args.groups + gi + 1);
+        // 1 .. NS pieces (the host's groups); the clamp keeps the slots inside
+        // this warp's buffer regardless
+        const int cnt = min(static_cast<int>(g1 - g0), NS);
+        DescRegs r;
+        if (lane < cnt) {
+            const uint4 *p = reinterpret_cast<const uint4 *>(args.pieces + g0 + lane);
+            r.lo = __ldg(p);
+            r.hi = __ldg(p + 1);
+        } else {
+            r.lo = make_uint4(0, 0, 0, 0);
+            r.hi = make_uint4(0, 0, 0, 0);
+        }
+        if (args.per_problem) {  // one problem per group
+            const int prob = static_cast<int>(shfl_desc(r, 0).prob);
+            if (kind_of(args.per_problem[prob].flags) != KIND) continue;
+            if (prob != cached) {
+                make_sc(args.per_problem[prob], s);
+                cached = prob;
+            }
+        }
+        for (int k = 0; k < cnt; ++k) piece_issue<T>(geom_of<T>(shfl_desc(r, k)), buf + 512 * k, lane);
+        cp_async_commit();
+        Chunk<T> av[NS];
+        if (READS_A) {
+#pragma unroll
+            for (int k = 0; k < NS; ++k) {
+                if (k >= cnt) break;  // uniform across the warp
+                av[k] = piece_load_a<T>(geom_of<T>(shfl_desc(r, k)), lane);
+            }
+            if (KIND == K_AXPBY2) prescale<T>(av, cnt, s);
+        }
+        cp_async_wait<0>();
+        __syncwarp();
+#pragma unroll
+        for (int k = 0; k < NS; ++k) {
+            if (k >= cnt) break;
+            const Geom<T> g = geom_of<T>(shfl_desc(r, k));
+            s.conj_mask = g.conj ? 0x80000000u : 0u;
+            piece_drain<T, KIND>(g, s, buf + 512 * k, av[k], lane);
+        }
+        __syncwarp();  // the slots are free before the next group is staged
+    }
+}
+
 // Writes one tile (staged in `buf` if it is a fast tile).  `cached` holds
 // the problem whose scalars are in `s`.
 template <typename T, int KIND, int NB>
@@ -653,7 +813,7 @@ inline int sm_count() {
 }
 
 template <typename T, int KIND>
-cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
+cudaError_t launch_tiles(const RemapLaunch &a, cudaStream_t st) {
     auto kern = remap_kernel<T, KIND>;
     constexpr int kWarps = Cfg<T>::WARPS;
     const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND>::NBUF * Cfg<T>::BUF_BYTES;
@@ -673,6 +833,38 @@ cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     kern<<<blocks, kWarps * 32, smem, st>>>(a);
     count_launch();
     return cudaGetLastError();
+}
+
+template <typename T, int KIND>
+cudaError_t launch_small(const RemapLaunch &a, cudaStream_t st) {
+    using SC = SCfg<T, KIND>;
+    auto kern = remap_small_kernel<T, KIND>;
+    const size_t smem = static_cast<size_t>(SC::WARPS) * SC::BUF_BYTES;
+    static int per_sm = 0;
+    if (per_sm == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, SC::WARPS * 32, smem);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) per_sm = 1;
+    }
+    const int64_t want = (a.ngroups + SC::WARPS - 1) / SC::WARPS;
+    const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;
+    const int blocks = static_cast<int>(want < cap ? want : cap);
+    if (blocks <= 0) return cudaSuccess;
+    kern<<<blocks, SC::WARPS * 32, smem, st>>>(a);
+    count_launch();
+    return cudaGetLastError();
+}
+
+// The tile kernel over the full-size tiles, then the small-tile kernel over
+// the groups of pieces (each launched only when it has work).
+template <typename T, int KIND>
+cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
+    cudaError_t e = a.ntiles > 0 ? launch_tiles<T, KIND>(a, st) : cudaSuccess;
+    if (e == cudaSuccess && a.ngroups > 0) e = launch_small<T, KIND>(a, st);
+    return e;
 }
 
 // Kernel for (element type, combine kind).  Real types never take K_CPLX.

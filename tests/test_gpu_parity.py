@@ -45,6 +45,18 @@ def test_fuzz_direct(case, dev):
     check_problem(C.fuzz_problem(case), dev, guard=3 if case % 4 == 0 else 0)
 
 
+@pytest.mark.parametrize("case", range(96))
+def test_small_blocks(case, dev):
+    """Small and odd blocks: the small-tile kernel's pieces and groups, in
+    direct and message mode (the two agree bit for bit)."""
+    p = C.small_block_problem(case)
+    _, direct = check_problem(p, dev)
+    _, msg = check_problem(p, dev, mode="message")
+    assert np.array_equal(msg.arena, direct.arena, equal_nan=True)
+    if case % 3 == 0:  # guard elements around every buffer stay untouched
+        check_problem(p, dev, guard=2)
+
+
 @pytest.mark.parametrize("case", range(120, 180))
 def test_fuzz_message_equals_direct(case, dev):
     p = C.fuzz_problem(case)

@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 
 from workloads import configs as C
+from workloads import layouts as L
 
 costa = pytest.importorskip("paper_2106_06601_gb300")
 
@@ -182,3 +183,98 @@ def test_c4_and_fuzz_tile_order():
         check_order(p)
     for case in range(300):
         check_order(C.fuzz_problem(case))
+
+
+def _in_buffers(t, spec, es, which):
+    """Every access of the tiles `t` on side `which` ("dst" = A, "src" = B)
+    falls inside the rank buffers of `spec` (corner test: tiles are affine)."""
+    nx, ny = t["nx"].astype(np.int64), t["ny"].astype(np.int64)
+    tr = (t["flags"] & 1) != 0
+    base = t[which].astype(np.int64)
+    ld = (t["dld"] if which == "dst" else t["sld"]).astype(np.int64)
+    if which == "dst":
+        sx, sy = np.ones_like(ld), ld
+    else:
+        sx, sy = np.where(tr, ld, 1), np.where(tr, 1, ld)
+    for cx in (0, 1):
+        for cy in (0, 1):
+            rel = base + ((nx - 1) * cx * sx + (ny - 1) * cy * sy) * es - FAKE
+            buf = rel >> 32
+            off = rel - (buf << 32)
+            assert np.all(buf >= 0) and np.all(buf < spec.nbuf), which
+            assert np.all(off >= 0) and np.all(off < spec.bufsize[buf] * es), which
+
+
+def _covered(t, es):
+    """Target element addresses covered by the tiles `t`."""
+    out = []
+    for d in t:
+        x = np.arange(int(d["nx"]), dtype=np.int64)
+        y = np.arange(int(d["ny"]), dtype=np.int64)
+        out.append((int(d["dst"]) + (x[None, :] + y[:, None] * int(d["dld"])) * es).ravel())
+    return np.concatenate(out) if out else np.zeros(0, np.int64)
+
+
+def _pow2(v):
+    return 1 << int(np.ceil(np.log2(max(1, v))))
+
+
+def check_split(p, exact=False):
+    """The split between the tile kernel and the small-tile kernel: pieces
+    are fast, one warp pass each (every run has its lanes), inside the
+    buffers, at most piece_x x piece_y; groups hold at most a full tile's
+    passes, of one problem; full-size tiles and pieces together cover A
+    exactly once (checked element by element when `exact`)."""
+    es = {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[p.dtype]
+    vec = 16 // es
+    px, py = {4: (16, 8), 8: (8, 8), 16: (8, 4)}[es]
+    cap = 32 * 32 * es // 512
+    LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+    try:
+        big, pieces, groups = costa.costa_debug_split(LA, LB, p.op)
+        whole = costa.costa_debug_tiles(LA, LB, p.op)
+    finally:
+        LA.destroy()
+        LB.destroy()
+    area = lambda t: int((t["nx"].astype(np.int64) * t["ny"].astype(np.int64)).sum())
+    assert area(big) + area(pieces) == p.A.m * p.A.n == area(whole)
+    if len(pieces):
+        nx, ny = pieces["nx"].astype(np.int64), pieces["ny"].astype(np.int64)
+        tr = (pieces["flags"] & 1) != 0
+        assert np.all(pieces["flags"] & 2), "pieces take the vector path"
+        assert np.all((nx >= 1) & (nx <= px) & (ny >= 1) & (ny <= py))
+        assert np.all(nx % vec == 0) and np.all(np.where(tr, ny, nx) % vec == 0)
+        lanes_d = np.array([_pow2(v // vec) for v in nx]) * ny
+        lanes_s = np.where(tr, nx * np.array([_pow2(v // vec) for v in ny]), lanes_d)
+        assert np.all(lanes_d <= 32) and np.all(lanes_s <= 32)
+        _in_buffers(pieces, p.A, es, "dst")
+        _in_buffers(pieces, p.B, es, "src")
+        g = groups.astype(np.int64)
+        assert g[0] == 0 and g[-1] == len(pieces)
+        sizes = np.diff(g)
+        assert np.all(sizes >= 1) and np.all(sizes <= cap)
+        for a, b in zip(g[:-1], g[1:]):
+            assert len(np.unique(pieces["prob"][a:b])) == 1
+    else:
+        assert len(groups) == 0
+    if exact:
+        cov = np.concatenate((_covered(big, es), _covered(pieces, es)))
+        assert len(cov) == p.A.m * p.A.n and len(np.unique(cov)) == len(cov)
+        assert np.array_equal(np.sort(cov), np.sort(_covered(whole, es)))
+
+
+@pytest.mark.parametrize("name", ["c1", "c2", "c3", "c5"])
+def test_config_split(name):
+    check_split(C.CONFIGS[name](), exact=(name == "c1"))
+
+
+def test_c4_and_fuzz_split():
+    for p in C.c4()[:8]:
+        check_split(p)
+    for case in range(200):
+        check_split(C.fuzz_problem(case), exact=True)
+
+
+def test_small_block_split():
+    for case in range(120):
+        check_split(C.small_block_problem(case), exact=True)

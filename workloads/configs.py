@@ -178,6 +178,38 @@ COMPLEX_SCALARS = [(complex(0.5, -0.75), complex(1.0, 0.0)),
                    (complex(-0.6, 0.3), 0.0)]
 
 
+SMALL_BLOCKS = (1, 2, 3, 4, 5, 8, 12, 16, 24)
+ALIGNED_SMALL_BLOCKS = (4, 8, 12, 16)
+
+
+def small_block_problem(case: int) -> Problem:
+    """Block-cyclic layouts with small blocks on 2 x 2 grids, both storage
+    orders, cycling through the element types and ops; drawn from stream
+    LAYOUT + 5000 + case.  Odd cases take odd block sizes (1 .. 24) and padded
+    leading dimensions; even cases take block sizes that are multiples of 4,
+    matrix sizes that are multiples of 16 and unpadded storage, so that their
+    tiles start on 16-byte boundaries."""
+    rng = IntStream(SEED0 + 200, LAYOUT + 5000 + case)
+    dtype = ("f32", "f64", "c64", "c128")[(case // 2) % 4]
+    op = "NTC"[(case // 8) % 3]
+    aligned = case % 2 == 0
+    if aligned:
+        m, n = 16 * rng.between(1, 6), 16 * rng.between(1, 6)
+        sizes, pad = ALIGNED_SMALL_BLOCKS, lambda: 0
+    else:
+        m, n = rng.between(1, 90), rng.between(1, 90)
+        sizes, pad = SMALL_BLOCKS, lambda: rng.below(3)
+    mbB, nbB, mbA, nbA = (sizes[rng.below(len(sizes))] for _ in range(4))
+    sb, sa = ("C", "R")[(case // 24) % 2], ("C", "R")[(case // 48) % 2]
+    B = L.block_cyclic(m, n, mbB, nbB, 2, 2, storage=sb, ld_pad=pad(), name="B")
+    am, an = (m, n) if op == "N" else (n, m)
+    A = L.block_cyclic(am, an, mbA, nbA, 2, 2, grid_order="C", storage=sa, ld_pad=pad(), name="A")
+    alpha, beta = SCALARS[rng.below(len(SCALARS))]
+    a_kind = "nan" if beta == 0 else "uniform"
+    return Problem(f"small{case}", dtype, op, alpha, beta, A, B, "uniform", a_kind, SEED0 + 200,
+                   index=case % 64)
+
+
 def fuzz_problem(case: int, *, dtype=None, op=None, P=None, max_dim: int = 160) -> Problem:
     """A random small problem; everything is drawn from stream LAYOUT + case."""
     rng = IntStream(SEED0 + 100, LAYOUT + case)
