@@ -54,7 +54,7 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--workload", default="c2", choices=list(C.CONFIGS))
+    ap.add_argument("--workload", default="c2", choices=list(C.CONFIGS) + list(C.EXTRA_WORKLOADS))
     ap.add_argument("--mode", default="direct", choices=["direct", "message"])
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=20)
@@ -173,7 +173,7 @@ def job_throughput(bytes_per_rank: int, world: int, steps: int, max_ms: float) -
 
 
 def problems(workload, small=False):
-    p = (C.CONFIGS_SMALL if small else C.CONFIGS)[workload]()
+    p = (C.CONFIGS_SMALL if small else {**C.CONFIGS, **C.EXTRA_WORKLOADS})[workload]()
     return p if isinstance(p, list) else [p]
 
 
@@ -302,6 +302,7 @@ def run_gpu(args, rank, world, local_rank):
     phases = None
     if args.mode == "message":
         phases = message_phases(args, probs, stats, step, stream, dev)
+    kernels = direct_kernels(costa, mats)
     for m in mats:
         m[3].destroy()
         m[4].destroy()
@@ -312,7 +313,26 @@ def run_gpu(args, rank, world, local_rank):
     return dict(value=value, ms_per_step=ms_per_step, total_ms=total_ms, per=per,
                 launches=launches, clocks=clk, e2e=e2e, plan_s=plan_s, stats=stats,
                 nbytes=nbytes, achieved=achieved, peak=peak, peak_kind=peak_kind,
-                traffic=traffic, probs=probs, phases=phases)
+                traffic=traffic, probs=probs, phases=phases, kernels=kernels)
+
+
+def direct_kernels(costa, mats):
+    """Which remap kernels the direct list runs: the tile kernel, and the
+    small-tile kernel when small tiles hold at least half of the elements of
+    the (batched) list, by the planner's rule (costa_debug_split)."""
+    small = total = 0
+    tile_kernel = False
+    for p, _, _, LA, LB in mats:
+        t, pieces, _ = costa.costa_debug_split(LA, LB, p.op)
+        if len(pieces):
+            small += int((pieces["nx"].astype("int64") * pieces["ny"]).sum())
+            tile_kernel |= len(t) > 0
+        total += p.A.m * p.A.n
+    if len(mats) > 1 and 2 * small < total:
+        return "remap_kernel (direct)"
+    if small == 0:
+        return "remap_kernel (direct)"
+    return ("remap_kernel + " if tile_kernel else "") + "remap_small_kernel (direct)"
 
 
 def message_phases(args, probs, stats, step, stream, dev):
@@ -370,7 +390,7 @@ def roofline(args, r):
                      "timing": f"phase events over {ph['steps']} steps after the timed region"})
         return base
     base.update({"achieved": round(r["achieved"], 2), "frac": round(r["achieved"] / r["peak"], 4),
-                 "traffic": r["traffic"], "kernel": "remap_kernel (direct)",
+                 "traffic": r["traffic"], "kernel": r["kernels"],
                  "algorithmic_bytes_per_launch": r["nbytes"],
                  "avg_launch_ms": round(statistics.mean(r["per"]), 5),
                  "median_launch_ms": round(statistics.median(r["per"]), 5),

@@ -119,10 +119,24 @@ def c5(rows: int = 131072, cols: int = 4096) -> Problem:
 
 CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5}
 
+
+def small_blocks(n: int = 8192, mb: int = 8, dtype: str = "f64") -> Problem:
+    """The small-block case (not one of the configurations above): c2's
+    shape and scalars with mb x mb blocks on both sides, 4 x 4 grids, the
+    target's owners a seeded permutation."""
+    perm = IntStream(_seed(6), LAYOUT).permutation(16)
+    B = L.block_cyclic(n, n, mb, mb, 4, 4, grid_order="R", name="B")
+    A = L.block_cyclic(n, n, mb, mb, 4, 4, grid_order="R", rank_perm=perm, name="A")
+    return Problem(f"bc{mb}", dtype, "T", 2.0, 0.5, A, B, "uniform", "uniform", _seed(6))
+
+
+# Further workloads for measurement only.
+EXTRA_WORKLOADS = {"bc8": small_blocks}
+
 # The same layouts and tile shapes at about 1 GB on the device, for profiler
 # captures (the workloads proper stay the ones above).
 CONFIGS_SMALL = {"c1": c1, "c2": lambda: c2(4096), "c3": lambda: c3(8192),
-                 "c4": lambda: c4(16), "c5": lambda: c5(rows=16384)}
+                 "c4": lambda: c4(16), "c5": lambda: c5(rows=16384), "bc8": lambda: small_blocks(4096)}
 
 WORKLOAD_TEXT = {
     "c1": "256x256 f64 BC16 2x2R -> BC32 2x2C, N, alpha=1 beta=0, P=4",
@@ -130,6 +144,8 @@ WORKLOAD_TEXT = {
     "c3": "16384x16384 c128 BC32 8x8 -> irregular 8x8 (512..3584), C, alpha=1 beta=0, P=64",
     "c4": "64 x 2048x3072 f32 BC{16..128} 4x4, N/T alternating, alpha=1 beta=0, P=16, batched",
     "c5": "131072x4096 f64 BC32 16x16 -> 4096x131072 in 256 row panels, T, alpha=1 beta=1, P=256",
+    "bc8": "8192x8192 f64 BC8 4x4 -> BC8 4x4 permuted owners, T, alpha=2 beta=0.5, P=16 "
+           "(small-block case, not a configuration)",
 }
 
 
