@@ -72,8 +72,15 @@ typedef enum { COSTA_COL_MAJOR = 0, COSTA_ROW_MAJOR = 1 } costa_order;
 typedef enum { COSTA_MODE_DIRECT = 0, COSTA_MODE_MESSAGE = 1 } costa_mode;
 
 /* Storage of one block (Sec. 6, Fig. 1: pointer, stride, ordering).
- *  ptr   - device address of the block's (0, 0) element; aligned to the
- *          element size (16 bytes for COSTA_C128).
+ *  ptr   - address of the block's (0, 0) element; aligned to the element
+ *          size (16 bytes for COSTA_C128).  The block must lie in memory the
+ *          current device can address: its own device memory, managed
+ *          memory, or host memory allocated or registered with CUDA
+ *          (cudaHostAlloc / cudaHostRegister), which the kernels then read
+ *          and write directly over the host link.  This is checked when a
+ *          plan is built, before any kernel runs (COSTA_ERR_LAYOUT for
+ *          pageable host memory, another device's memory or an address
+ *          unknown to CUDA).
  *  ld    - leading dimension in elements: the distance between consecutive
  *          columns (column-major) or rows (row-major); ld >= rows
  *          (column-major) or ld >= cols (row-major); ld < 2^31.

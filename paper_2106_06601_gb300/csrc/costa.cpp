@@ -570,6 +570,126 @@ void append_direct_tiles(const ProblemHost &ph, int prob, int es, int ts, std::v
     if (!contiguous) order_tiles_local(list, first, list.size(), es, ts);
 }
 
+// ---- storage access ----
+//
+// Every nonempty block's first and last element must lie in one allocation
+// the current device can address: its own device memory, managed memory, or
+// host memory allocated or registered with CUDA (the kernels then read and
+// write it over the host link; with unified addressing the host address
+// serves the device too).  Pageable host memory, another device's memory and
+// unknown addresses are rejected with COSTA_ERR_LAYOUT before any kernel
+// runs.  Allocation ranges come from the driver (one query per allocation,
+// then a binary search per block); the result is kept per layout and device.
+
+typedef int (*PointerAttrFn)(void *data, int attribute, unsigned long long ptr);
+
+PointerAttrFn pointer_attr_fn() {
+    static PointerAttrFn fn = [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuPointerGetAttribute", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            f = nullptr;
+        }
+        return reinterpret_cast<PointerAttrFn>(f);
+    }();
+    return fn;
+}
+
+struct AccessRange {
+    uint64_t lo, hi;  // [lo, hi)
+};
+
+// The allocation holding `p` if the device `dev` may access it; on failure
+// a message in `why`.
+bool access_range(uint64_t p, int dev, AccessRange &r, std::string &why) {
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, reinterpret_cast<const void *>(p)) != cudaSuccess) {
+        cudaGetLastError();
+        why = "address unknown to CUDA";
+        return false;
+    }
+    switch (a.type) {
+    case cudaMemoryTypeDevice:
+        if (a.device != dev) {
+            why = "memory of device " + std::to_string(a.device) + ", not of the current device " + std::to_string(dev);
+            return false;
+        }
+        break;
+    case cudaMemoryTypeManaged:
+        break;
+    case cudaMemoryTypeHost:
+        if (reinterpret_cast<uint64_t>(a.devicePointer) != p) {
+            why = "host memory not mapped at the same address on the device";
+            return false;
+        }
+        break;
+    default:
+        why = "pageable host memory (allocate it with cudaHostAlloc or register it with cudaHostRegister)";
+        return false;
+    }
+    r.lo = p;
+    r.hi = p + 1;
+    if (PointerAttrFn fn = pointer_attr_fn()) {
+        unsigned long long start = 0;
+        size_t size = 0;
+        constexpr int kRangeStart = 11, kRangeSize = 12;  // CU_POINTER_ATTRIBUTE_RANGE_START_ADDR / _SIZE
+        if (fn(&start, kRangeStart, p) == 0 && fn(&size, kRangeSize, p) == 0 && size > 0 && start <= p &&
+            p < start + size) {
+            r.lo = start;
+            r.hi = start + size;
+        }
+    }
+    return true;
+}
+
+costa_status check_access(costa_layout_s *L, int dev, const char *which) {
+    if (L->checked_device == dev) return COSTA_OK;
+    const int64_t es = esize_of(L->dt);
+    std::vector<AccessRange> known;  // sorted by lo, disjoint
+    auto covered = [&](uint64_t a, uint64_t b) {  // [a, b] inside one known range
+        auto it = std::upper_bound(known.begin(), known.end(), a,
+                                   [](uint64_t v, const AccessRange &r) { return v < r.lo; });
+        if (it == known.begin()) return false;
+        --it;
+        return a >= it->lo && b < it->hi;
+    };
+    auto add = [&](const AccessRange &r) {
+        auto it = std::lower_bound(known.begin(), known.end(), r.lo,
+                                   [](const AccessRange &k, uint64_t v) { return k.lo < v; });
+        known.insert(it, r);
+    };
+    for (int i = 0; i < L->nbr; ++i) {
+        const int64_t rows = L->R[i + 1] - L->R[i];
+        for (int j = 0; j < L->nbc; ++j) {
+            const int64_t cols = L->C[j + 1] - L->C[j];
+            if (rows == 0 || cols == 0) continue;
+            const DevBlock &b = L->blocks[static_cast<size_t>(i) * L->nbc + j];
+            const int64_t last = b.order == COSTA_COL_MAJOR ? (rows - 1) + (cols - 1) * int64_t(b.ld)
+                                                            : (rows - 1) * int64_t(b.ld) + (cols - 1);
+            const uint64_t first = b.ptr, end = b.ptr + static_cast<uint64_t>((last + 1) * es - 1);
+            if (covered(first, end)) continue;
+            AccessRange r;
+            std::string why;
+            if (!access_range(first, dev, r, why))
+                return fail(COSTA_ERR_LAYOUT, "%s block (%d, %d): %s", which, i, j, why.c_str());
+            if (r.hi <= end) {  // no range from the driver, or the block leaves it
+                AccessRange r2;
+                if (!access_range(end, dev, r2, why))
+                    return fail(COSTA_ERR_LAYOUT, "%s block (%d, %d), last element: %s", which, i, j, why.c_str());
+                if (r.hi - r.lo > 1 || r2.hi - r2.lo > 1)  // ranges known: the block spans two allocations
+                    return fail(COSTA_ERR_LAYOUT, "%s block (%d, %d) spans two allocations", which, i, j);
+                continue;  // both ends accessible, no ranges to cache
+            }
+            add(r);
+        }
+    }
+    L->checked_device = dev;
+    return COSTA_OK;
+}
+
 // Builds the overlay, the tile list and the device tables, and runs the
 // volume kernel.
 costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, const costa_op *ops,
@@ -579,6 +699,11 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     cudaError_t ce = cudaGetDevice(&plan->device);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaGetDevice");
     if (n > 65535) return fail(COSTA_ERR_INVALID_ARG, "batch of %d exceeds 65535 pairs", n);
+    for (int k = 0; k < n; ++k) {
+        costa_status st = check_access(As[k], plan->device, "A");
+        if (st == COSTA_OK) st = check_access(Bs[k], plan->device, "B");
+        if (st != COSTA_OK) return st;
+    }
     plan->dtype = As[0]->dt;
     plan->esize = esize_of(plan->dtype);
     plan->P = As[0]->nranks;

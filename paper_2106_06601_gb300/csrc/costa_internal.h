@@ -37,6 +37,7 @@ struct costa_layout_s {
     std::vector<int64_t> R, C;
     std::vector<int32_t> owner;
     std::vector<costa::DevBlock> blocks;
+    int checked_device = -1;  // device whose access to every block was checked
 };
 
 namespace costa {
