@@ -495,16 +495,7 @@ __device__ __forceinline__ DescRegs load_batch(const RemapLaunch &a, int64_t fir
     return r;
 }
 
-__device__ __forceinline__ TileDesc shfl_desc(const DescRegs &r, int src) {
-    uint4 lo, hi;
-    lo.x = __shfl_sync(0xffffffffu, r.lo.x, src);
-    lo.y = __shfl_sync(0xffffffffu, r.lo.y, src);
-    lo.z = __shfl_sync(0xffffffffu, r.lo.z, src);
-    lo.w = __shfl_sync(0xffffffffu, r.lo.w, src);
-    hi.x = __shfl_sync(0xffffffffu, r.hi.x, src);
-    hi.y = __shfl_sync(0xffffffffu, r.hi.y, src);
-    hi.z = __shfl_sync(0xffffffffu, r.hi.z, src);
-    hi.w = __shfl_sync(0xffffffffu, r.hi.w, src);
+__device__ __forceinline__ TileDesc unpack_desc(const uint4 &lo, const uint4 &hi) {
     TileDesc d;
     d.src = (static_cast<uint64_t>(lo.y) << 32) | lo.x;
     d.dst = (static_cast<uint64_t>(lo.w) << 32) | lo.z;
@@ -515,6 +506,19 @@ __device__ __forceinline__ TileDesc shfl_desc(const DescRegs &r, int src) {
     d.prob = static_cast<uint16_t>(hi.w & 0xFFFFu);
     d.flags = static_cast<uint16_t>(hi.w >> 16);
     return d;
+}
+
+__device__ __forceinline__ TileDesc shfl_desc(const DescRegs &r, int src) {
+    uint4 lo, hi;
+    lo.x = __shfl_sync(0xffffffffu, r.lo.x, src);
+    lo.y = __shfl_sync(0xffffffffu, r.lo.y, src);
+    lo.z = __shfl_sync(0xffffffffu, r.lo.z, src);
+    lo.w = __shfl_sync(0xffffffffu, r.lo.w, src);
+    hi.x = __shfl_sync(0xffffffffu, r.hi.x, src);
+    hi.y = __shfl_sync(0xffffffffu, r.hi.y, src);
+    hi.z = __shfl_sync(0xffffffffu, r.hi.z, src);
+    hi.w = __shfl_sync(0xffffffffu, r.hi.w, src);
+    return unpack_desc(lo, hi);
 }
 
 template <typename T> __device__ __forceinline__ Geom<T> geom_of(const TileDesc &d) {
@@ -658,7 +662,7 @@ template <typename T, int KIND> struct SCfg {
                               : sizeof(T) == 16 ? (KCfg<T, KIND>::READS_A ? COSTA_SMINB_16A : COSTA_SMINB_16)
                               : KCfg<T, KIND>::HEAVY ? COSTA_SMINB_8H : COSTA_SMINB_8;
     static constexpr int NS = group_pieces(static_cast<int>(sizeof(T)));
-    static constexpr int BUF_BYTES = NS * 512;
+    static constexpr int BUF_BYTES = NS * 512 + NS * 32;  // slots, then the group's descriptors
 };
 
 template <typename T, int KIND>
@@ -680,31 +684,32 @@ __global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB
         // 1 .. NS pieces (the host's groups); the clamp keeps the slots inside
         // this warp's buffer regardless
         const int cnt = min(static_cast<int>(g1 - g0), NS);
-        DescRegs r;
+        // lane k copies piece k's descriptor next to the slots; every lane
+        // then reads each descriptor with one broadcast load per half
+        uint4 *dsm = reinterpret_cast<uint4 *>(buf + NS * 512);
         if (lane < cnt) {
             const uint4 *p = reinterpret_cast<const uint4 *>(args.pieces + g0 + lane);
-            r.lo = __ldg(p);
-            r.hi = __ldg(p + 1);
-        } else {
-            r.lo = make_uint4(0, 0, 0, 0);
-            r.hi = make_uint4(0, 0, 0, 0);
+            dsm[2 * lane] = __ldg(p);
+            dsm[2 * lane + 1] = __ldg(p + 1);
         }
+        __syncwarp();
+        auto desc = [&](int k) { return unpack_desc(dsm[2 * k], dsm[2 * k + 1]); };
         if (args.per_problem) {  // one problem per group
-            const int prob = static_cast<int>(shfl_desc(r, 0).prob);
+            const int prob = static_cast<int>(desc(0).prob);
             if (kind_of(args.per_problem[prob].flags) != KIND) continue;
             if (prob != cached) {
                 make_sc(args.per_problem[prob], s);
                 cached = prob;
             }
         }
-        for (int k = 0; k < cnt; ++k) piece_issue<T>(geom_of<T>(shfl_desc(r, k)), buf + 512 * k, lane);
+        for (int k = 0; k < cnt; ++k) piece_issue<T>(geom_of<T>(desc(k)), buf + 512 * k, lane);
         cp_async_commit();
         Chunk<T> av[NS];
         if (READS_A) {
 #pragma unroll
             for (int k = 0; k < NS; ++k) {
                 if (k >= cnt) break;  // uniform across the warp
-                av[k] = piece_load_a<T>(geom_of<T>(shfl_desc(r, k)), lane);
+                av[k] = piece_load_a<T>(geom_of<T>(desc(k)), lane);
             }
             if (KIND == K_AXPBY2) prescale<T>(av, cnt, s);
         }
@@ -713,7 +718,7 @@ __global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB
 #pragma unroll
         for (int k = 0; k < NS; ++k) {
             if (k >= cnt) break;
-            const Geom<T> g = geom_of<T>(shfl_desc(r, k));
+            const Geom<T> g = geom_of<T>(desc(k));
             s.conj_mask = g.conj ? 0x80000000u : 0u;
             piece_drain<T, KIND>(g, s, buf + 512 * k, av[k], lane);
         }
