@@ -159,10 +159,8 @@ struct SplitList {
 };
 
 // A small tile is a fast tile needing fewer passes than small_limit: half
-// of a full tile's passes, a quarter for 8-byte elements (measured on
-// GB300: 16 x 16 tiles of 8-byte elements run faster in the tile kernel,
-// those of 4- and 16-byte elements in the small-tile kernel).
-int small_limit(int es) { return es == 8 ? tile_passes(es) / 4 : tile_passes(es) / 2; }
+// of a full tile's passes (so 16 x 16 tiles of every element type are small).
+int small_limit(int es) { return tile_passes(es) / 2; }
 
 bool is_small(const TileDesc &d, int es) {
     // a pass moves at most 32 chunks: a larger tile cannot be small

@@ -642,7 +642,7 @@ __device__ __forceinline__ void piece_drain(const Geom<T> &g, const Sc &s, unsig
 #define COSTA_SMINB_4 5
 #endif
 #ifndef COSTA_SMINB_8
-#define COSTA_SMINB_8 4
+#define COSTA_SMINB_8 5
 #endif
 #ifndef COSTA_SMINB_8H
 #define COSTA_SMINB_8H 3
