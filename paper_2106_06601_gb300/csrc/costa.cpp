@@ -162,6 +162,12 @@ struct SplitList {
 // of a full tile's passes (so 16 x 16 tiles of every element type are small).
 int small_limit(int es) { return tile_passes(es) / 2; }
 
+// Share (percent) of a list's elements that small tiles must hold for the
+// list to use the small-tile kernel.
+#ifndef COSTA_SMALL_SHARE
+#define COSTA_SMALL_SHARE 50
+#endif
+
 bool is_small(const TileDesc &d, int es) {
     // a pass moves at most 32 chunks: a larger tile cannot be small
     const int64_t area = static_cast<int64_t>(d.nx) * d.ny;
@@ -186,7 +192,7 @@ SplitList split_small(std::vector<TileDesc> &&list, int es) {
         all_elems += e;
         if (is_small(d, es)) small_elems += e;
     }
-    if (2 * small_elems < all_elems) {
+    if (100 * small_elems < COSTA_SMALL_SHARE * all_elems || small_elems == 0) {
         out.big = std::move(list);
         return out;
     }

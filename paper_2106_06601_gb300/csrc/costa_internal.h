@@ -157,7 +157,10 @@ COSTA_HD constexpr int tile_extent(int esize) { return esize == 16 ? COSTA_TS_16
 COSTA_HD constexpr int piece_x(int esize) { return esize == 4 ? 16 : 8; }
 COSTA_HD constexpr int piece_y(int esize) { return esize == 16 ? 4 : 8; }
 COSTA_HD constexpr int tile_passes(int esize) { return tile_extent(esize) * tile_extent(esize) * esize / 512; }
-COSTA_HD constexpr int group_pieces(int esize) { return tile_passes(esize); }
+#ifndef COSTA_GROUP_4
+#define COSTA_GROUP_4 8
+#endif
+COSTA_HD constexpr int group_pieces(int esize) { return esize == 4 ? COSTA_GROUP_4 : tile_passes(esize); }
 
 // Launches the remap kernel for (args.dtype, kind) over a tile list.  With
 // args.per_problem set, the kernel skips the tiles of problems of another kind.
