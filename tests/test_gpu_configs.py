@@ -93,10 +93,10 @@ def blocks_have_no_nan(p, Ad):
     return True
 
 
-@pytest.mark.parametrize("name", ["c2", "c3", "c5"])
+@pytest.mark.parametrize("name", ["c2", "c3", "c5", "c5b", "bc8"])
 def test_config_full_size(name, dev):
     import paper_2106_06601_gb300 as costa
-    p = C.CONFIGS[name]()
+    p = {**C.CONFIGS, **C.EXTRA_WORKLOADS}[name]()
     mat = Mat(p, dev)
     try:
         ij = sample_points(p.A, 200_000, 7)

@@ -130,13 +130,25 @@ def small_blocks(n: int = 8192, mb: int = 8, dtype: str = "f64") -> Problem:
     return Problem(f"bc{mb}", dtype, "T", 2.0, 0.5, A, B, "uniform", "uniform", _seed(6))
 
 
+def c5b(rows: int = 131072, cols: int = 4096) -> Problem:
+    """The other reading of c5's target: A (cols x rows) in 256 column panels
+    of rows / 256 columns, rank k owning panel k, column-major with ld = cols
+    (each panel one contiguous buffer)."""
+    B = L.block_cyclic(rows, cols, 32, 32, 16, 16, grid_order="R", name="B")
+    w = rows // 256
+    A = L.packed_blocks([0, cols], [k * w for k in range(257)], np.arange(256, dtype=np.int32).reshape(1, 256),
+                        256, name="A")
+    return Problem("c5b", "f64", "T", 1.0, 1.0, A, B, "normal", "normal", _seed(5))
+
+
 # Further workloads for measurement only.
-EXTRA_WORKLOADS = {"bc8": small_blocks}
+EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b}
 
 # The same layouts and tile shapes at about 1 GB on the device, for profiler
 # captures (the workloads proper stay the ones above).
 CONFIGS_SMALL = {"c1": c1, "c2": lambda: c2(4096), "c3": lambda: c3(8192),
-                 "c4": lambda: c4(16), "c5": lambda: c5(rows=16384), "bc8": lambda: small_blocks(4096)}
+                 "c4": lambda: c4(16), "c5": lambda: c5(rows=16384), "bc8": lambda: small_blocks(4096),
+                 "c5b": lambda: c5b(rows=16384)}
 
 WORKLOAD_TEXT = {
     "c1": "256x256 f64 BC16 2x2R -> BC32 2x2C, N, alpha=1 beta=0, P=4",
@@ -146,6 +158,8 @@ WORKLOAD_TEXT = {
     "c5": "131072x4096 f64 BC32 16x16 -> 4096x131072 in 256 row panels, T, alpha=1 beta=1, P=256",
     "bc8": "8192x8192 f64 BC8 4x4 -> BC8 4x4 permuted owners, T, alpha=2 beta=0.5, P=16 "
            "(small-block case, not a configuration)",
+    "c5b": "131072x4096 f64 BC32 16x16 -> 4096x131072 in 256 column panels of 512, T, alpha=1 beta=1, "
+           "P=256 (the other reading of c5's target)",
 }
 
 
