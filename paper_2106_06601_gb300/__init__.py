@@ -39,6 +39,11 @@ class _Block(ctypes.Structure):
                 ("reserved", ctypes.c_int32)]
 
 
+# costa_block as a numpy record, for building block arrays without a Python loop
+_BLOCK_DTYPE = np.dtype([("ptr", np.uint64), ("ld", np.int64), ("order", np.int32), ("reserved", np.int32)])
+assert _BLOCK_DTYPE.itemsize == ctypes.sizeof(_Block)
+
+
 class PlanStats(ctypes.Structure):
     _fields_ = [("total_volume", ctypes.c_int64), ("local_identity", ctypes.c_int64),
                 ("local_relabeled", ctypes.c_int64), ("n_cells", ctypes.c_int64),
@@ -159,15 +164,13 @@ def costa_layout_create(dtype: str, nranks: int, row_splits, col_splits, owners,
     order = _i32(block_order).reshape(-1)
     nblk = nbr * nbc
     assert own.size == nblk and ptrs.size == nblk and ld.size == nblk and order.size == nblk
-    blocks = (_Block * max(1, nblk))()
-    for k in range(nblk):
-        blocks[k].ptr = int(ptrs[k])
-        blocks[k].ld = int(ld[k])
-        blocks[k].order = int(order[k])
-        blocks[k].reserved = 0
+    blocks = np.zeros(max(1, nblk), dtype=_BLOCK_DTYPE)
+    blocks["ptr"][:nblk] = ptrs
+    blocks["ld"][:nblk] = ld
+    blocks["order"][:nblk] = order
     out = ctypes.c_void_p()
     _check(_lib.costa_layout_create(ctypes.byref(out), DTYPES[dtype], nranks, nbr, _p(R), nbc,
-                                    _p(C), _p(own), blocks))
+                                    _p(C), _p(own), blocks.ctypes.data))
     return Layout(out.value, dtype)
 
 
