@@ -15,6 +15,7 @@
 #include <memory>
 #include <mutex>
 #include <string>
+#include <thread>
 #include <vector>
 
 #include <cuda_runtime_api.h>
@@ -129,6 +130,44 @@ costa_status check_extents(const std::vector<TileDesc> &list, int es, const char
     return COSTA_OK;
 }
 
+// ---- host threads for plan building ----
+//
+// parallel_for(n, grain, f) calls f(begin, end) on up to plan_threads()
+// contiguous chunks of [0, n), the calling thread taking the first.  It is
+// used only where every chunk writes its own precomputed output range, so a
+// plan does not depend on the number of threads.  COSTA_PLAN_THREADS sets the
+// thread count (default: the hardware threads, at most 16).
+int plan_threads() {
+    static const int t = [] {
+        const char *e = std::getenv("COSTA_PLAN_THREADS");
+        int v = e ? std::atoi(e) : 0;
+        if (v < 1) v = static_cast<int>(std::min(16u, std::max(1u, std::thread::hardware_concurrency())));
+        return std::min(v, 64);
+    }();
+    return t;
+}
+
+thread_local bool t_in_parallel = false;  // nested parallel_for calls run serially
+
+template <typename F> void parallel_for(int64_t n, int64_t grain, F &&f) {
+    const int64_t chunks = std::min<int64_t>(plan_threads(), (n + grain - 1) / std::max<int64_t>(grain, 1));
+    if (chunks <= 1 || t_in_parallel) {
+        if (n > 0) f(int64_t(0), n);
+        return;
+    }
+    std::vector<std::thread> workers;
+    workers.reserve(static_cast<size_t>(chunks - 1));
+    for (int64_t c = 1; c < chunks; ++c)
+        workers.emplace_back([&f, n, c, chunks] {
+            t_in_parallel = true;
+            f(n * c / chunks, n * (c + 1) / chunks);
+        });
+    t_in_parallel = true;
+    f(int64_t(0), n / chunks);
+    t_in_parallel = false;
+    for (std::thread &w : workers) w.join();
+}
+
 void set_fast(TileDesc &d, int es);
 
 int next_pow2(int v) {
@@ -184,56 +223,79 @@ bool is_small(const TileDesc &d, int es) {
 // offsets are multiples of the 16-byte chunk, so the pieces stay on the
 // vector path.  Pieces are grouped in list order, at most group_pieces(es)
 // per group and one problem per group.
+// Cuts a small tile into its pieces (writing them to `out` when non-null);
+// returns the number of pieces, or -1 if a piece would leave the vector path
+// (not expected for a fast tile).
+int cut_pieces(const TileDesc &d, int es, TileDesc *out) {
+    const int px = piece_x(es), py = piece_y(es);
+    const bool tr = (d.flags & TF_TRANSPOSE) != 0;
+    int k = 0;
+    for (int y0 = 0; y0 < d.ny; y0 += py)
+        for (int x0 = 0; x0 < d.nx; x0 += px, ++k) {
+            if (!out) continue;
+            TileDesc pc = d;
+            pc.nx = static_cast<uint16_t>(std::min(px, d.nx - x0));
+            pc.ny = static_cast<uint16_t>(std::min(py, d.ny - y0));
+            pc.dst = d.dst + static_cast<uint64_t>((x0 + static_cast<int64_t>(y0) * d.dld) * es);
+            pc.src = d.src + static_cast<uint64_t>(
+                                 (tr ? static_cast<int64_t>(x0) * d.sld + y0 : x0 + static_cast<int64_t>(y0) * d.sld) * es);
+            set_fast(pc, es);
+            if (!(pc.flags & TF_FAST)) return -1;
+            out[k] = pc;
+        }
+    return k;
+}
+
 SplitList split_small(std::vector<TileDesc> &&list, int es) {
     SplitList out;
+    const int64_t n = static_cast<int64_t>(list.size());
+    std::vector<int32_t> npc(static_cast<size_t>(n));  // pieces of a small tile, 0 for the others
+    parallel_for(n, 1 << 15, [&](int64_t a, int64_t b) {
+        for (int64_t i = a; i < b; ++i) npc[i] = is_small(list[i], es) ? cut_pieces(list[i], es, nullptr) : 0;
+    });
     int64_t small_elems = 0, all_elems = 0;
-    for (const TileDesc &d : list) {
-        const int64_t e = static_cast<int64_t>(d.nx) * d.ny;
+    for (int64_t i = 0; i < n; ++i) {
+        const int64_t e = static_cast<int64_t>(list[i].nx) * list[i].ny;
         all_elems += e;
-        if (is_small(d, es)) small_elems += e;
+        if (npc[i] > 0) small_elems += e;
     }
     if (100 * small_elems < COSTA_SMALL_SHARE * all_elems || small_elems == 0) {
         out.big = std::move(list);
         return out;
     }
-    const int px = piece_x(es), py = piece_y(es), cap = group_pieces(es);
-    int in_group = 0, group_prob = -1;
-    auto add_piece = [&](const TileDesc &pc) {
-        if (in_group == cap || pc.prob != group_prob || out.groups.empty()) {
-            out.groups.push_back(static_cast<uint32_t>(out.pieces.size()));
-            in_group = 0;
-            group_prob = pc.prob;
-        }
-        out.pieces.push_back(pc);
-        ++in_group;
-    };
-    std::vector<TileDesc> cut;
-    for (const TileDesc &d : list) {
-        if (!is_small(d, es)) {
-            out.big.push_back(d);
-            continue;
-        }
-        const bool tr = (d.flags & TF_TRANSPOSE) != 0;
-        cut.clear();
-        bool ok = true;
-        for (int y0 = 0; y0 < d.ny && ok; y0 += py)
-            for (int x0 = 0; x0 < d.nx && ok; x0 += px) {
-                TileDesc pc = d;
-                pc.nx = static_cast<uint16_t>(std::min(px, d.nx - x0));
-                pc.ny = static_cast<uint16_t>(std::min(py, d.ny - y0));
-                pc.dst = d.dst + static_cast<uint64_t>((x0 + static_cast<int64_t>(y0) * d.dld) * es);
-                pc.src = d.src + static_cast<uint64_t>(
-                                     (tr ? static_cast<int64_t>(x0) * d.sld + y0 : x0 + static_cast<int64_t>(y0) * d.sld) *
-                                     es);
-                set_fast(pc, es);
-                ok = (pc.flags & TF_FAST) != 0;
-                cut.push_back(pc);
+    // positions: pieces of small tile i at poff[i], big tile i at boff[i]
+    std::vector<int64_t> poff(static_cast<size_t>(n) + 1), boff(static_cast<size_t>(n) + 1);
+    for (int64_t i = 0; i < n; ++i) {
+        poff[i + 1] = poff[i] + npc[i];
+        boff[i + 1] = boff[i] + (npc[i] > 0 ? 0 : 1);
+    }
+    out.pieces.resize(static_cast<size_t>(poff[n]));
+    out.big.resize(static_cast<size_t>(boff[n]));
+    std::atomic<bool> off_path{false};
+    parallel_for(n, 1 << 14, [&](int64_t a, int64_t b) {
+        for (int64_t i = a; i < b; ++i) {
+            if (npc[i] == 0) {
+                out.big[boff[i]] = list[i];
+            } else if (cut_pieces(list[i], es, out.pieces.data() + poff[i]) < 0) {
+                off_path = true;
             }
-        if (!ok) {  // not expected for a fast tile; keep it whole
-            out.big.push_back(d);
-            continue;
         }
-        for (const TileDesc &pc : cut) add_piece(pc);
+    });
+    if (off_path) {  // not expected: keep every small tile whole
+        out.pieces.clear();
+        out.big = std::move(list);
+        return out;
+    }
+    // groups in list order: at most group_pieces(es) pieces of one problem
+    const int cap = group_pieces(es);
+    int in_group = 0, group_prob = -1;
+    for (size_t k = 0; k < out.pieces.size(); ++k) {
+        if (in_group == cap || out.pieces[k].prob != group_prob || out.groups.empty()) {
+            out.groups.push_back(static_cast<uint32_t>(k));
+            in_group = 0;
+            group_prob = out.pieces[k].prob;
+        }
+        ++in_group;
     }
     if (!out.groups.empty()) out.groups.push_back(static_cast<uint32_t>(out.pieces.size()));
     return out;
@@ -531,13 +593,15 @@ void order_tiles_local(std::vector<TileDesc> &list, size_t first, size_t last, i
     while ((1 << es_shift) < es) ++es_shift;
     std::vector<std::pair<uint64_t, uint32_t>> keys(n);
     std::vector<uint64_t> off(n);
+    parallel_for(static_cast<int64_t>(n), 1 << 15, [&](int64_t a, int64_t b) {
+        for (int64_t i = a; i < b; ++i) {
+            const TileDesc &d = list[first + static_cast<size_t>(i)];
+            off[i] = (d.dst - groups[gid[i]].second) >> es_shift;
+            keys[i] = {off[i] / (static_cast<uint64_t>(d.dld) * strip_elems), static_cast<uint32_t>(i)};
+        }
+    });
     uint64_t max_strip = 0;
-    for (size_t i = 0; i < n; ++i) {
-        const TileDesc &d = list[first + i];
-        off[i] = (d.dst - groups[gid[i]].second) >> es_shift;
-        keys[i] = {off[i] / (static_cast<uint64_t>(d.dld) * strip_elems), static_cast<uint32_t>(i)};
-        max_strip = std::max(max_strip, keys[i].first);
-    }
+    for (const auto &k : keys) max_strip = std::max(max_strip, k.first);
     // key = group * (max_strip + 1) + strip, so that the sort needs only the
     // bits the keys span
     const uint64_t span = max_strip + 1;
@@ -545,27 +609,47 @@ void order_tiles_local(std::vector<TileDesc> &list, size_t first, size_t last, i
         for (size_t i = 0; i < n; ++i) keys[i].first += gid[keys[i].second] * span;
     radix_sort_pairs(keys);
     // inside each strip, by target address
-    for (size_t a = 0; a < n;) {
-        size_t b = a + 1;
-        while (b < n && keys[b].first == keys[a].first) ++b;
-        std::sort(keys.begin() + static_cast<std::ptrdiff_t>(a), keys.begin() + static_cast<std::ptrdiff_t>(b),
-                  [&](const std::pair<uint64_t, uint32_t> &x, const std::pair<uint64_t, uint32_t> &y) {
-                      return off[x.second] < off[y.second];
-                  });
-        a = b;
-    }
+    std::vector<size_t> runs;  // starts of the runs of equal keys, then n
+    for (size_t a = 0; a < n; ++a)
+        if (a == 0 || keys[a].first != keys[a - 1].first) runs.push_back(a);
+    runs.push_back(n);
+    parallel_for(static_cast<int64_t>(runs.size()) - 1, std::max<int64_t>(256, (1 << 15) * static_cast<int64_t>(runs.size()) / std::max<int64_t>(1, static_cast<int64_t>(n))), [&](int64_t r0, int64_t r1) {
+        for (int64_t r = r0; r < r1; ++r)
+            std::sort(keys.begin() + static_cast<std::ptrdiff_t>(runs[r]),
+                      keys.begin() + static_cast<std::ptrdiff_t>(runs[r + 1]),
+                      [&](const std::pair<uint64_t, uint32_t> &x, const std::pair<uint64_t, uint32_t> &y) {
+                          return off[x.second] < off[y.second];
+                      });
+    });
     std::vector<TileDesc> tmp(n);
-    for (size_t k = 0; k < n; ++k) tmp[k] = list[first + keys[k].second];
+    parallel_for(static_cast<int64_t>(n), 1 << 15, [&](int64_t a, int64_t b) {
+        for (int64_t k = a; k < b; ++k) tmp[k] = list[first + keys[k].second];
+    });
     std::copy(tmp.begin(), tmp.end(), list.begin() + static_cast<std::ptrdiff_t>(first));
 }
 
 // Appends the direct tiles of problem `prob` in the kernel's order.
 void append_direct_tiles(const ProblemHost &ph, int prob, int es, int ts, std::vector<TileDesc> &list) {
     const size_t first = list.size();
-    for_each_tile(ph, [&](const AxisTile &rt, const AxisTile &ct) {
-        TileDesc d = direct_tile(ph, rt, ct, es, prob);
-        set_fast(d, es);
-        list.push_back(d);
+    // the order of for_each_tile, built in parallel over bands of kSuper row
+    // pieces: band su holds the tiles [su * nv, (su + band rows) * nv)
+    const int kSuper = super_tile(es);
+    const int64_t nu = static_cast<int64_t>(ph.rows.tiles.size()), nv = static_cast<int64_t>(ph.cols.tiles.size());
+    list.resize(first + static_cast<size_t>(nu * nv));
+    TileDesc *out = list.data() + first;
+    const int64_t band_tiles = std::max<int64_t>(1, int64_t(kSuper) * nv);
+    parallel_for((nu + kSuper - 1) / kSuper, std::max<int64_t>(1, (1 << 15) / band_tiles), [&](int64_t b0, int64_t b1) {
+        for (int64_t band = b0; band < b1; ++band) {
+            const int64_t su = band * kSuper, ue = std::min<int64_t>(su + kSuper, nu);
+            TileDesc *o = out + su * nv;
+            for (int64_t sv = 0; sv < nv; sv += kSuper)
+                for (int64_t v = sv; v < std::min<int64_t>(sv + kSuper, nv); ++v)
+                    for (int64_t u = su; u < ue; ++u) {
+                        TileDesc d = direct_tile(ph, ph.rows.tiles[u], ph.cols.tiles[v], es, prob);
+                        set_fast(d, es);
+                        *o++ = d;
+                    }
+        }
     });
     if (!use_local_order(ph)) return;
     // a target whose tiles are each one contiguous run gains nothing
@@ -736,8 +820,23 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     }
     // the direct tile list, in (problem, row piece, column piece) order
     std::vector<TileDesc> list;
-    list.reserve(static_cast<size_t>(tiles));
-    for (int k = 0; k < n; ++k) append_direct_tiles(plan->probs[k], k, es, ts, list);
+    if (n == 1) {
+        append_direct_tiles(plan->probs[0], 0, es, ts, list);
+    } else {  // a batch: problems in parallel, each into its own range
+        std::vector<int64_t> start(static_cast<size_t>(n) + 1, 0);
+        for (int k = 0; k < n; ++k)
+            start[k + 1] = start[k] + static_cast<int64_t>(plan->probs[k].rows.tiles.size()) *
+                                          static_cast<int64_t>(plan->probs[k].cols.tiles.size());
+        list.resize(static_cast<size_t>(start[n]));
+        parallel_for(n, std::max<int64_t>(1, (int64_t(1) << 15) * n / std::max<int64_t>(1, start[n])),
+                     [&](int64_t k0, int64_t k1) {
+                         for (int64_t k = k0; k < k1; ++k) {
+                             std::vector<TileDesc> part;
+                             append_direct_tiles(plan->probs[k], static_cast<int>(k), es, ts, part);
+                             std::copy(part.begin(), part.end(), list.begin() + start[k]);
+                         }
+                     });
+    }
     {
         costa_status st = check_extents(list, es, "direct");
         if (st != COSTA_OK) return st;

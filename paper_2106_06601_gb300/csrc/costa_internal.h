@@ -71,6 +71,9 @@ struct Interval {
 //   source element (x, y) at src + (x + y * sld) elements (copy tile)
 //                         or src + (x * sld + y) elements (transposed tile)
 struct TileDesc {
+    // Left uninitialized: tile lists are sized first and then filled in
+    // place, in parallel, so zeroing them would only add a serial pass.
+    COSTA_HD TileDesc() {}
     uint64_t src;    // device address of source element (0, 0)
     uint64_t dst;    // device address of target element (0, 0)
     int32_t sld;     // source stride (elements)
