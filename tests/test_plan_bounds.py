@@ -278,3 +278,38 @@ def test_c4_and_fuzz_split():
 def test_small_block_split():
     for case in range(120):
         check_split(C.small_block_problem(case), exact=True)
+
+
+_DUMP = """
+import hashlib, sys
+sys.path.insert(0, %r)
+import numpy as np
+import paper_2106_06601_gb300 as costa
+from workloads import configs as C
+from tests.test_plan_bounds import _layout
+h = hashlib.sha256()
+for p in (C.c3(8192), C.small_blocks(2048), C.c5(rows=16384), C.small_block_problem(4)):
+    LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+    for part in costa.costa_debug_split(LA, LB, p.op):
+        h.update(np.ascontiguousarray(part).tobytes())
+    LA.destroy()
+    LB.destroy()
+print(h.hexdigest())
+"""
+
+
+def test_plan_independent_of_thread_count():
+    """Tile lists, their order and the pieces are the same whatever the
+    number of planning threads."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = []
+    for t in ("1", "3", "8"):
+        env = dict(os.environ, COSTA_PLAN_THREADS=t)
+        r = subprocess.run([sys.executable, "-c", _DUMP % root], env=env, capture_output=True, text=True,
+                           cwd=root, timeout=600)
+        assert r.returncode == 0, r.stderr
+        out.append(r.stdout.strip())
+    assert out[0] == out[1] == out[2]
