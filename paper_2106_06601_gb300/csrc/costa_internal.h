@@ -151,7 +151,10 @@ struct VolumeLaunch {
 #ifndef COSTA_TS_16
 #define COSTA_TS_16 32
 #endif
-COSTA_HD constexpr int tile_extent(int esize) { return esize == 16 ? COSTA_TS_16 : 32; }
+#ifndef COSTA_TS_4
+#define COSTA_TS_4 32
+#endif
+COSTA_HD constexpr int tile_extent(int esize) { return esize == 16 ? COSTA_TS_16 : esize == 4 ? COSTA_TS_4 : 32; }
 
 // Small tiles are cut by the host into pieces of at most piece_x x piece_y
 // elements, each exactly one warp pass (32 lanes x 16 bytes at most), and
