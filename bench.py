@@ -46,7 +46,8 @@ KERNEL_SOURCES = ["paper_2106_06601_gb300/csrc/remap_impl.cuh",
                   "paper_2106_06601_gb300/csrc/remap_f32.cu",
                   "paper_2106_06601_gb300/csrc/remap_c64.cu",
                   "paper_2106_06601_gb300/csrc/remap_c128.cu",
-                  "paper_2106_06601_gb300/csrc/costa.cpp"]  # tile lists and their order
+                  "paper_2106_06601_gb300/csrc/tiles.cpp",  # tile lists, their order, small-tile pieces
+                  "paper_2106_06601_gb300/csrc/tiles.h"]
 
 
 def parse():

@@ -21,6 +21,7 @@
 #include <cuda_runtime_api.h>
 
 #include "costa_internal.h"
+#include "tiles.h"
 
 namespace costa {
 
@@ -48,76 +49,8 @@ costa_status cuda_fail(cudaError_t e, const char *what) {
     return fail(COSTA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-int esize_of(int dt) {
-    switch (dt) {
-    case COSTA_F32: return 4;
-    case COSTA_F64: return 8;
-    case COSTA_C64: return 8;
-    case COSTA_C128: return 16;
-    default: return 0;
-    }
-}
-
 double ms_since(std::chrono::steady_clock::time_point t0) {
     return std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
-}
-
-// ---------------------------------------------------------------------------
-// Grid overlay along one axis (Sec. 5): the sorted union of A's splits and
-// op(B)'s splits cuts the axis into intervals, each inside exactly one block
-// of A and one block of op(B) (the unique cover).  Empty blocks are skipped.
-// ---------------------------------------------------------------------------
-struct AxisCut {
-    std::vector<Interval> intervals;
-    std::vector<AxisTile> tiles;
-};
-
-// Cuts one axis into pieces of at most ts elements.  When an interval starts
-// off a 16-byte boundary (vec elements) of the side chosen by `align_a`
-// (A's block if true, else op(B)'s), one short first piece reaches the
-// boundary, so that the remaining pieces start aligned and can use vector
-// accesses; otherwise the pieces are ts long from the interval's start.
-AxisCut cut_axis(const std::vector<int64_t> &SA, const std::vector<int64_t> &SB, int64_t extent,
-                 int ts, int vec, bool align_a) {
-    AxisCut out;
-    const int nA = static_cast<int>(SA.size()) - 1, nB = static_cast<int>(SB.size()) - 1;
-    int ka = 0, kb = 0;
-    int64_t pos = 0;
-    while (pos < extent) {
-        while (ka + 1 < nA && SA[ka + 1] <= pos) ++ka;
-        while (kb + 1 < nB && SB[kb + 1] <= pos) ++kb;
-        const int64_t end = std::min(SA[ka + 1], SB[kb + 1]);
-        const int64_t len = end - pos;
-        const int cell = static_cast<int>(out.intervals.size());
-        out.intervals.push_back(Interval{ka, kb, len});
-        const int64_t a0 = pos - SA[ka], b0 = pos - SB[kb];
-        int64_t q = 0;
-        const int64_t phase = (align_a ? a0 : b0) % vec;
-        while (q < len) {
-            const int64_t want = (q == 0 && phase != 0) ? vec - phase : ts;
-            const int64_t piece = std::min<int64_t>(want, len - q);
-            out.tiles.push_back(AxisTile{ka, kb, static_cast<int32_t>(a0 + q),
-                                         static_cast<int32_t>(b0 + q),
-                                         static_cast<int32_t>(piece), cell});
-            q += piece;
-        }
-        pos = end;
-    }
-    return out;
-}
-
-// Cuts axis 0 (rows) or 1 (columns) of A for the pair (A, op(B)).  Each axis
-// is aligned to the side whose contiguous axis it is (decided by the first
-// block's order: column-major makes rows contiguous), so that side's runs
-// start on 16-byte boundaries.
-AxisCut cut_pair_axis(const costa_layout_s *A, const costa_layout_s *B, int op, int axis, int ts) {
-    const bool tr = op != COSTA_OP_N;
-    const int vec = 16 / esize_of(A->dt);
-    const bool a_rows_fast = A->blocks.empty() || A->blocks[0].order == COSTA_COL_MAJOR;
-    const bool b_col = B->blocks.empty() || B->blocks[0].order == COSTA_COL_MAJOR;
-    const bool b_rows_fast = tr ? !b_col : b_col;  // op(B)'s contiguous axis is rows
-    if (axis == 0) return cut_axis(A->R, tr ? B->C : B->R, A->m, ts, vec, a_rows_fast || !b_rows_fast);
-    return cut_axis(A->C, tr ? B->R : B->C, A->n, ts, vec, !a_rows_fast || b_rows_fast);
 }
 
 // Every tile of a list fits the kernel's tile extent along both axes (the
@@ -128,177 +61,6 @@ costa_status check_extents(const std::vector<TileDesc> &list, int es, const char
         if (d.nx < 1 || d.ny < 1 || d.nx > ts || d.ny > ts)
             return fail(COSTA_ERR_INTERNAL, "%s tile %d x %d exceeds the tile extent %d", what, d.nx, d.ny, ts);
     return COSTA_OK;
-}
-
-// ---- host threads for plan building ----
-//
-// parallel_for(n, grain, f) calls f(begin, end) on up to plan_threads()
-// contiguous chunks of [0, n), the calling thread taking the first.  It is
-// used only where every chunk writes its own precomputed output range, so a
-// plan does not depend on the number of threads.  COSTA_PLAN_THREADS sets the
-// thread count (default: the hardware threads, at most 16).
-int plan_threads() {
-    static const int t = [] {
-        const char *e = std::getenv("COSTA_PLAN_THREADS");
-        int v = e ? std::atoi(e) : 0;
-        if (v < 1) v = static_cast<int>(std::min(16u, std::max(1u, std::thread::hardware_concurrency())));
-        return std::min(v, 64);
-    }();
-    return t;
-}
-
-thread_local bool t_in_parallel = false;  // nested parallel_for calls run serially
-
-template <typename F> void parallel_for(int64_t n, int64_t grain, F &&f) {
-    const int64_t chunks = std::min<int64_t>(plan_threads(), (n + grain - 1) / std::max<int64_t>(grain, 1));
-    if (chunks <= 1 || t_in_parallel) {
-        if (n > 0) f(int64_t(0), n);
-        return;
-    }
-    std::vector<std::thread> workers;
-    workers.reserve(static_cast<size_t>(chunks - 1));
-    for (int64_t c = 1; c < chunks; ++c)
-        workers.emplace_back([&f, n, c, chunks] {
-            t_in_parallel = true;
-            f(n * c / chunks, n * (c + 1) / chunks);
-        });
-    t_in_parallel = true;
-    f(int64_t(0), n / chunks);
-    t_in_parallel = false;
-    for (std::thread &w : workers) w.join();
-}
-
-void set_fast(TileDesc &d, int es);
-
-int next_pow2(int v) {
-    int p = 1;
-    while (p < v) p <<= 1;
-    return p;
-}
-
-// Warp passes the tile kernel needs for a fast tile: the larger of its
-// staging and drain pass counts, with the kernel's lane maps (a run of c
-// chunks takes the next power of two >= c lanes; 32 lanes per pass).
-int fast_tile_passes(const TileDesc &d, int es) {
-    const int vec = 16 / es;
-    const bool tr = (d.flags & TF_TRANSPOSE) != 0;
-    const int runs = tr ? d.nx : d.ny;
-    const int rpp_s = 32 / next_pow2((tr ? d.ny : d.nx) / vec);
-    const int rpp_d = 32 / next_pow2(d.nx / vec);
-    return std::max((runs + rpp_s - 1) / rpp_s, (d.ny + rpp_d - 1) / rpp_d);
-}
-
-// A tile list split for the two remap kernels: full-size tiles for the tile
-// kernel, and the one-pass pieces of the small tiles with their groups for
-// the small-tile kernel.
-struct SplitList {
-    std::vector<TileDesc> big, pieces;
-    std::vector<uint32_t> groups;  // group g = pieces [groups[g], groups[g + 1])
-    int64_t ngroups() const { return groups.empty() ? 0 : static_cast<int64_t>(groups.size()) - 1; }
-};
-
-// A small tile is a fast tile needing fewer passes than small_limit: half
-// of a full tile's passes (so 16 x 16 tiles of every element type are small).
-int small_limit(int es) { return tile_passes(es) / 2; }
-
-// Share (percent) of a list's elements that small tiles must hold for the
-// list to use the small-tile kernel.
-#ifndef COSTA_SMALL_SHARE
-#define COSTA_SMALL_SHARE 50
-#endif
-
-bool is_small(const TileDesc &d, int es) {
-    // a pass moves at most 32 chunks: a larger tile cannot be small
-    const int64_t area = static_cast<int64_t>(d.nx) * d.ny;
-    if (area * es >= int64_t(512) * small_limit(es) || !(d.flags & TF_FAST)) return false;
-    return fast_tile_passes(d, es) < small_limit(es);
-}
-
-// Splits a list between the kernels.  Only a list whose small tiles hold at
-// least half of its elements uses the small-tile kernel: in a mixed list the
-// warps on small tiles wait on latency while the others keep DRAM busy, and
-// one launch over the whole list measured faster than two (c4: 6157 against
-// 5787 GB/s).  A small tile is cut into pieces of at most piece_x x piece_y
-// (x fastest, so that consecutive pieces continue the target's runs); piece
-// offsets are multiples of the 16-byte chunk, so the pieces stay on the
-// vector path.  Pieces are grouped in list order, at most group_pieces(es)
-// per group and one problem per group.
-// Cuts a small tile into its pieces (writing them to `out` when non-null);
-// returns the number of pieces, or -1 if a piece would leave the vector path
-// (not expected for a fast tile).
-int cut_pieces(const TileDesc &d, int es, TileDesc *out) {
-    const int px = piece_x(es), py = piece_y(es);
-    const bool tr = (d.flags & TF_TRANSPOSE) != 0;
-    int k = 0;
-    for (int y0 = 0; y0 < d.ny; y0 += py)
-        for (int x0 = 0; x0 < d.nx; x0 += px, ++k) {
-            if (!out) continue;
-            TileDesc pc = d;
-            pc.nx = static_cast<uint16_t>(std::min(px, d.nx - x0));
-            pc.ny = static_cast<uint16_t>(std::min(py, d.ny - y0));
-            pc.dst = d.dst + static_cast<uint64_t>((x0 + static_cast<int64_t>(y0) * d.dld) * es);
-            pc.src = d.src + static_cast<uint64_t>(
-                                 (tr ? static_cast<int64_t>(x0) * d.sld + y0 : x0 + static_cast<int64_t>(y0) * d.sld) * es);
-            set_fast(pc, es);
-            if (!(pc.flags & TF_FAST)) return -1;
-            out[k] = pc;
-        }
-    return k;
-}
-
-SplitList split_small(std::vector<TileDesc> &&list, int es) {
-    SplitList out;
-    const int64_t n = static_cast<int64_t>(list.size());
-    std::vector<int32_t> npc(static_cast<size_t>(n));  // pieces of a small tile, 0 for the others
-    parallel_for(n, 1 << 15, [&](int64_t a, int64_t b) {
-        for (int64_t i = a; i < b; ++i) npc[i] = is_small(list[i], es) ? cut_pieces(list[i], es, nullptr) : 0;
-    });
-    int64_t small_elems = 0, all_elems = 0;
-    for (int64_t i = 0; i < n; ++i) {
-        const int64_t e = static_cast<int64_t>(list[i].nx) * list[i].ny;
-        all_elems += e;
-        if (npc[i] > 0) small_elems += e;
-    }
-    if (100 * small_elems < COSTA_SMALL_SHARE * all_elems || small_elems == 0) {
-        out.big = std::move(list);
-        return out;
-    }
-    // positions: pieces of small tile i at poff[i], big tile i at boff[i]
-    std::vector<int64_t> poff(static_cast<size_t>(n) + 1), boff(static_cast<size_t>(n) + 1);
-    for (int64_t i = 0; i < n; ++i) {
-        poff[i + 1] = poff[i] + npc[i];
-        boff[i + 1] = boff[i] + (npc[i] > 0 ? 0 : 1);
-    }
-    out.pieces.resize(static_cast<size_t>(poff[n]));
-    out.big.resize(static_cast<size_t>(boff[n]));
-    std::atomic<bool> off_path{false};
-    parallel_for(n, 1 << 14, [&](int64_t a, int64_t b) {
-        for (int64_t i = a; i < b; ++i) {
-            if (npc[i] == 0) {
-                out.big[boff[i]] = list[i];
-            } else if (cut_pieces(list[i], es, out.pieces.data() + poff[i]) < 0) {
-                off_path = true;
-            }
-        }
-    });
-    if (off_path) {  // not expected: keep every small tile whole
-        out.pieces.clear();
-        out.big = std::move(list);
-        return out;
-    }
-    // groups in list order: at most group_pieces(es) pieces of one problem
-    const int cap = group_pieces(es);
-    int in_group = 0, group_prob = -1;
-    for (size_t k = 0; k < out.pieces.size(); ++k) {
-        if (in_group == cap || out.pieces[k].prob != group_prob || out.groups.empty()) {
-            out.groups.push_back(static_cast<uint32_t>(k));
-            in_group = 0;
-            group_prob = out.pieces[k].prob;
-        }
-        ++in_group;
-    }
-    if (!out.groups.empty()) out.groups.push_back(static_cast<uint32_t>(out.pieces.size()));
-    return out;
 }
 
 // Device copies of a split list inside a plan's arena.
@@ -313,13 +75,6 @@ struct DevList {
 
 struct SplitOffsets {
     size_t tiles, pieces, groups;
-};
-
-struct ProblemHost {
-    const costa_layout_s *A;
-    const costa_layout_s *B;
-    costa_op op;
-    AxisCut rows, cols;
 };
 
 // One device allocation holding all tables of a plan, built on the host
@@ -450,212 +205,6 @@ costa_status validate_pair(const costa_layout_s *A, const costa_layout_s *B, int
         return fail(COSTA_ERR_SHAPE, "A is %lld x %lld but op(B) is %lld x %lld", (long long)A->m,
                     (long long)A->n, (long long)bm, (long long)bn);
     return COSTA_OK;
-}
-
-bool aligned16(uint64_t addr, int64_t ld_bytes) { return ((addr | static_cast<uint64_t>(ld_bytes)) & 15) == 0; }
-
-// The tile (rt, ct) of a problem in the kernel's canonical frame (x = A's
-// contiguous axis): source and target addresses of element (0, 0), strides,
-// extents, and whether source and target runs lie on different axes.
-TileDesc direct_tile(const ProblemHost &ph, const AxisTile &rt, const AxisTile &ct, int es, int prob) {
-    const DevBlock &dA = ph.A->blocks[static_cast<size_t>(rt.a_blk) * ph.A->nbc + ct.a_blk];
-    const bool tr = ph.op != COSTA_OP_N;
-    const DevBlock &dB = tr ? ph.B->blocks[static_cast<size_t>(ct.b_blk) * ph.B->nbc + rt.b_blk]
-                            : ph.B->blocks[static_cast<size_t>(rt.b_blk) * ph.B->nbc + ct.b_blk];
-    const bool b_col = dB.order == COSTA_COL_MAJOR;
-    const int64_t rb = tr ? ct.b_off : rt.b_off, cb = tr ? rt.b_off : ct.b_off;
-    const bool src_fast_i = tr ? !b_col : b_col;  // source runs along A's rows
-    const bool a_col = dA.order == COSTA_COL_MAJOR;
-    TileDesc d;
-    d.src = dB.ptr + static_cast<uint64_t>((b_col ? rb + cb * dB.ld : rb * dB.ld + cb) * es);
-    d.dst = dA.ptr + static_cast<uint64_t>(
-                         (a_col ? rt.a_off + static_cast<int64_t>(ct.a_off) * dA.ld
-                                : static_cast<int64_t>(rt.a_off) * dA.ld + ct.a_off) * es);
-    d.sld = dB.ld;
-    d.dld = dA.ld;
-    d.nx = static_cast<uint16_t>(a_col ? rt.len : ct.len);
-    d.ny = static_cast<uint16_t>(a_col ? ct.len : rt.len);
-    d.prob = static_cast<uint16_t>(prob);
-    d.flags = 0;
-    if (a_col != src_fast_i) d.flags |= TF_TRANSPOSE;
-    if (ph.op == COSTA_OP_C) d.flags |= TF_CONJ;
-    return d;
-}
-
-// Sets TF_FAST when every run is whole 16-byte chunks on both sides.
-void set_fast(TileDesc &d, int es) {
-    const int vec = 16 / es;
-    const bool tr = (d.flags & TF_TRANSPOSE) != 0;
-    const int src_run = tr ? d.ny : d.nx;
-    const bool fast = aligned16(d.dst, static_cast<int64_t>(d.dld) * es) &&
-                      aligned16(d.src, static_cast<int64_t>(d.sld) * es) && d.nx % vec == 0 &&
-                      src_run % vec == 0;
-    d.flags = static_cast<uint16_t>(fast ? (d.flags | TF_FAST) : (d.flags & ~TF_FAST));
-}
-
-// Visits the tiles of a problem in super-tiles of k x k pieces,
-// row pieces fastest inside each: the tiles that warps work on at the same
-// time then cover compact regions of A and of B (runs of kSuper tiles along
-// both axes) instead of one band of rows across every column.
-// Default k: 16 for 16-byte elements (16 x 16 tiles), 8 otherwise (measured
-// on GB300).  The environment variable COSTA_SUPER_TILE (1..64) overrides it,
-// for tuning.
-int super_tile(int esize) {
-    static const int env = [] {
-        const char *e = std::getenv("COSTA_SUPER_TILE");
-        const int v = e ? std::atoi(e) : 0;
-        return v >= 1 && v <= 64 ? v : 0;
-    }();
-    return env ? env : (esize == 16 ? 16 : 8);
-}
-
-template <typename F> void for_each_tile(const ProblemHost &ph, F &&f) {
-    const int kSuper = super_tile(esize_of(ph.A->dt));
-    const int nu = static_cast<int>(ph.rows.tiles.size()), nv = static_cast<int>(ph.cols.tiles.size());
-    for (int su = 0; su < nu; su += kSuper)
-        for (int sv = 0; sv < nv; sv += kSuper)
-            for (int v = sv; v < std::min(sv + kSuper, nv); ++v)
-                for (int u = su; u < std::min(su + kSuper, nu); ++u) f(ph.rows.tiles[u], ph.cols.tiles[v]);
-}
-
-// Tile order in the target's own storage.  For a transposed problem (op = T
-// or C) the source tiles that warps read at the same time are scattered
-// across the source whatever the order, so the order serves the target,
-// which is read and written: each target buffer is walked in strips of
-// kLocalStrip tiles across its non-contiguous axis, each strip down the
-// buffer's contiguous axis, so that concurrent tiles form long contiguous
-// runs of target memory.  Measured on GB300: +6.6% on 16384^2 c128 (C) and
-// +2% on 8192^2 f64 (T); no gain for 4-byte elements (32 x 32 f32 tiles) and
-// a loss for op = N, whose source runs the global order keeps.  The
-// environment variable COSTA_TILE_ORDER (global | local) overrides the rule,
-// for tuning.
-constexpr int kLocalStrip = 2;
-
-bool use_local_order(const ProblemHost &ph) {
-    static const int env = [] {
-        const char *e = std::getenv("COSTA_TILE_ORDER");
-        if (!e) return -1;
-        if (std::strcmp(e, "global") == 0) return 0;
-        if (std::strcmp(e, "local") == 0) return 1;
-        return -1;
-    }();
-    if (env >= 0) return env == 1;
-    return ph.op != COSTA_OP_N && esize_of(ph.A->dt) >= 8;
-}
-
-// Stable LSD radix sort of (key, index) pairs by key, 11 bits per pass (the
-// counts and the scatter targets stay in cache); passes stop at the highest
-// bit in which two keys differ, and a pass whose digit is equal for every
-// key is skipped.
-void radix_sort_pairs(std::vector<std::pair<uint64_t, uint32_t>> &v) {
-    constexpr int kBits = 11, kBuckets = 1 << kBits;
-    std::vector<std::pair<uint64_t, uint32_t>> tmp(v.size());
-    std::vector<size_t> count(kBuckets + 1);
-    uint64_t lo = ~uint64_t(0), hi = 0;
-    for (const auto &e : v) {
-        lo = std::min(lo, e.first);
-        hi = std::max(hi, e.first);
-    }
-    for (int shift = 0; shift < 64; shift += kBits) {
-        if (((lo ^ hi) >> shift) == 0) break;  // keys agree on every higher bit
-        std::fill(count.begin(), count.end(), size_t(0));
-        for (const auto &e : v) ++count[((e.first >> shift) & (kBuckets - 1)) + 1];
-        bool uniform = false;
-        for (int d = 1; d <= kBuckets; ++d)
-            if (count[d] == v.size()) uniform = true;
-        if (uniform) continue;
-        for (int d = 1; d <= kBuckets; ++d) count[d] += count[d - 1];
-        for (const auto &e : v) tmp[count[(e.first >> shift) & (kBuckets - 1)]++] = e;
-        v.swap(tmp);
-    }
-}
-
-// Reorders tiles [first, last) (one problem) into the target-local order.
-// Tiles are grouped by target stride; within a group an element's local
-// coordinates are taken from its offset to the group's lowest target
-// address: y = offset / stride (the non-contiguous axis), then strips of
-// kLocalStrip * ts along y, ordered by address inside each strip.
-void order_tiles_local(std::vector<TileDesc> &list, size_t first, size_t last, int es, int ts) {
-    const size_t n = last - first;
-    if (n < 2) return;
-    std::vector<std::pair<int32_t, uint64_t>> groups;  // (stride, lowest target address)
-    std::vector<uint32_t> gid(n);
-    for (size_t i = 0; i < n; ++i) {
-        const TileDesc &d = list[first + i];
-        size_t g = 0;
-        while (g < groups.size() && groups[g].first != d.dld) ++g;
-        if (g == groups.size()) groups.emplace_back(d.dld, d.dst);
-        else groups[g].second = std::min(groups[g].second, d.dst);
-        gid[i] = static_cast<uint32_t>(g);
-    }
-    const uint64_t strip_elems = static_cast<uint64_t>(kLocalStrip) * static_cast<uint64_t>(ts);
-    int es_shift = 0;
-    while ((1 << es_shift) < es) ++es_shift;
-    std::vector<std::pair<uint64_t, uint32_t>> keys(n);
-    std::vector<uint64_t> off(n);
-    parallel_for(static_cast<int64_t>(n), 1 << 15, [&](int64_t a, int64_t b) {
-        for (int64_t i = a; i < b; ++i) {
-            const TileDesc &d = list[first + static_cast<size_t>(i)];
-            off[i] = (d.dst - groups[gid[i]].second) >> es_shift;
-            keys[i] = {off[i] / (static_cast<uint64_t>(d.dld) * strip_elems), static_cast<uint32_t>(i)};
-        }
-    });
-    uint64_t max_strip = 0;
-    for (const auto &k : keys) max_strip = std::max(max_strip, k.first);
-    // key = group * (max_strip + 1) + strip, so that the sort needs only the
-    // bits the keys span
-    const uint64_t span = max_strip + 1;
-    if (groups.size() > 1 && span <= ~uint64_t(0) / groups.size())
-        for (size_t i = 0; i < n; ++i) keys[i].first += gid[keys[i].second] * span;
-    radix_sort_pairs(keys);
-    // inside each strip, by target address
-    std::vector<size_t> runs;  // starts of the runs of equal keys, then n
-    for (size_t a = 0; a < n; ++a)
-        if (a == 0 || keys[a].first != keys[a - 1].first) runs.push_back(a);
-    runs.push_back(n);
-    parallel_for(static_cast<int64_t>(runs.size()) - 1, std::max<int64_t>(256, (1 << 15) * static_cast<int64_t>(runs.size()) / std::max<int64_t>(1, static_cast<int64_t>(n))), [&](int64_t r0, int64_t r1) {
-        for (int64_t r = r0; r < r1; ++r)
-            std::sort(keys.begin() + static_cast<std::ptrdiff_t>(runs[r]),
-                      keys.begin() + static_cast<std::ptrdiff_t>(runs[r + 1]),
-                      [&](const std::pair<uint64_t, uint32_t> &x, const std::pair<uint64_t, uint32_t> &y) {
-                          return off[x.second] < off[y.second];
-                      });
-    });
-    std::vector<TileDesc> tmp(n);
-    parallel_for(static_cast<int64_t>(n), 1 << 15, [&](int64_t a, int64_t b) {
-        for (int64_t k = a; k < b; ++k) tmp[k] = list[first + keys[k].second];
-    });
-    std::copy(tmp.begin(), tmp.end(), list.begin() + static_cast<std::ptrdiff_t>(first));
-}
-
-// Appends the direct tiles of problem `prob` in the kernel's order.
-void append_direct_tiles(const ProblemHost &ph, int prob, int es, int ts, std::vector<TileDesc> &list) {
-    const size_t first = list.size();
-    // the order of for_each_tile, built in parallel over bands of kSuper row
-    // pieces: band su holds the tiles [su * nv, (su + band rows) * nv)
-    const int kSuper = super_tile(es);
-    const int64_t nu = static_cast<int64_t>(ph.rows.tiles.size()), nv = static_cast<int64_t>(ph.cols.tiles.size());
-    list.resize(first + static_cast<size_t>(nu * nv));
-    TileDesc *out = list.data() + first;
-    const int64_t band_tiles = std::max<int64_t>(1, int64_t(kSuper) * nv);
-    parallel_for((nu + kSuper - 1) / kSuper, std::max<int64_t>(1, (1 << 15) / band_tiles), [&](int64_t b0, int64_t b1) {
-        for (int64_t band = b0; band < b1; ++band) {
-            const int64_t su = band * kSuper, ue = std::min<int64_t>(su + kSuper, nu);
-            TileDesc *o = out + su * nv;
-            for (int64_t sv = 0; sv < nv; sv += kSuper)
-                for (int64_t v = sv; v < std::min<int64_t>(sv + kSuper, nv); ++v)
-                    for (int64_t u = su; u < ue; ++u) {
-                        TileDesc d = direct_tile(ph, ph.rows.tiles[u], ph.cols.tiles[v], es, prob);
-                        set_fast(d, es);
-                        *o++ = d;
-                    }
-        }
-    });
-    if (!use_local_order(ph)) return;
-    // a target whose tiles are each one contiguous run gains nothing
-    bool contiguous = true;
-    for (size_t i = first; i < list.size() && contiguous; ++i) contiguous = list[i].nx == list[i].dld;
-    if (!contiguous) order_tiles_local(list, first, list.size(), es, ts);
 }
 
 // ---- storage access ----
