@@ -176,8 +176,11 @@ costa_status costa_relabel(int P, const int64_t *V, int *sigma, int64_t *local_v
  *                same either way.
  *  sigma_out   - nullable host array of P ints; receives sigma (identity when
  *                relabel == 0).
+ * Once the plan for (A, B, op) exists, a call only enqueues kernels on
+ * `stream`, so it can be captured in a CUDA graph and replayed (build the
+ * plan with a first call or costa_plan_stats_get before capturing).
  * Errors: INVALID_ARG, SHAPE (dims(A) != dims(op(B)), P differs), DTYPE,
- * ALLOC, CUDA. */
+ * LAYOUT (storage the device cannot address, see costa_block), ALLOC, CUDA. */
 costa_status costa_transform(costa_layout A, costa_layout B, costa_op op,
                              const void *alpha, const void *beta, int relabel,
                              int *sigma_out, void *stream);

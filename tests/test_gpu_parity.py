@@ -269,3 +269,36 @@ def test_phase_timing(dev):
     finally:
         costa.costa_phase_timing(False)
         g.close()
+
+
+def test_transform_replays_in_cuda_graph(dev):
+    """Once its plan exists, a transform call only enqueues kernels on the
+    caller's stream, so it can be captured in a CUDA graph and replayed; the
+    replays give the oracle's result (for beta != 0 each replay reads the A
+    left by the previous one)."""
+    import paper_2106_06601_gb300 as costa
+    p = C.fuzz_problem(12, dtype="f64", P=4)
+    p.alpha, p.beta = 2.0, 0.5
+    g = OnDevice(p, dev)
+    try:
+        s = torch.cuda.Stream(dev)
+        costa.costa_transform(g.LA, g.LB, p.op, p.alpha, p.beta, relabel=True, stream=s.cuda_stream)
+        torch.cuda.synchronize(dev)
+        g.reset_A()
+        torch.cuda.synchronize(dev)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=s):
+            costa.costa_transform(g.LA, g.LB, p.op, p.alpha, p.beta, relabel=True,
+                                  stream=torch.cuda.current_stream().cuda_stream)
+        # capture records without running: A is unchanged until the replays
+        want = g.Ah.copy()
+        for _ in range(3):
+            graph.replay()
+            torch.cuda.synchronize(dev)
+            import oracle
+            oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, want.buffers(), p.B, g.Bh.buffers())
+            got = g.Ad.download()
+            ok = (got.arena == want.arena) | (np.isnan(got.arena) & np.isnan(want.arena))
+            assert np.all(ok)
+    finally:
+        g.close()
