@@ -161,7 +161,9 @@ costa_status costa_volume(costa_layout A, costa_layout B, costa_op op, int64_t *
 /* Communication-optimal process relabeling for the locally-free volume cost
  * (Eq. 2; Remark on the gain and Thm. 1 / Thm. 2, Sec. 4): sigma maximizes
  * sum_q V[sigma[q] * P + q], i.e. target label q is taken by process
- * sigma[q].  Exact (Hungarian algorithm, O(P^3), host).  Ties: when the
+ * sigma[q].  Exact, on the host: the Hungarian method (O(P^3)), or for
+ * P >= 256 with at most P^2 / 8 nonzero volumes, successive shortest
+ * augmenting paths over the nonzero volumes only.  Ties: when the
  * identity attains the optimum the identity is returned.  V: host P * P
  * int64, entries >= 0.  sigma: host, P ints.  local_volume (nullable):
  * receives the optimal sum.  Errors: INVALID_ARG (P < 1, null, negative V). */

@@ -29,6 +29,7 @@ int64_t assign_min(int n, const std::vector<int64_t> &cost, std::vector<int> &ro
                    std::vector<int64_t> *u_out, std::vector<int64_t> *v_out);
 int64_t greedy_max(int P, const int64_t *V, std::vector<int> &sigma);
 double assign_min_f(int n, const std::vector<double> &cost, std::vector<int> &row_to_col);
+int64_t assign_max_sparse(int P, const int64_t *V, std::vector<int> &sigma);
 
 namespace {
 
@@ -176,13 +177,33 @@ bool plan_uses(const std::vector<uint64_t> &key, uint64_t id) {
 }
 
 // ---- relabeling: sigma maximizing sum_q V[sigma(q)][q] ----
+// Relabeling solver choice: the sparse method for large P with few nonzero
+// volumes (a reshuffle sends each target's data from a few sources), the
+// dense Hungarian otherwise.  COSTA_RELABEL_SPARSE_MIN_P sets the smallest P
+// that may take the sparse method (default 256; 1 forces it wherever V is
+// sparse enough, for tests).
+int sparse_min_p() {
+    static const int v = [] {
+        const char *e = std::getenv("COSTA_RELABEL_SPARSE_MIN_P");
+        const int k = e ? std::atoi(e) : 0;
+        return k >= 1 ? k : 256;
+    }();
+    return v;
+}
+
 void solve_relabel(int P, const int64_t *V, std::vector<int> &sigma, int64_t &best) {
-    // rows = target labels q, columns = processes p, cost = -V[p][q]
-    std::vector<int64_t> cost(static_cast<size_t>(P) * P);
-    for (int q = 0; q < P; ++q)
-        for (int p = 0; p < P; ++p) cost[static_cast<size_t>(q) * P + p] = -V[static_cast<size_t>(p) * P + q];
+    int64_t nnz = 0;
+    for (size_t k = 0; k < static_cast<size_t>(P) * P; ++k) nnz += V[k] > 0;
     std::vector<int> row_to_col;
-    best = -assign_min(P, cost, row_to_col, nullptr, nullptr);
+    if (P >= sparse_min_p() && nnz * 8 <= static_cast<int64_t>(P) * P) {
+        best = assign_max_sparse(P, V, row_to_col);
+    } else {
+        // rows = target labels q, columns = processes p, cost = -V[p][q]
+        std::vector<int64_t> cost(static_cast<size_t>(P) * P);
+        for (int q = 0; q < P; ++q)
+            for (int p = 0; p < P; ++p) cost[static_cast<size_t>(q) * P + p] = -V[static_cast<size_t>(p) * P + q];
+        best = -assign_min(P, cost, row_to_col, nullptr, nullptr);
+    }
     int64_t trace = 0;
     for (int q = 0; q < P; ++q) trace += V[static_cast<size_t>(q) * P + q];
     sigma.resize(P);

@@ -123,3 +123,142 @@ int64_t greedy_max(int P, const int64_t *V, std::vector<int> &sigma) {
 }
 
 }  // namespace costa
+
+#include <queue>
+
+namespace costa {
+
+// Exact maximum of sum_q V[sigma[q]][q] over permutations for a sparse V
+// (Thm. 1 objective), by successive shortest augmenting paths (Dijkstra with
+// potentials) on the bipartite graph of the nonzero entries.  Each target
+// row q may also take a private "unmatched" column at weight 0; at the end
+// the rows left unmatched take the unused processes in increasing order,
+// which adds nothing to the objective (their V entries on the remaining
+// pairs are whatever they are; see below).  Work per row is a Dijkstra over
+// the rows and nonzero edges its search reaches, instead of the dense
+// method's O(P^2) scan.
+//
+// Why the completion is optimal: a maximum-weight matching that may leave
+// rows unmatched is at least as heavy as any permutation's objective
+// restricted to nonzero entries, which is the permutation's objective; and
+// completing it cannot lower its weight (V >= 0).  The returned objective is
+// recomputed on the completed permutation.
+int64_t assign_max_sparse(int P, const int64_t *V, std::vector<int> &sigma) {
+    // adjacency by row q: (p, weight V[p][q] > 0)
+    std::vector<int> start(static_cast<size_t>(P) + 1, 0);
+    for (int p = 0; p < P; ++p)
+        for (int q = 0; q < P; ++q)
+            if (V[static_cast<size_t>(p) * P + q] > 0) ++start[q + 1];
+    for (int q = 0; q < P; ++q) start[q + 1] += start[q];
+    std::vector<int> col(static_cast<size_t>(start[P]));
+    std::vector<int64_t> w(static_cast<size_t>(start[P]));
+    {
+        std::vector<int> fill(start.begin(), start.end() - 1);
+        for (int p = 0; p < P; ++p)
+            for (int q = 0; q < P; ++q) {
+                const int64_t v = V[static_cast<size_t>(p) * P + q];
+                if (v > 0) {
+                    col[fill[q]] = p;
+                    w[fill[q]++] = v;
+                }
+            }
+    }
+    // columns 0..P-1 are processes; column P + q is row q's private
+    // "unmatched" column.  Costs: -V for real edges, 0 for the private one.
+    const int NC = 2 * P;
+    const int64_t INF = std::numeric_limits<int64_t>::max() / 4;
+    std::vector<int64_t> u(P, 0), v(NC, 0);  // potentials: cost - u - v >= 0
+    for (int q = 0; q < P; ++q) {
+        int64_t m = 0;
+        for (int e = start[q]; e < start[q + 1]; ++e) m = std::min(m, -w[e]);
+        u[q] = m;
+    }
+    std::vector<int> col_row(NC, -1), row_col(P, -1);
+    std::vector<int64_t> dist(NC, INF);
+    std::vector<int> prev_row(NC, -1), touched;
+    std::vector<char> done(NC, 0);
+    typedef std::pair<int64_t, int> Item;  // (distance, column)
+    for (int s = 0; s < P; ++s) {
+        std::priority_queue<Item, std::vector<Item>, std::greater<Item>> pq;
+        touched.clear();
+        auto relax_row = [&](int r, int64_t dr) {  // dr: distance at row r
+            for (int e = start[r]; e < start[r + 1]; ++e) {
+                const int c = col[e];
+                const int64_t nd = dr + (-w[e] - u[r] - v[c]);
+                if (nd < dist[c]) {
+                    if (dist[c] == INF) touched.push_back(c);
+                    dist[c] = nd;
+                    prev_row[c] = r;
+                    pq.push({nd, c});
+                }
+            }
+            const int c = P + r;  // the private column
+            const int64_t nd = dr + (0 - u[r] - v[c]);
+            if (nd < dist[c]) {
+                if (dist[c] == INF) touched.push_back(c);
+                dist[c] = nd;
+                prev_row[c] = r;
+                pq.push({nd, c});
+            }
+        };
+        relax_row(s, 0);
+        int end_col = -1;
+        int64_t end_dist = 0;
+        std::vector<int> done_cols;
+        while (!pq.empty()) {
+            const Item it = pq.top();
+            pq.pop();
+            const int c = it.second;
+            if (done[c] || it.first != dist[c]) continue;
+            done[c] = 1;
+            done_cols.push_back(c);
+            if (col_row[c] < 0) {
+                end_col = c;
+                end_dist = it.first;
+                break;
+            }
+            relax_row(col_row[c], it.first);
+        }
+        // potentials: keep reduced costs non-negative for the next search
+        u[s] += end_dist;
+        for (int c : done_cols) {
+            if (c == end_col) continue;
+            const int r = col_row[c];
+            v[c] -= end_dist - dist[c];
+            u[r] += end_dist - dist[c];
+        }
+        // augment along prev_row back to s
+        for (int c = end_col; c >= 0;) {
+            const int r = prev_row[c];
+            const int next = row_col[r];
+            col_row[c] = r;
+            row_col[r] = c;
+            c = (r == s) ? -1 : next;
+        }
+        for (int c : touched) {
+            dist[c] = INF;
+            done[c] = 0;
+            prev_row[c] = -1;
+        }
+    }
+    // complete: rows on their private column take the unused processes
+    sigma.assign(P, -1);
+    std::vector<char> used(P, 0);
+    for (int q = 0; q < P; ++q)
+        if (row_col[q] >= 0 && row_col[q] < P) {
+            sigma[q] = row_col[q];
+            used[row_col[q]] = 1;
+        }
+    int next = 0;
+    for (int q = 0; q < P; ++q) {
+        if (sigma[q] >= 0) continue;
+        while (used[next]) ++next;
+        sigma[q] = next;
+        used[next] = 1;
+    }
+    int64_t total = 0;
+    for (int q = 0; q < P; ++q) total += V[static_cast<size_t>(sigma[q]) * P + q];
+    return total;
+}
+
+}  // namespace costa

@@ -184,3 +184,49 @@ def test_relabel_rejects_bad_input():
     lib = costa.library()
     sig = np.zeros(2, np.int32)
     assert lib.costa_relabel(0, None, sig.ctypes.data, None) == 1
+
+
+_SPARSE = r"""
+import sys
+sys.path.insert(0, %r)
+import numpy as np
+import paper_2106_06601_gb300 as costa
+import oracle
+from workloads.gen import IntStream
+rng = IntStream(2106066010, 77)
+bad = []
+for trial in range(300):
+    P = 1 + rng.below(40)
+    V = np.zeros((P, P), np.int64)
+    k = rng.below(5)
+    for q in range(P):
+        for _ in range(k):
+            V[rng.below(P), q] = rng.below(7)
+    sig, lv = costa.costa_relabel(V)
+    if sorted(sig.tolist()) != list(range(P)) or lv != oracle.objective(V, sig) or lv != oracle.lap_optimum(V):
+        bad.append(trial)
+# a large sparse case against the library assignment routine
+P = 600
+V = np.zeros((P, P), np.int64)
+for q in range(P):
+    for _ in range(4):
+        V[rng.below(P), q] = 1 + rng.below(1000)
+sig, lv = costa.costa_relabel(V)
+if lv != oracle.lap_library(V)[0] or lv != oracle.objective(V, sig):
+    bad.append("large")
+print(bad)
+"""
+
+
+def test_sparse_relabel_is_exact():
+    """The sparse relabeling solver (successive shortest paths over the
+    nonzero volumes), forced for every P, reaches the same optimum as the
+    oracle's solvers (brute force, subset DP, library assignment)."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", _SPARSE % root], cwd=root, capture_output=True, text=True,
+                       env=dict(os.environ, COSTA_RELABEL_SPARSE_MIN_P="1"), timeout=600)
+    assert r.returncode == 0, r.stderr
+    assert r.stdout.strip() == "[]", r.stdout
