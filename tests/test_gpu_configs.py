@@ -170,3 +170,37 @@ def test_config_c4_batched(dev):
     finally:
         for m in mats:
             m.close()
+
+
+def test_more_than_2_31_elements(dev):
+    """A matrix of 65536 x 36864 f32 (2.4e9 elements, 9.7 GB per side): every
+    element count, offset and volume sum passes 2^31.  Sampled outputs against
+    the oracle; V sums to m * n; B untouched."""
+    import paper_2106_06601_gb300 as costa
+    from workloads import layouts as L
+    m, n = 65536, 36864
+    perm = [(5 * k + 3) % 16 for k in range(16)]
+    B = L.block_cyclic(m, n, 128, 128, 4, 4, name="B")
+    A = L.block_cyclic(n, m, 256, 256, 4, 4, rank_perm=perm, name="A")
+    p = C.Problem("big", "f32", "T", 2.0, 0.5, A, B, "uniform", "uniform", C.SEED0 + 31)
+    assert p.A.m * p.A.n > 2 ** 31
+    mat = Mat(p, dev)
+    try:
+        ij = sample_points(p.A, 100_000, 11)
+        # the far corner, whose offsets are the largest
+        ij = np.concatenate([ij, np.array([[p.A.m - 1, p.A.n - 1], [p.A.m - 1, 0], [0, p.A.n - 1]])])
+        ia, ib = mat.sample_index(ij)
+        a_pre = mat.Ad.arena[ia].cpu().numpy()
+        b = mat.Bd.arena[ib].cpu().numpy()
+        b_sum = mat.Bd.arena.sum(dtype=torch.float64).item()
+        stream = torch.cuda.current_stream().cuda_stream
+        costa.costa_transform(mat.LA, mat.LB, p.op, p.alpha, p.beta, relabel=True, stream=stream)
+        torch.cuda.synchronize()
+        check_samples(p, a_pre, b, mat.Ad.arena[ia].cpu().numpy())
+        assert mat.Bd.arena.sum(dtype=torch.float64).item() == b_sum
+        V = costa.costa_volume(mat.LA, mat.LB, p.op, stream)
+        assert int(V.sum()) == p.A.m * p.A.n
+    finally:
+        mat.close()
+        del mat
+        torch.cuda.empty_cache()
