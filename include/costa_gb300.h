@@ -363,7 +363,8 @@ costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void
  * pass each (at most 8 x 8 elements; 16 x 8 for 4-byte and 8 x 4 for
  * 16-byte elements, x along A's contiguous axis), which the small-tile
  * kernel moves in groups of up to a full tile's passes; the other tiles stay
- * with the tile kernel.  Writes up to cap_tiles full-size tiles to `tiles`
+ * with the tile kernel (those whose runs are not 16-byte aligned after the
+ * others, for its one-element-per-lane instance).  Writes up to cap_tiles full-size tiles to `tiles`
  * and up to cap_pieces pieces to `pieces` (32-byte descriptors as in
  * costa_debug_tiles), and up to cap_groups group offsets to `groups` (group
  * g covers pieces [groups[g], groups[g + 1]), so there are *ngroups + 1

@@ -68,14 +68,16 @@ costa_status check_extents(const std::vector<TileDesc> &list, int es, const char
 struct DevList {
     const TileDesc *tiles = nullptr;
     int64_t ntiles = 0;
+    const TileDesc *mtiles = nullptr;
+    int64_t nmtiles = 0;
     const TileDesc *pieces = nullptr;
     const uint32_t *groups = nullptr;
     int64_t ngroups = 0;
-    bool empty() const { return ntiles == 0 && ngroups == 0; }
+    bool empty() const { return ntiles == 0 && nmtiles == 0 && ngroups == 0; }
 };
 
 struct SplitOffsets {
-    size_t tiles, pieces, groups;
+    size_t tiles, mtiles, pieces, groups;
 };
 
 // One device allocation holding all tables of a plan, built on the host
@@ -91,13 +93,17 @@ struct Arena {
     template <typename V> size_t add_vec(const std::vector<V> &v) {
         return add(v.data(), v.size() * sizeof(V));
     }
-    SplitOffsets add_split(const SplitList &l) { return {add_vec(l.big), add_vec(l.pieces), add_vec(l.groups)}; }
+    SplitOffsets add_split(const SplitList &l) {
+        return {add_vec(l.big), add_vec(l.mis), add_vec(l.pieces), add_vec(l.groups)};
+    }
 };
 
 DevList resolve(const char *dbase, const SplitOffsets &o, const SplitList &l) {
     DevList d;
     d.tiles = reinterpret_cast<const TileDesc *>(dbase + o.tiles);
     d.ntiles = static_cast<int64_t>(l.big.size());
+    d.mtiles = reinterpret_cast<const TileDesc *>(dbase + o.mtiles);
+    d.nmtiles = static_cast<int64_t>(l.mis.size());
     d.pieces = reinterpret_cast<const TileDesc *>(dbase + o.pieces);
     d.groups = reinterpret_cast<const uint32_t *>(dbase + o.groups);
     d.ngroups = l.ngroups();
@@ -739,6 +745,8 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         RemapLaunch l = L;
         l.tiles = list.tiles;
         l.ntiles = list.ntiles;
+        l.mtiles = list.mtiles;
+        l.nmtiles = list.nmtiles;
         l.pieces = list.pieces;
         l.groups = list.groups;
         l.ngroups = list.ngroups;
@@ -764,6 +772,8 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     RemapLaunch lp{};
     lp.tiles = m.pack.tiles;
     lp.ntiles = m.pack.ntiles;
+    lp.mtiles = m.pack.mtiles;
+    lp.nmtiles = m.pack.nmtiles;
     lp.pieces = m.pack.pieces;
     lp.groups = m.pack.groups;
     lp.ngroups = m.pack.ngroups;
@@ -1143,13 +1153,15 @@ costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void
     std::vector<TileDesc> list;
     append_direct_tiles(ph, 0, es, ts, list);
     const SplitList sp = split_small(std::move(list), es);
-    *ntiles = static_cast<int64_t>(sp.big.size());
+    std::vector<TileDesc> whole = sp.big;  // the tile kernel's tiles: aligned, then misaligned
+    whole.insert(whole.end(), sp.mis.begin(), sp.mis.end());
+    *ntiles = static_cast<int64_t>(whole.size());
     *npieces = static_cast<int64_t>(sp.pieces.size());
     *ngroups = sp.ngroups();
     const size_t kt = static_cast<size_t>(std::min<int64_t>(cap_tiles, *ntiles));
     const size_t kp = static_cast<size_t>(std::min<int64_t>(cap_pieces, *npieces));
     const size_t kg = static_cast<size_t>(std::min<int64_t>(cap_groups, static_cast<int64_t>(sp.groups.size())));
-    if (kt) std::memcpy(tiles, sp.big.data(), kt * sizeof(TileDesc));
+    if (kt) std::memcpy(tiles, whole.data(), kt * sizeof(TileDesc));
     if (kp) std::memcpy(pieces, sp.pieces.data(), kp * sizeof(TileDesc));
     if (kg) std::memcpy(groups, sp.groups.data(), kg * sizeof(uint32_t));
     return COSTA_OK;

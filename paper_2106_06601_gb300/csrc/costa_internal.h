@@ -115,8 +115,10 @@ COSTA_HD inline int kind_of(int32_t flags) {
 
 
 struct RemapLaunch {
-    const TileDesc *tiles;       // full-size tiles (the tile kernel)
+    const TileDesc *tiles;       // aligned full-size tiles (the tile kernel)
     int64_t ntiles;
+    const TileDesc *mtiles;      // misaligned tiles (the tile kernel, one element per lane)
+    int64_t nmtiles;
     const TileDesc *pieces;      // one-pass pieces of small tiles (the small-tile kernel)
     const uint32_t *groups;      // group g = pieces [groups[g], groups[g + 1])
     int64_t ngroups;

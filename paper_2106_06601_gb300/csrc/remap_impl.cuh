@@ -21,8 +21,8 @@
 //      transform after receive).
 // If A and the source share their contiguous axis the staged rows are read
 // straight; otherwise they are read across rows (the transpose of Sec. 6's
-// "cache-friendly ... kernel for matrix transposition").  Ragged or
-// misaligned tiles take an element-wise path.
+// "cache-friendly ... kernel for matrix transposition").  Tiles whose runs
+// are not 16-byte aligned take the same pipeline one element per lane.
 //
 // The kernel walks a list of tile descriptors (TileDesc) resolved on the host:
 // the direct list (every tile: B -> A), or the message path of Alg. 3 /
@@ -140,6 +140,14 @@ template <typename T> struct Chunk {
 __device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
     const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
+}
+// One element (4, 8 or 16 bytes) at its natural alignment.
+template <int BYTES> __device__ __forceinline__ void cp_async_elem(void *smem, const void *gmem) {
+    const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+    if constexpr (BYTES == 16)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
+    else
+        asm volatile("cp.async.ca.shared.global [%0], [%1], %2;\n" ::"r"(s), "l"(gmem), "n"(BYTES) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 template <int N> __device__ __forceinline__ void cp_async_wait() {
@@ -430,8 +438,10 @@ template <int KIND> __device__ __forceinline__ double2 premul(double2 a, const S
     return KIND == K_AXPBY2 ? make_double2(__dmul_rn(s.br, a.x), __dmul_rn(s.br, a.y)) : a;
 }
 
-// Element-wise path for ragged or misaligned tiles, lanes strided along the
-// contiguous axis of each phase; uses a TS x (TS + 1) array in `buf`.
+// Element-wise fallback of the aligned kernel for a tile that is not on the
+// vector path (the host lists none there; misaligned tiles go to the
+// one-element-per-lane instance): lanes strided along the contiguous axis of
+// each phase, through a TS x (TS + 1) array in `buf`.
 template <typename T, int KIND>
 __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
     using C = Cfg<T>;
@@ -460,6 +470,79 @@ __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsi
     }
 }
 
+// ---- misaligned tiles: the same pipeline, one element per lane ----
+//
+// A tile whose runs do not start on 16-byte boundaries (an odd leading
+// dimension, a block at an odd offset) cannot use 16-byte chunks.  It takes
+// the same steps with one element per lane: cp.async of single elements into
+// shared memory, A's elements loaded into registers before the wait, and
+// element-wide, still coalesced, stores.  Staged rows are TS elements wide;
+// element c of row r lives at position c ^ (r mod TS), so that lanes reading
+// one position across consecutive rows (the transposed read) hit distinct
+// banks.
+
+template <typename T>
+__device__ __forceinline__ T *slot_e(unsigned char *buf, int r, int c) {
+    using C = Cfg<T>;
+    return reinterpret_cast<T *>(buf) + r * C::TS + (c ^ (r & (C::TS - 1)));
+}
+
+template <typename T>
+__device__ __forceinline__ void stage_issue_e(const Geom<T> &g, unsigned char *buf, int lane) {
+    const int runs = g.transpose ? g.nx : g.ny;
+    const int len = g.transpose ? g.ny : g.nx;  // elements per run
+    const LaneMap m = lane_map(len, lane);
+    if (m.c >= len) return;
+#pragma unroll 4
+    for (int r = m.r0; r < runs; r += m.rpp)
+        cp_async_elem<sizeof(T)>(slot_e<T>(buf, r, m.c), g.src + static_cast<int64_t>(r) * g.sld + m.c);
+}
+
+// Element e of the warp's NPASS * VEC register elements (compile-time e).
+template <typename T> __device__ __forceinline__ T &elem(Chunk<T> (&av)[Cfg<T>::NPASS], int e) {
+    return av[e / Cfg<T>::VEC].e[e % Cfg<T>::VEC];
+}
+
+template <typename T, int KIND>
+__device__ __forceinline__ void load_a_e(const Geom<T> &g, const Sc &s, Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
+    using C = Cfg<T>;
+    if (KIND == K_COPY || KIND == K_SCALE) return;
+    constexpr int NE = C::NPASS * C::VEC;  // elements per lane, full tile
+    const LaneMap m = lane_map(g.nx, lane);
+    const bool on = m.c < g.nx;
+    const int npass = (g.ny + m.rpp - 1) / m.rpp;
+    const int npad = (npass + C::VEC - 1) / C::VEC * C::VEC;  // whole chunks for prescale
+#pragma unroll
+    for (int p = 0; p < NE; ++p) {
+        if (p >= npad) break;  // uniform across the warp
+        const int y = p * m.rpp + m.r0;
+        T a;
+        if constexpr (ET<T>::CPLX) a = T{0, 0}; else a = T(0);
+        if (on && p < npass && y < g.ny) a = g.dst[static_cast<int64_t>(y) * g.dld + m.c];
+        elem<T>(av, p) = a;
+    }
+    if (KIND == K_AXPBY2) prescale<T>(av, (npass + C::VEC - 1) / C::VEC, s);
+}
+
+template <typename T, int KIND>
+__device__ __forceinline__ void stage_drain_e(const Geom<T> &g, const Sc &s, unsigned char *buf,
+                                              Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
+    using C = Cfg<T>;
+    constexpr int NE = C::NPASS * C::VEC;
+    const LaneMap m = lane_map(g.nx, lane);
+    if (m.c >= g.nx) return;
+    const int npass = (g.ny + m.rpp - 1) / m.rpp;
+#pragma unroll
+    for (int p = 0; p < NE; ++p) {
+        if (p >= npass) break;
+        const int y = p * m.rpp + m.r0;
+        if (y < g.ny) {
+            const T b = g.transpose ? *slot_e<T>(buf, m.c, y) : *slot_e<T>(buf, y, m.c);
+            g.dst[static_cast<int64_t>(y) * g.dld + m.c] = combine<KIND>(b, elem<T>(av, p), s);
+        }
+    }
+}
+
 // Scalars of a problem in the kernel's form.
 __device__ __forceinline__ void make_sc(const Scalars &S, Sc &s) {
     s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
@@ -480,12 +563,13 @@ struct DescRegs {
     uint4 lo, hi;
 };
 
+template <bool MIS>
 __device__ __forceinline__ DescRegs load_batch(const RemapLaunch &a, int64_t first, int64_t stride,
                                                int64_t b, int lane) {
     DescRegs r;
     const int64_t t = first + (b * 32 + lane) * stride;
-    if (t < a.ntiles) {
-        const uint4 *p = reinterpret_cast<const uint4 *>(a.tiles + t);
+    if (t < (MIS ? a.nmtiles : a.ntiles)) {
+        const uint4 *p = reinterpret_cast<const uint4 *>((MIS ? a.mtiles : a.tiles) + t);
         r.lo = __ldg(p);
         r.hi = __ldg(p + 1);
     } else {
@@ -545,16 +629,16 @@ struct TileStream {
 // Next tile of the warp; false when none is left.  With per-problem scalars,
 // tiles of problems of another kind are skipped (another launch covers
 // them).  Called by all 32 lanes with the same state.
-template <typename T, int KIND>
+template <typename T, int KIND, bool MIS>
 __device__ __forceinline__ bool next_tile(const RemapLaunch &a, int64_t first, int64_t stride,
                                           TileStream &ts, Geom<T> &g, int lane) {
     for (;;) {
         const int64_t t = first + ts.j * stride;
-        if (t >= a.ntiles) return false;
+        if (t >= (MIS ? a.nmtiles : a.ntiles)) return false;
         const int k = static_cast<int>(ts.j & 31);
         if (k == 0 && ts.j > 0) {
             ts.cur = ts.nxt;
-            ts.nxt = load_batch(a, first, stride, (ts.j >> 5) + 1, lane);
+            ts.nxt = load_batch<MIS>(a, first, stride, (ts.j >> 5) + 1, lane);
         }
         const TileDesc d = shfl_desc(ts.cur, k);
         ++ts.j;
@@ -726,9 +810,17 @@ __global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB
     }
 }
 
-// Writes one tile (staged in `buf` if it is a fast tile).  `cached` holds
-// the problem whose scalars are in `s`.
-template <typename T, int KIND, int NB>
+// Stages a tile's source: 16-byte chunks, or single elements in the kernel
+// for misaligned tiles (MIS).
+template <typename T, bool MIS>
+__device__ __forceinline__ void stage_any(const Geom<T> &g, unsigned char *buf, int lane) {
+    if constexpr (MIS) stage_issue_e<T>(g, buf, lane);
+    else if (g.fast) stage_issue<T>(g, buf, lane);  // the element-wise fallback stages nothing
+}
+
+// Writes one staged tile.  `cached` holds the problem whose scalars are in
+// `s`.
+template <typename T, int KIND, int NB, bool MIS>
 __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &g, Sc &s, int &cached,
                                            unsigned char *buf, int lane) {
     using C = Cfg<T>;
@@ -737,10 +829,16 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
         cached = g.prob;
     }
     s.conj_mask = g.conj ? 0x80000000u : 0u;
-    if (g.fast) {
+    if constexpr (MIS) {
+        Chunk<T> av[C::NPASS];
+        load_a_e<T, KIND>(g, s, av, lane);
+        cp_async_wait<NB - 1>();  // this tile's copies (later tiles' may still fly)
+        __syncwarp();
+        stage_drain_e<T, KIND>(g, s, buf, av, lane);
+    } else if (g.fast) {
         Chunk<T> av[C::NPASS];
         load_a<T, KIND>(g, s, av, lane);
-        cp_async_wait<NB - 1>();  // this tile's copies (later tiles' may still fly)
+        cp_async_wait<NB - 1>();
         __syncwarp();
         stage_drain<T, KIND>(g, s, buf, av, lane);
     } else {
@@ -749,7 +847,12 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
     __syncwarp();  // the buffer is free before it is staged into again
 }
 
-template <typename T, int KIND>
+// The tile kernel.  MIS = false moves the aligned ("fast") tiles of
+// args.tiles with 16-byte chunks; MIS = true moves the misaligned tiles of
+// args.mtiles one element per lane.  The host puts every tile in the right
+// list; a tile of the other kind is skipped, so no 16-byte access is ever
+// made at a misaligned address.
+template <typename T, int KIND, bool MIS>
 __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB)
     remap_kernel(const RemapLaunch args) {
     using C = Cfg<T>;
@@ -765,17 +868,17 @@ __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB
     if (!args.per_problem) make_sc(args.s, s);
     TileStream ts;
     ts.j = 0;
-    ts.cur = load_batch(args, first, stride, 0, lane);
-    ts.nxt = load_batch(args, first, stride, 1, lane);
+    ts.cur = load_batch<MIS>(args, first, stride, 0, lane);
+    ts.nxt = load_batch<MIS>(args, first, stride, 1, lane);
 
     // ring[0] is the tile being written, ring[k] the tile k ahead, staged in
     // buffer (cur + k) % NB
     if constexpr (NB == 1) {  // no look-ahead: copy, wait, write, one tile at a time
         Geom<T> g;
-        while (next_tile<T, KIND>(args, first, stride, ts, g, lane)) {
-            if (g.fast) stage_issue<T>(g, bufs, lane);
+        while (next_tile<T, KIND, MIS>(args, first, stride, ts, g, lane)) {
+            stage_any<T, MIS>(g, bufs, lane);
             cp_async_commit();
-            write_tile<T, KIND, 1>(args, g, s, cached, bufs, lane);
+            write_tile<T, KIND, 1, MIS>(args, g, s, cached, bufs, lane);
         }
         return;
     }
@@ -783,19 +886,19 @@ __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB
     bool have[NB > 1 ? NB : 2];
 #pragma unroll
     for (int k = 0; k < NB - 1; ++k) {
-        have[k] = (k == 0 || have[k - 1]) && next_tile<T, KIND>(args, first, stride, ts, ring[k], lane);
-        if (have[k] && ring[k].fast) stage_issue<T>(ring[k], bufs + k * C::BUF_BYTES, lane);
+        have[k] = (k == 0 || have[k - 1]) && next_tile<T, KIND, MIS>(args, first, stride, ts, ring[k], lane);
+        if (have[k]) stage_any<T, MIS>(ring[k], bufs + k * C::BUF_BYTES, lane);
         cp_async_commit();
     }
     int cur = 0;
     constexpr int LA = NB > 1 ? NB - 1 : 1;  // index of the look-ahead slot
     while (have[0]) {
-        have[LA] = have[LA - 1] && next_tile<T, KIND>(args, first, stride, ts, ring[LA], lane);
+        have[LA] = have[LA - 1] && next_tile<T, KIND, MIS>(args, first, stride, ts, ring[LA], lane);
         int ahead = cur + NB - 1;
         if (ahead >= NB) ahead -= NB;
-        if (have[LA] && ring[LA].fast) stage_issue<T>(ring[LA], bufs + ahead * C::BUF_BYTES, lane);
+        if (have[LA]) stage_any<T, MIS>(ring[LA], bufs + ahead * C::BUF_BYTES, lane);
         cp_async_commit();
-        write_tile<T, KIND, NB>(args, ring[0], s, cached, bufs + cur * C::BUF_BYTES, lane);
+        write_tile<T, KIND, NB, MIS>(args, ring[0], s, cached, bufs + cur * C::BUF_BYTES, lane);
 #pragma unroll
         for (int k = 0; k < LA; ++k) {
             ring[k] = ring[k + 1];
@@ -817,9 +920,9 @@ inline int sm_count() {
     return cached;
 }
 
-template <typename T, int KIND>
+template <typename T, int KIND, bool MIS>
 cudaError_t launch_tiles(const RemapLaunch &a, cudaStream_t st) {
-    auto kern = remap_kernel<T, KIND>;
+    auto kern = remap_kernel<T, KIND, MIS>;
     constexpr int kWarps = Cfg<T>::WARPS;
     const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND>::NBUF * Cfg<T>::BUF_BYTES;
     static int per_sm = 0;
@@ -831,7 +934,8 @@ cudaError_t launch_tiles(const RemapLaunch &a, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         if (per_sm < 1) per_sm = 1;
     }
-    const int64_t want = (a.ntiles + kWarps - 1) / kWarps;
+    const int64_t n = MIS ? a.nmtiles : a.ntiles;
+    const int64_t want = (n + kWarps - 1) / kWarps;
     const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;
     const int blocks = static_cast<int>(want < cap ? want : cap);
     if (blocks <= 0) return cudaSuccess;
@@ -863,11 +967,13 @@ cudaError_t launch_small(const RemapLaunch &a, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-// The tile kernel over the full-size tiles, then the small-tile kernel over
-// the groups of pieces (each launched only when it has work).
+// The tile kernel over the aligned full-size tiles, then over the
+// misaligned ones, then the small-tile kernel over the groups of pieces
+// (each launched only when it has work).
 template <typename T, int KIND>
 cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
-    cudaError_t e = a.ntiles > 0 ? launch_tiles<T, KIND>(a, st) : cudaSuccess;
+    cudaError_t e = a.ntiles > 0 ? launch_tiles<T, KIND, false>(a, st) : cudaSuccess;
+    if (e == cudaSuccess && a.nmtiles > 0) e = launch_tiles<T, KIND, true>(a, st);
     if (e == cudaSuccess && a.ngroups > 0) e = launch_small<T, KIND>(a, st);
     return e;
 }

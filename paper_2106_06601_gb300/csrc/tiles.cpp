@@ -136,8 +136,21 @@ int cut_pieces(const TileDesc &d, int es, TileDesc *out) {
     return k;
 }
 
-SplitList split_small(std::vector<TileDesc> &&list, int es) {
+SplitList split_small(std::vector<TileDesc> &&all, int es) {
     SplitList out;
+    // misaligned tiles go to their own instance of the tile kernel
+    std::vector<TileDesc> list;
+    {
+        size_t nmis = 0;
+        for (const TileDesc &d : all) nmis += (d.flags & TF_FAST) ? 0 : 1;
+        if (nmis == 0) {
+            list = std::move(all);
+        } else {
+            list.reserve(all.size() - nmis);
+            out.mis.reserve(nmis);
+            for (const TileDesc &d : all) ((d.flags & TF_FAST) ? list : out.mis).push_back(d);
+        }
+    }
     const int64_t n = static_cast<int64_t>(list.size());
     std::vector<int32_t> npc(static_cast<size_t>(n));  // pieces of a small tile, 0 for the others
     parallel_for(n, 1 << 15, [&](int64_t a, int64_t b) {

@@ -74,11 +74,13 @@ template <typename F> void parallel_for(int64_t n, int64_t grain, F &&f) {
     for (std::thread &w : workers) w.join();
 }
 
-// A tile list split for the two remap kernels: full-size tiles for the tile
-// kernel, and the one-pass pieces of the small tiles with their groups for
-// the small-tile kernel.
+// A tile list split between the remap kernels: aligned and misaligned
+// full-size tiles for the two instances of the tile kernel, and the one-pass
+// pieces of the small tiles with their groups for the small-tile kernel.
 struct SplitList {
-    std::vector<TileDesc> big, pieces;
+    std::vector<TileDesc> big;  // aligned ("fast") full-size tiles
+    std::vector<TileDesc> mis;  // misaligned tiles (one element per lane)
+    std::vector<TileDesc> pieces;
     std::vector<uint32_t> groups;  // group g = pieces [groups[g], groups[g + 1])
     int64_t ngroups() const { return groups.empty() ? 0 : static_cast<int64_t>(groups.size()) - 1; }
 };
