@@ -80,7 +80,11 @@ typedef enum { COSTA_MODE_DIRECT = 0, COSTA_MODE_MESSAGE = 1 } costa_mode;
  *          and write directly over the host link.  This is checked when a
  *          plan is built, before any kernel runs (COSTA_ERR_LAYOUT for
  *          pageable host memory, another device's memory or an address
- *          unknown to CUDA).
+ *          unknown to CUDA).  A source run (a column or row piece of a
+ *          block) that does not start or end on a 16-byte boundary may be
+ *          read in whole aligned 16-byte chunks: up to 15 bytes before and
+ *          after it, in the same aligned chunks (so on the same page), are
+ *          read and not used.  Nothing outside A's blocks is written.
  *  ld    - leading dimension in elements: the distance between consecutive
  *          columns (column-major) or rows (row-major); ld >= rows
  *          (column-major) or ld >= cols (row-major); ld < 2^31.

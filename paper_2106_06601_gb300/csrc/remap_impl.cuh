@@ -470,16 +470,160 @@ __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsi
     }
 }
 
-// ---- misaligned tiles: the same pipeline, one element per lane ----
+// ---- misaligned tiles ----
 //
 // A tile whose runs do not start on 16-byte boundaries (an odd leading
-// dimension, a block at an odd offset) cannot use 16-byte chunks.  It takes
-// the same steps with one element per lane: cp.async of single elements into
-// shared memory, A's elements loaded into registers before the wait, and
-// element-wide, still coalesced, stores.  Staged rows are TS elements wide;
-// element c of row r lives at position c ^ (r mod TS), so that lanes reading
-// one position across consecutive rows (the transposed read) hit distinct
-// banks.
+// dimension, a block at an odd offset) or whose extents are not whole chunks
+// takes one of two paths, by combine kind (measured on GB300: each is the
+// faster one for its kinds).
+//  - Kinds that do not read A move 16-byte chunks over each run's window
+//    (the aligned chunks that cover the run), like an aligned tile.
+//  - Kinds that read A move one element per lane.
+// Both stage into the TS x CPR swizzled slots of an aligned tile's buffer
+// plus one extra column of TS chunks.
+
+// ---- 16-byte windows (kinds that do not read A) ----
+//
+// A run of len elements at phase ph (its start address mod 16, in elements)
+// has ceil((ph + len) / VEC) window chunks, at most CPR + 1.
+//  - Source: every window chunk is copied whole.  The bytes beyond the run
+//    lie in the same aligned 16-byte chunk as bytes of the run (so on the
+//    same page of the same allocation) and are only read, never used.
+//  - A: a window chunk wholly inside the run is stored with one 16-byte
+//    access; a chunk that the run covers in part (the first and the last of a
+//    run) is stored element by element, so nothing outside the tile is
+//    written.
+// The staged run keeps its phase: element c of source run r sits at window
+// position ph_r + c.  Window chunk k < CPR lives in slot k of staged row r;
+// chunk CPR in the extra column.
+//
+// Lanes take the window chunks k < CPR with the aligned tile's lane map, and
+// chunk CPR of every run in one more pass.  A lane's runs are a multiple of
+// VEC apart (runs per pass = 32 / lanes per run >= 32 / CPR = VEC, both
+// powers of two), so they share their phase: the lane's chunk covers the same
+// tile columns in all its passes and, transposed, reads the same staged rows.
+
+template <typename T> struct WCfg {
+    static constexpr int XCOL = Cfg<T>::TS * Cfg<T>::CPR * 16;  // byte offset of the extra column
+    static constexpr int BUF_BYTES = (XCOL + Cfg<T>::TS * 16 + 127) / 128 * 128;
+};
+
+// Staged element at window position q of run r.
+template <typename T>
+__device__ __forceinline__ const T &welem(unsigned char *buf, int r, int q) {
+    using C = Cfg<T>;
+    const int j = q / C::VEC;
+    const unsigned char *c = j < C::CPR ? slot<T>(buf, r, j) : buf + WCfg<T>::XCOL + r * 16;
+    return reinterpret_cast<const T *>(c)[q % C::VEC];
+}
+
+// Phase (start address mod 16, in elements) of run r of a surface whose run
+// 0 starts at p and whose runs are ld elements apart.
+template <typename T>
+__device__ __forceinline__ int phase(const T *p, int64_t ld, int r) {
+    constexpr int V = Cfg<T>::VEC;
+    const int p0 = static_cast<int>((reinterpret_cast<uintptr_t>(p) & 15u) / sizeof(T));
+    return (p0 + r * static_cast<int>(ld & (V - 1))) & (V - 1);
+}
+
+// Window chunks per run of len elements (the most any phase needs), and
+// those of them below CPR.
+template <typename T> __device__ __forceinline__ int wchunks(int len) {
+    return (len + 2 * Cfg<T>::VEC - 2) / Cfg<T>::VEC;
+}
+template <typename T> __device__ __forceinline__ int wmain(int len) { return min(Cfg<T>::CPR, wchunks<T>(len)); }
+
+template <typename T>
+__device__ __forceinline__ void stage_issue_w(const Geom<T> &g, unsigned char *buf, int lane) {
+    using C = Cfg<T>;
+    const int runs = g.transpose ? g.nx : g.ny;
+    const int len = g.transpose ? g.ny : g.nx;  // elements per run
+    const int cm = wmain<T>(len);
+    const LaneMap m = lane_map(cm, lane);
+    const int ph = phase<T>(g.src, g.sld, m.r0);  // the phase of all this lane's runs
+    if (m.c < cm && m.c * C::VEC < ph + len) {
+        const T *s0 = g.src - ph + m.c * C::VEC;
+#pragma unroll 4
+        for (int r = m.r0; r < runs; r += m.rpp)
+            cp_async16(slot<T>(buf, r, m.c), s0 + static_cast<int64_t>(r) * g.sld);
+    }
+    if (wchunks<T>(len) > C::CPR && lane < runs) {  // chunk CPR: lane = run
+        const int pr = phase<T>(g.src, g.sld, lane);
+        if (C::CPR * C::VEC < pr + len)
+            cp_async16(buf + WCfg<T>::XCOL + lane * 16,
+                       g.src + static_cast<int64_t>(lane) * g.sld - pr + C::CPR * C::VEC);
+    }
+}
+
+// The staged elements of tile columns x0 .. x0 + VEC - 1 of tile row y
+// (columns outside [0, nx) read an in-tile element; they are not stored).
+template <typename T>
+__device__ __forceinline__ Chunk<T> staged_window(const Geom<T> &g, unsigned char *buf, int x0, int y) {
+    using C = Cfg<T>;
+    Chunk<T> b;
+    if (g.transpose) {
+#pragma unroll
+        for (int i = 0; i < C::VEC; ++i) {
+            const int x = min(max(x0 + i, 0), g.nx - 1);  // source run x, position y
+            b.e[i] = welem<T>(buf, x, phase<T>(g.src, g.sld, x) + y);
+        }
+    } else {
+        const int ph = phase<T>(g.src, g.sld, y);  // source run y, positions x
+#pragma unroll
+        for (int i = 0; i < C::VEC; ++i) b.e[i] = welem<T>(buf, y, ph + min(max(x0 + i, 0), g.nx - 1));
+    }
+    return b;
+}
+
+// Writes the tile columns of x0 .. x0 + VEC - 1 (a window chunk of tile row
+// y) that lie in [0, nx): with one 16-byte store when all do (FULL).
+template <typename T, int KIND, bool FULL>
+__device__ __forceinline__ void drain_window(const Geom<T> &g, const Sc &s, unsigned char *buf, int x0, int y) {
+    using C = Cfg<T>;
+    const Chunk<T> b = staged_window<T>(g, buf, x0, y);
+    Chunk<T> o;
+#pragma unroll
+    for (int i = 0; i < C::VEC; ++i) o.e[i] = combine<KIND>(b.e[i], T(), s);
+    T *row = g.dst + static_cast<int64_t>(y) * g.dld;
+    if constexpr (FULL) {
+        store(row + x0, o);
+    } else {
+#pragma unroll
+        for (int i = 0; i < C::VEC; ++i)
+            if (x0 + i >= 0 && x0 + i < g.nx) row[x0 + i] = o.e[i];
+    }
+}
+
+// Full window chunks go out in the lane-map passes, with 16-byte stores
+// only; the partial ones (a run's first chunk when its phase is not 0, its
+// last when the run does not fill it) in one more pass, lane = tile row.
+template <typename T, int KIND>
+__device__ __forceinline__ void stage_drain_w(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
+    using C = Cfg<T>;
+    static_assert(KIND == K_COPY || KIND == K_SCALE, "the window path does not read A");
+    const int cm = wmain<T>(g.nx);
+    const LaneMap m = lane_map(cm, lane);
+    const int x0 = m.c * C::VEC - phase<T>(g.dst, g.dld, m.r0);  // first tile column of the lane's chunk
+    if (m.c < cm && x0 >= 0 && x0 + C::VEC <= g.nx) {
+#pragma unroll 4
+        for (int y = m.r0; y < g.ny; y += m.rpp) drain_window<T, KIND, true>(g, s, buf, x0, y);
+    }
+    if (lane < g.ny) {
+        const int ph = phase<T>(g.dst, g.dld, lane);
+        const int last = (ph + g.nx - 1) / C::VEC;  // last window chunk of the row
+        const int xl = last * C::VEC - ph;
+        if (ph > 0) drain_window<T, KIND, false>(g, s, buf, -ph, lane);
+        if (xl + C::VEC > g.nx && (last > 0 || ph == 0)) drain_window<T, KIND, false>(g, s, buf, xl, lane);
+    }
+}
+
+// ---- one element per lane (kinds that read A) ----
+//
+// cp.async of single elements into shared memory, A's elements loaded into
+// registers before the wait, and element-wide, still coalesced, stores.
+// Staged rows are TS elements wide; element c of row r lives at position
+// c ^ (r mod TS), so that lanes reading one position across consecutive rows
+// (the transposed read) hit distinct banks.
 
 template <typename T>
 __device__ __forceinline__ T *slot_e(unsigned char *buf, int r, int c) {
@@ -812,9 +956,10 @@ __global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB
 
 // Stages a tile's source: 16-byte chunks, or single elements in the kernel
 // for misaligned tiles (MIS).
-template <typename T, bool MIS>
+template <typename T, int KIND, bool MIS>
 __device__ __forceinline__ void stage_any(const Geom<T> &g, unsigned char *buf, int lane) {
-    if constexpr (MIS) stage_issue_e<T>(g, buf, lane);
+    if constexpr (MIS && KCfg<T, KIND>::READS_A) stage_issue_e<T>(g, buf, lane);
+    else if constexpr (MIS) stage_issue_w<T>(g, buf, lane);
     else if (g.fast) stage_issue<T>(g, buf, lane);  // the element-wise fallback stages nothing
 }
 
@@ -829,12 +974,16 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
         cached = g.prob;
     }
     s.conj_mask = g.conj ? 0x80000000u : 0u;
-    if constexpr (MIS) {
+    if constexpr (MIS && KCfg<T, KIND>::READS_A) {
         Chunk<T> av[C::NPASS];
         load_a_e<T, KIND>(g, s, av, lane);
         cp_async_wait<NB - 1>();  // this tile's copies (later tiles' may still fly)
         __syncwarp();
         stage_drain_e<T, KIND>(g, s, buf, av, lane);
+    } else if constexpr (MIS) {
+        cp_async_wait<NB - 1>();
+        __syncwarp();
+        stage_drain_w<T, KIND>(g, s, buf, lane);
     } else if (g.fast) {
         Chunk<T> av[C::NPASS];
         load_a<T, KIND>(g, s, av, lane);
@@ -857,9 +1006,10 @@ __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB
     remap_kernel(const RemapLaunch args) {
     using C = Cfg<T>;
     constexpr int NB = KCfg<T, KIND>::NBUF;
+    constexpr int BB = MIS ? WCfg<T>::BUF_BYTES : C::BUF_BYTES;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    unsigned char *bufs = smem_raw + warp * NB * C::BUF_BYTES;
+    unsigned char *bufs = smem_raw + warp * NB * BB;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * C::WARPS;
     const int64_t first = static_cast<int64_t>(blockIdx.x) * C::WARPS + warp;
 
@@ -876,7 +1026,7 @@ __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB
     if constexpr (NB == 1) {  // no look-ahead: copy, wait, write, one tile at a time
         Geom<T> g;
         while (next_tile<T, KIND, MIS>(args, first, stride, ts, g, lane)) {
-            stage_any<T, MIS>(g, bufs, lane);
+            stage_any<T, KIND, MIS>(g, bufs, lane);
             cp_async_commit();
             write_tile<T, KIND, 1, MIS>(args, g, s, cached, bufs, lane);
         }
@@ -887,7 +1037,7 @@ __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB
 #pragma unroll
     for (int k = 0; k < NB - 1; ++k) {
         have[k] = (k == 0 || have[k - 1]) && next_tile<T, KIND, MIS>(args, first, stride, ts, ring[k], lane);
-        if (have[k]) stage_any<T, MIS>(ring[k], bufs + k * C::BUF_BYTES, lane);
+        if (have[k]) stage_any<T, KIND, MIS>(ring[k], bufs + k * BB, lane);
         cp_async_commit();
     }
     int cur = 0;
@@ -896,9 +1046,9 @@ __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB
         have[LA] = have[LA - 1] && next_tile<T, KIND, MIS>(args, first, stride, ts, ring[LA], lane);
         int ahead = cur + NB - 1;
         if (ahead >= NB) ahead -= NB;
-        if (have[LA]) stage_any<T, MIS>(ring[LA], bufs + ahead * C::BUF_BYTES, lane);
+        if (have[LA]) stage_any<T, KIND, MIS>(ring[LA], bufs + ahead * BB, lane);
         cp_async_commit();
-        write_tile<T, KIND, NB, MIS>(args, ring[0], s, cached, bufs + cur * C::BUF_BYTES, lane);
+        write_tile<T, KIND, NB, MIS>(args, ring[0], s, cached, bufs + cur * BB, lane);
 #pragma unroll
         for (int k = 0; k < LA; ++k) {
             ring[k] = ring[k + 1];
@@ -924,7 +1074,8 @@ template <typename T, int KIND, bool MIS>
 cudaError_t launch_tiles(const RemapLaunch &a, cudaStream_t st) {
     auto kern = remap_kernel<T, KIND, MIS>;
     constexpr int kWarps = Cfg<T>::WARPS;
-    const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND>::NBUF * Cfg<T>::BUF_BYTES;
+    const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND>::NBUF *
+                        (MIS ? WCfg<T>::BUF_BYTES : Cfg<T>::BUF_BYTES);
     static int per_sm = 0;
     if (per_sm == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -972,8 +1123,12 @@ cudaError_t launch_small(const RemapLaunch &a, cudaStream_t st) {
 // (each launched only when it has work).
 template <typename T, int KIND>
 cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
+    // 16-byte elements sit at 16-byte aligned addresses, so every tile of
+    // theirs is aligned and their misaligned instance is not built
+    if (sizeof(T) == 16 && a.nmtiles > 0) return cudaErrorInvalidValue;
     cudaError_t e = a.ntiles > 0 ? launch_tiles<T, KIND, false>(a, st) : cudaSuccess;
-    if (e == cudaSuccess && a.nmtiles > 0) e = launch_tiles<T, KIND, true>(a, st);
+    if constexpr (sizeof(T) != 16)
+        if (e == cudaSuccess && a.nmtiles > 0) e = launch_tiles<T, KIND, true>(a, st);
     if (e == cudaSuccess && a.ngroups > 0) e = launch_small<T, KIND>(a, st);
     return e;
 }

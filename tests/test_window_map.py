@@ -1,0 +1,124 @@
+"""CPU check of the index arithmetic of the misaligned-tile window path
+(`stage_issue_w`, `stage_drain_w` in the remap kernel source), replayed per
+lane for random tiles before any kernel runs it.
+
+For a tile of nx x ny elements (nx, ny <= 32), transposed or not, with any
+element-aligned start addresses and leading dimensions of source and target,
+the replay checks that:
+  - every 16-byte source copy is aligned and lies inside the aligned window
+    of its run, [floor16(run start), ceil16(run end));
+  - every shared-memory access stays inside the warp's buffer;
+  - every 16-byte store to A is aligned;
+  - every target element of the tile is written exactly once, with the staged
+    value of its own source element, and nothing outside the tile is written.
+The arithmetic below restates the kernel's (lane map, phases, window chunks,
+swizzled slots, extra column); a change there must be mirrored here."""
+import random
+
+import pytest
+
+TS = 32
+
+
+def lane_map(chunks, lane):
+    sh = 0 if chunks <= 1 else (chunks - 1).bit_length()
+    return lane & ((1 << sh) - 1), lane >> sh, 32 >> sh
+
+
+def replay(es, rnd):
+    vec = 16 // es
+    cpr = TS // vec
+    xcol = TS * cpr * 16
+    buf_bytes = (xcol + TS * 16 + 127) // 128 * 128
+
+    def slot(r, c):
+        assert 0 <= c < cpr and 0 <= r < TS
+        return (r * cpr + (c ^ ((r // vec) & 7))) * 16
+
+    def welem(r, q):
+        j = q // vec
+        return (slot(r, j) if j < cpr else xcol + r * 16) + (q % vec) * es
+
+    def phase(p, ld, r):
+        return ((p & 15) // es + r * (ld & (vec - 1))) & (vec - 1)
+
+    def wchunks(n):
+        return (n + 2 * vec - 2) // vec
+
+    def wmain(n):
+        return min(cpr, wchunks(n))
+
+    nx = TS if rnd.random() < 0.3 else rnd.randint(1, TS)
+    ny = TS if rnd.random() < 0.3 else rnd.randint(1, TS)
+    tr = rnd.random() < 0.5
+    runs, ln = (nx, ny) if tr else (ny, nx)
+    sld = ln + rnd.randint(0, 9)
+    dld = nx + rnd.randint(0, 9)
+    src = (1 << 20) + rnd.randrange(64) * es
+    dst = (1 << 24) + rnd.randrange(64) * es
+    smem = {}
+
+    def copy16(sa, ga, r):
+        assert ga % 16 == 0 and sa % 16 == 0 and 0 <= sa and sa + 16 <= buf_bytes
+        start, end = src + r * sld * es, src + (r * sld + ln) * es
+        assert start // 16 * 16 <= ga and ga + 16 <= -(-end // 16) * 16
+        for b in range(vec):
+            smem[sa + b * es] = ga + b * es
+
+    # stage_issue_w
+    cm = wmain(ln)
+    for lane in range(32):
+        c, r0, rpp = lane_map(cm, lane)
+        assert rpp % vec == 0
+        ph = phase(src, sld, r0)
+        if c < cm and c * vec < ph + ln:
+            for r in range(r0, runs, rpp):
+                assert phase(src, sld, r) == ph
+                copy16(slot(r, c), src + (r * sld - ph + c * vec) * es, r)
+        if wchunks(ln) > cpr and lane < runs:
+            pr = phase(src, sld, lane)
+            if cpr * vec < pr + ln:
+                copy16(xcol + lane * 16, src + (lane * sld - pr + cpr * vec) * es, lane)
+
+    written = set()
+
+    def drain(x0, y, full):
+        for i in range(vec):
+            x = min(max(x0 + i, 0), nx - 1)
+            if tr:
+                sa, want = welem(x, phase(src, sld, x) + y), src + (x * sld + y) * es
+            else:
+                sa, want = welem(y, phase(src, sld, y) + x), src + (y * sld + x) * es
+            assert 0 <= sa < buf_bytes and smem.get(sa) == want
+        if full:
+            assert (dst + (y * dld + x0) * es) % 16 == 0 and 0 <= x0 and x0 + vec <= nx
+        for i in range(vec):
+            if 0 <= x0 + i < nx:
+                assert (y, x0 + i) not in written
+                written.add((y, x0 + i))
+
+    # stage_drain_w
+    cmd = wmain(nx)
+    for lane in range(32):
+        c, r0, rpp = lane_map(cmd, lane)
+        x0 = c * vec - phase(dst, dld, r0)
+        if c < cmd and x0 >= 0 and x0 + vec <= nx:
+            for y in range(r0, ny, rpp):
+                assert c * vec - phase(dst, dld, y) == x0
+                drain(x0, y, True)
+        if lane < ny:
+            ph = phase(dst, dld, lane)
+            last = (ph + nx - 1) // vec
+            xl = last * vec - ph
+            if ph > 0:
+                drain(-ph, lane, False)
+            if xl + vec > nx and (last > 0 or ph == 0):
+                drain(xl, lane, False)
+    assert written == {(y, x) for y in range(ny) for x in range(nx)}
+
+
+@pytest.mark.parametrize("es", [4, 8])
+def test_window_map(es):
+    rnd = random.Random(2106066010 + es)
+    for _ in range(8000):
+        replay(es, rnd)
