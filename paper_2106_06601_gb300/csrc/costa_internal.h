@@ -117,7 +117,7 @@ COSTA_HD inline int kind_of(int32_t flags) {
 struct RemapLaunch {
     const TileDesc *tiles;       // aligned full-size tiles (the tile kernel)
     int64_t ntiles;
-    const TileDesc *mtiles;      // misaligned tiles (the tile kernel, one element per lane)
+    const TileDesc *mtiles;      // misaligned tiles (the tile kernel's second instance)
     int64_t nmtiles;
     const TileDesc *pieces;      // one-pass pieces of small tiles (the small-tile kernel)
     const uint32_t *groups;      // group g = pieces [groups[g], groups[g + 1])

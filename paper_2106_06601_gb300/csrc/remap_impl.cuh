@@ -22,7 +22,9 @@
 // If A and the source share their contiguous axis the staged rows are read
 // straight; otherwise they are read across rows (the transpose of Sec. 6's
 // "cache-friendly ... kernel for matrix transposition").  Tiles whose runs
-// are not 16-byte aligned take the same pipeline one element per lane.
+// are not 16-byte aligned take the same pipeline in a second instance of the
+// kernel: over aligned 16-byte windows of their runs, or one element per
+// lane for the kinds that read A.
 //
 // The kernel walks a list of tile descriptors (TileDesc) resolved on the host:
 // the direct list (every tile: B -> A), or the message path of Alg. 3 /
@@ -954,8 +956,9 @@ __global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB
     }
 }
 
-// Stages a tile's source: 16-byte chunks, or single elements in the kernel
-// for misaligned tiles (MIS).
+// Stages a tile's source: 16-byte chunks; in the instance for misaligned
+// tiles (MIS), the runs' 16-byte windows or, for kinds that read A, single
+// elements.
 template <typename T, int KIND, bool MIS>
 __device__ __forceinline__ void stage_any(const Geom<T> &g, unsigned char *buf, int lane) {
     if constexpr (MIS && KCfg<T, KIND>::READS_A) stage_issue_e<T>(g, buf, lane);
@@ -998,9 +1001,9 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
 
 // The tile kernel.  MIS = false moves the aligned ("fast") tiles of
 // args.tiles with 16-byte chunks; MIS = true moves the misaligned tiles of
-// args.mtiles one element per lane.  The host puts every tile in the right
-// list; a tile of the other kind is skipped, so no 16-byte access is ever
-// made at a misaligned address.
+// args.mtiles (see "misaligned tiles" above).  The host puts every tile in
+// the right list, so no 16-byte access is ever made at a misaligned
+// address.
 template <typename T, int KIND, bool MIS>
 __global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB)
     remap_kernel(const RemapLaunch args) {

@@ -79,7 +79,7 @@ template <typename F> void parallel_for(int64_t n, int64_t grain, F &&f) {
 // pieces of the small tiles with their groups for the small-tile kernel.
 struct SplitList {
     std::vector<TileDesc> big;  // aligned ("fast") full-size tiles
-    std::vector<TileDesc> mis;  // misaligned tiles (one element per lane)
+    std::vector<TileDesc> mis;  // misaligned tiles (16-byte windows or single elements)
     std::vector<TileDesc> pieces;
     std::vector<uint32_t> groups;  // group g = pieces [groups[g], groups[g + 1])
     int64_t ngroups() const { return groups.empty() ? 0 : static_cast<int64_t>(groups.size()) - 1; }
