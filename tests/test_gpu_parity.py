@@ -302,3 +302,21 @@ def test_transform_replays_in_cuda_graph(dev):
             assert np.all(ok)
     finally:
         g.close()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64", "c64"])
+@pytest.mark.parametrize("op", ["N", "T", "C"])
+def test_misaligned_runs(dtype, op, dev):
+    """Runs off 16-byte boundaries: odd leading dimensions, odd block sizes
+    and buffers at odd element offsets (guards).  Copy and scale take the
+    16-byte window path, the kinds that read A the element path; both must
+    write every element of A once and nothing outside A's blocks."""
+    m, n = 150, 171
+    am, an = (m, n) if op == "N" else (n, m)
+    for k, (pad_b, pad_a, guard) in enumerate(((1, 0, 0), (0, 3, 0), (2, 1, 3), (3, 2, 1))):
+        B = L.block_cyclic(m, n, 13 + 2 * k, 37, 2, 3, storage="RC"[k % 2], ld_pad=pad_b)
+        A = L.block_cyclic(am, an, 29, 7 + 4 * k, 3, 2, storage="CR"[k % 2], ld_pad=pad_a)
+        for alpha, beta in ((1.0, 0.0), (2.0, 0.0), (2.0, 0.5), (-0.3, 0.7)):
+            p = C.Problem("misaligned", dtype, op, alpha, beta, A, B, "uniform",
+                          "nan" if beta == 0 else "uniform", C.SEED0 + 11 + k)
+            check_problem(p, dev, guard=guard)
