@@ -58,12 +58,12 @@ typedef enum { COSTA_F32 = 0, COSTA_F64 = 1, COSTA_C64 = 2, COSTA_C128 = 3 } cos
 /* op(B): identity, transpose, conjugate transpose (on real types C == T). */
 typedef enum { COSTA_OP_N = 0, COSTA_OP_T = 1, COSTA_OP_C = 2 } costa_op;
 
-/* Element order inside one block (Sec. 6: "row- or col-major ordering"). */
+/* Element order inside one block (Sec. 6: each block is row- or column-major). */
 typedef enum { COSTA_COL_MAJOR = 0, COSTA_ROW_MAJOR = 1 } costa_order;
 
 /* How the data moves on the device:
  *  DIRECT  - one fused kernel reads B's blocks and writes A's blocks
- *            (every pair is treated like the paper's "local blocks", Sec. 6);
+ *            (every pair is treated like a block that stays on its rank, Sec. 6);
  *  MESSAGE - the paper's data flow (Alg. 3, Sec. 6): packages for remote
  *            (source, relabeled target) pairs are packed into one staging
  *            buffer at the exclusive-scan offsets of V, then unpacked and

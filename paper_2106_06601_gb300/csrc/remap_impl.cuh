@@ -20,8 +20,8 @@
 //      alpha and beta as one fma per element on the way out (Sec. 5:
 //      transform after receive).
 // If A and the source share their contiguous axis the staged rows are read
-// straight; otherwise they are read across rows (the transpose of Sec. 6's
-// "cache-friendly ... kernel for matrix transposition").  Tiles whose runs
+// straight; otherwise they are read across rows (the transposing kernel of
+// Sec. 6).  Tiles whose runs
 // are not 16-byte aligned take the same pipeline in a second instance of the
 // kernel: over aligned 16-byte windows of their runs, or one element per
 // lane for the kinds that read A.
