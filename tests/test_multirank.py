@@ -1,6 +1,7 @@
 """The bench's multi-GPU aggregation (one independent replica per rank,
 barrier, max-over-ranks time, whole-job throughput), run as world_size-2
-gloo process groups on the CPU."""
+gloo process groups on the CPU; and the source hash that keys its recorded
+DRAM traffic."""
 import os
 import socket
 
@@ -52,3 +53,13 @@ def test_single_process_identity():
     import bench
     assert bench.max_over_ranks(3.5) == 3.5
     assert bench.job_throughput(10**9, 1, 1, 1000.0) == 1.0
+
+
+def test_kernel_hash_ignores_comments_only():
+    import bench
+    src = 'int f(int x) { // add one\n  return x + 1; /* not "this" */\n}\nconst char *s = "a // b";\n'
+    same = '// header\nint f(int x) {\n\n  return x + 1;\n}\nconst char *s = "a // b";  // kept\n'
+    other = 'int f(int x) { return x + 2; }\nconst char *s = "a // b";\n'
+    assert bench.code_only(src) == bench.code_only(same)
+    assert bench.code_only(src) != bench.code_only(other)
+    assert '"a // b"' in bench.code_only(src)
