@@ -157,6 +157,7 @@ struct VolumeLaunch {
 #define COSTA_TS_4 32
 #endif
 COSTA_HD constexpr int tile_extent(int esize) { return esize == 16 ? COSTA_TS_16 : esize == 4 ? COSTA_TS_4 : 32; }
+static_assert(tile_extent(4) <= 32 && tile_extent(16) <= 32, "the kernels' lane maps need tiles of at most 32");
 
 // Small tiles are cut by the host into pieces of at most piece_x x piece_y
 // elements, each exactly one warp pass (32 lanes x 16 bytes at most), and

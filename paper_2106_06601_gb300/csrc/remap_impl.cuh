@@ -108,6 +108,12 @@ template <typename T> struct Cfg {
     static constexpr int BUF_BYTES_RAW = TS * PITCH * static_cast<int>(sizeof(T));
     static constexpr int BUF_BYTES = (BUF_BYTES_RAW + 127) / 128 * 128;
     static constexpr int WARPS = sizeof(T) == 4 ? COSTA_WARPS_4 : sizeof(T) == 16 ? COSTA_WARPS_16 : COSTA_WARPS_8;
+    // Lane maps give a run at most 32 lanes: a run's chunks (aligned path),
+    // its elements (misaligned path of the kinds that read A) and one lane
+    // per run or row (the window path's last pass) must each fit in a warp.
+    // A larger tile extent would leave runs per pass at 0, and the copy
+    // loops would never advance.
+    static_assert(TS >= 1 && TS <= 32 && TS % VEC == 0, "tile extent must be a multiple of VEC in [VEC, 32]");
 };
 
 // Launch shape per element type and combine kind (measured on GB300): warps
