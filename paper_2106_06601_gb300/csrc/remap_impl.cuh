@@ -62,6 +62,12 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_NBUF_4
 #define COSTA_NBUF_4 2
 #endif
+#ifndef COSTA_MINB_4A
+#define COSTA_MINB_4A 3
+#endif
+#ifndef COSTA_NBUF_4A
+#define COSTA_NBUF_4A 1
+#endif
 #ifndef COSTA_WARPS_8
 #define COSTA_WARPS_8 4
 #endif
@@ -122,17 +128,18 @@ template <typename T> struct Cfg {
 // flight ahead of the tile it writes).  8-byte types with the light kinds
 // run more warps without look-ahead; the general kinds (non-power-of-two
 // beta, complex scalars) need the registers of 3 blocks and use a 2-deep
-// ring.  16-byte kinds that read A hold a whole 16 KB tile of A in
-// registers; they run two blocks without look-ahead.  Overridable at build
-// time for tuning.
+// ring.  4-byte kinds that read A run 3 blocks without look-ahead, those
+// that do not 2 blocks with a 2-deep ring.  16-byte kinds that read A hold
+// a whole 16 KB tile of A in registers; they run two blocks without
+// look-ahead.  Overridable at build time for tuning.
 template <typename T, int KIND> struct KCfg {
     static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX;
     static constexpr bool READS_A = KIND != K_COPY && KIND != K_SCALE;
     static constexpr int WARPS = Cfg<T>::WARPS;
-    static constexpr int MINB = sizeof(T) == 4 ? COSTA_MINB_4
+    static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : COSTA_MINB_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
                               : HEAVY ? COSTA_MINB_8H : COSTA_MINB_8;
-    static constexpr int NBUF = sizeof(T) == 4 ? COSTA_NBUF_4
+    static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : COSTA_NBUF_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
                               : HEAVY ? COSTA_NBUF_8H : COSTA_NBUF_8;
 };
