@@ -122,8 +122,10 @@ def _i32(a) -> np.ndarray:
     return np.ascontiguousarray(a, dtype=np.int32)
 
 
-def _p(a: np.ndarray):
-    return a.ctypes.data_as(ctypes.c_void_p)
+def _p(a: np.ndarray) -> int:
+    """Address of an array's data, for a void* argument (the caller keeps the
+    array alive across the call)."""
+    return a.ctypes.data
 
 
 class Layout:
@@ -132,6 +134,7 @@ class Layout:
     def __init__(self, handle: int, dtype: str):
         self.handle = ctypes.c_void_p(handle)
         self.dtype = dtype
+        self.nranks = self.info()[2]
 
     def info(self):
         m, n = ctypes.c_int64(), ctypes.c_int64()
@@ -334,14 +337,25 @@ def _scalars(dtype: str, values) -> np.ndarray:
     return np.ascontiguousarray(np.asarray(values, dtype=_SCALAR_NP[dtype]).reshape(-1))
 
 
+# One host scalar of each element type as a ctypes value (real, or re/im pair).
+_SCALAR_CT = {"f32": ctypes.c_float, "f64": ctypes.c_double,
+              "c64": ctypes.c_float * 2, "c128": ctypes.c_double * 2}
+
+
+def _scalar1(dtype: str, v):
+    if dtype in ("f32", "f64"):
+        return _SCALAR_CT[dtype](v)
+    v = complex(v)
+    return _SCALAR_CT[dtype](v.real, v.imag)
+
+
 def costa_transform(A: Layout, B: Layout, op: str, alpha, beta, relabel: bool = False,
                     stream: int = 0, mode: str = "direct") -> np.ndarray:
     """A = alpha * op(B) + beta * A, asynchronous on `stream`; returns sigma."""
-    _, _, P, _ = A.info()
-    sigma = np.zeros(P, dtype=np.int32)
-    al, be = _scalars(A.dtype, [alpha]), _scalars(A.dtype, [beta])
-    _check(_lib.costa_transform_ex(A.handle, B.handle, OPS[op], _p(al), _p(be), int(relabel),
-                                   _p(sigma), MODES[mode], ctypes.c_void_p(stream)))
+    sigma = np.zeros(A.nranks, dtype=np.int32)
+    al, be = _scalar1(A.dtype, alpha), _scalar1(A.dtype, beta)
+    _check(_lib.costa_transform_ex(A.handle, B.handle, OPS[op], ctypes.byref(al), ctypes.byref(be),
+                                   int(relabel), sigma.ctypes.data, MODES[mode], stream))
     return sigma
 
 
