@@ -25,6 +25,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -470,12 +471,31 @@ def roofline(args, r):
     return base
 
 
-def run_cpu_oracle(args, probs, seconds_target: float):
+def cpu_model() -> str:
+    """The host CPU's model name, as lscpu or /proc/cpuinfo report it."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return platform.machine()
+
+
+def run_cpu_oracle(args, probs, seconds_target: float, threads: int | None = None):
     """The oracle, as it stands, on a bounded row slab of the first instance
     (the same layouts and values); returns (GB/s, threads, description)."""
     import oracle
     p = probs[0]
-    threads = oracle.default_threads()
+    threads = threads or oracle.default_threads()
     Bh = HostMatrix(p.B, p.dtype).fill(p.b_kind, p.seed, p.src_stream)
     Ah = HostMatrix(p.A, p.dtype).fill(p.a_kind, p.seed, p.tgt_stream)
     per_row_bytes = p.A.n * p.esize * (3 if p.beta != 0 else 2)
@@ -570,7 +590,10 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         gbs, threads, desc, _, _ = run_cpu_oracle(args, probs, args.cpu_seconds)
         cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
-               "sample": desc}
+               "sample": desc, "cpu_model": cpu_model()}
+        if args.workload in ("c1", "c2"):  # the single-threaded figure as well
+            gbs1, _, desc1, _, _ = run_cpu_oracle(args, probs, min(3.0, args.cpu_seconds), threads=1)
+            cpu["single_thread"] = {"value": round(gbs1, 4), "unit": "GB/s", "sample": desc1}
     if rank == 0:
         st = r["stats"]
         out = {
