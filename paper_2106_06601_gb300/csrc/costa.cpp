@@ -124,6 +124,7 @@ struct Plan {
     std::vector<ProblemHost> probs;
     void *d_mem = nullptr;
     DevList direct;                     // the direct list
+    DevList direct_halves;              // the same with its wide aligned tiles in x-halves (8-byte types)
     Scalars *d_scalars = nullptr;
     std::vector<Scalars> cached_scalars;
     int64_t total_tiles = 0, total_cells = 0;
@@ -419,6 +420,24 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     }
     const SplitList split = split_small(std::move(list), es);
     const SplitOffsets off_tiles = arena.add_split(split);
+    // 8-byte types: the aligned tiles also in x-halves of ts / 2, for the
+    // axpby kind with beta = +-2^k, in transposing problems whose A blocks are
+    // at most 256 elements along A's contiguous axis.  Measured on GB300:
+    // block-cyclic targets (blocks of 32 to 256) gain 2-8% on halves (8192^2
+    // f64 T, BC64 -> BC128: 6184 -> 6338 GB/s); targets of whole-panel blocks
+    // (1024 and 4096 rows) lose 2-6%, op = N gains nothing, and the other
+    // kinds lose on halves.
+    std::vector<char> halve(static_cast<size_t>(n), 0);
+    for (int k = 0; k < n; ++k) {
+        const costa_layout_s *a = plan->probs[k].A;
+        const bool rows_fast = a->blocks.empty() || a->blocks[0].order == COSTA_COL_MAJOR;
+        const std::vector<int64_t> &S = rows_fast ? a->R : a->C;
+        int64_t widest = 0;
+        for (size_t i = 0; i + 1 < S.size(); ++i) widest = std::max(widest, S[i + 1] - S[i]);
+        halve[k] = plan->probs[k].op != COSTA_OP_N && widest <= 256;
+    }
+    const std::vector<TileDesc> halves = es == 8 ? split_x_halves(split.big, ts / 2, es, halve) : std::vector<TileDesc>();
+    const size_t off_halves = halves.empty() ? 0 : arena.add_vec(halves);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
     std::vector<Scalars> sc(n);
@@ -454,6 +473,11 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     ce = cudaMemcpy(d, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(plan tables)");
     plan->direct = resolve(dbase, off_tiles, split);
+    plan->direct_halves = plan->direct;
+    if (!halves.empty()) {
+        plan->direct_halves.tiles = reinterpret_cast<const TileDesc *>(dbase + off_halves);
+        plan->direct_halves.ntiles = static_cast<int64_t>(halves.size());
+    }
     plan->d_scalars = reinterpret_cast<Scalars *>(dbase + off_sc);
     plan->total_tiles = tiles;
     plan->total_cells = cells;
@@ -741,7 +765,8 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     // one launch per combine kind present in the batch
     bool kinds[K_NKINDS] = {};
     for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
-    auto launch_list = [&](const DevList &list) -> cudaError_t {
+    // halves: the list for K_AXPBY2 (null: the same list)
+    auto launch_list = [&](const DevList &list, const DevList *halves) -> cudaError_t {
         RemapLaunch l = L;
         l.tiles = list.tiles;
         l.ntiles = list.ntiles;
@@ -752,7 +777,12 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         l.ngroups = list.ngroups;
         for (int kind = 0; kind < K_NKINDS; ++kind) {
             if (!kinds[kind]) continue;
-            cudaError_t e = launch_remap(l, kind, stream);
+            RemapLaunch lk = l;
+            if (kind == K_AXPBY2 && halves) {
+                lk.tiles = halves->tiles;
+                lk.ntiles = halves->ntiles;
+            }
+            cudaError_t e = launch_remap(lk, kind, stream);
             if (e != cudaSuccess) return e;
         }
         return cudaSuccess;
@@ -760,7 +790,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     cudaError_t ce;
     if (mode == COSTA_MODE_DIRECT) {
         ce = mark(0);
-        if (ce == cudaSuccess) ce = launch_list(plan->direct);
+        if (ce == cudaSuccess) ce = launch_list(plan->direct, &plan->direct_halves);
         if (ce == cudaSuccess) ce = mark(1);
         if (ce != cudaSuccess) return cuda_fail(ce, "remap kernel launch");
         if (timer) timer->nphases = 1;
@@ -788,10 +818,10 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     if (ce == cudaSuccess) ce = launch_remap(lp, K_COPY, stream);
     if (ce == cudaSuccess) ce = mark(1);
     if (ce != cudaSuccess) return cuda_fail(ce, "pack kernel launch");
-    ce = launch_list(m.local);
+    ce = launch_list(m.local, nullptr);
     if (ce == cudaSuccess) ce = mark(2);
     if (ce != cudaSuccess) return cuda_fail(ce, "local remap kernel launch");
-    ce = launch_list(m.unpack);
+    ce = launch_list(m.unpack, nullptr);
     if (ce == cudaSuccess) ce = mark(3);
     if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
     if (timer) timer->nphases = 3;

@@ -80,6 +80,9 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_MINB_8H
 #define COSTA_MINB_8H 3
 #endif
+#ifndef COSTA_MIS_MINB_8A
+#define COSTA_MIS_MINB_8A 4
+#endif
 #ifndef COSTA_NBUF_8H
 #define COSTA_NBUF_8H 2
 #endif
@@ -128,17 +131,20 @@ template <typename T> struct Cfg {
 // flight ahead of the tile it writes).  8-byte types with the light kinds
 // run more warps without look-ahead; the general kinds (non-power-of-two
 // beta, complex scalars) need the registers of 3 blocks and use a 2-deep
-// ring.  4-byte kinds that read A run 3 blocks without look-ahead, those
-// that do not 2 blocks with a 2-deep ring.  16-byte kinds that read A hold
+// ring; in the misaligned-tile instance the light kinds that read A (one
+// element per lane, a whole tile of A in registers) run 4 blocks, which
+// their registers fit without spills.  4-byte kinds that read A run 3
+// blocks without look-ahead, those that do not 2 blocks with a 2-deep ring.  16-byte kinds that read A hold
 // a whole 16 KB tile of A in registers; they run two blocks without
 // look-ahead.  Overridable at build time for tuning.
-template <typename T, int KIND> struct KCfg {
+template <typename T, int KIND, bool MIS = false> struct KCfg {
     static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX;
     static constexpr bool READS_A = KIND != K_COPY && KIND != K_SCALE;
     static constexpr int WARPS = Cfg<T>::WARPS;
     static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : COSTA_MINB_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
-                              : HEAVY ? COSTA_MINB_8H : COSTA_MINB_8;
+                              : HEAVY ? COSTA_MINB_8H
+                              : (MIS && READS_A) ? COSTA_MIS_MINB_8A : COSTA_MINB_8;
     static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : COSTA_NBUF_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
                               : HEAVY ? COSTA_NBUF_8H : COSTA_NBUF_8;
@@ -1018,10 +1024,10 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
 // the right list, so no 16-byte access is ever made at a misaligned
 // address.
 template <typename T, int KIND, bool MIS>
-__global__ void __launch_bounds__(KCfg<T, KIND>::WARPS * 32, KCfg<T, KIND>::MINB)
+__global__ void __launch_bounds__(KCfg<T, KIND, MIS>::WARPS * 32, KCfg<T, KIND, MIS>::MINB)
     remap_kernel(const RemapLaunch args) {
     using C = Cfg<T>;
-    constexpr int NB = KCfg<T, KIND>::NBUF;
+    constexpr int NB = KCfg<T, KIND, MIS>::NBUF;
     constexpr int BB = MIS ? WCfg<T>::BUF_BYTES : C::BUF_BYTES;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1090,7 +1096,7 @@ template <typename T, int KIND, bool MIS>
 cudaError_t launch_tiles(const RemapLaunch &a, cudaStream_t st) {
     auto kern = remap_kernel<T, KIND, MIS>;
     constexpr int kWarps = Cfg<T>::WARPS;
-    const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND>::NBUF *
+    const size_t smem = static_cast<size_t>(kWarps) * KCfg<T, KIND, MIS>::NBUF *
                         (MIS ? WCfg<T>::BUF_BYTES : Cfg<T>::BUF_BYTES);
     static int per_sm = 0;
     if (per_sm == 0) {

@@ -136,6 +136,32 @@ int cut_pieces(const TileDesc &d, int es, TileDesc *out) {
     return k;
 }
 
+std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, int es,
+                                     const std::vector<char> &halve) {
+    const int64_t n = static_cast<int64_t>(list.size());
+    auto cut = [&](const TileDesc &d) { return d.nx > hx && halve[d.prob]; };
+    std::vector<int64_t> pos(static_cast<size_t>(n) + 1, 0);
+    for (int64_t i = 0; i < n; ++i) pos[i + 1] = pos[i] + (cut(list[i]) ? 2 : 1);
+    std::vector<TileDesc> out;
+    if (pos[n] == n) return out;
+    out.resize(static_cast<size_t>(pos[n]));
+    parallel_for(n, 1 << 15, [&](int64_t a, int64_t b) {
+        for (int64_t i = a; i < b; ++i) {
+            const TileDesc &d = list[i];
+            TileDesc *o = &out[static_cast<size_t>(pos[i])];
+            o[0] = d;
+            if (!cut(d)) continue;
+            const bool tr = (d.flags & TF_TRANSPOSE) != 0;
+            o[0].nx = static_cast<uint16_t>(hx);
+            o[1] = d;
+            o[1].nx = static_cast<uint16_t>(d.nx - hx);
+            o[1].dst = d.dst + static_cast<uint64_t>(hx) * es;
+            o[1].src = d.src + static_cast<uint64_t>(tr ? static_cast<int64_t>(hx) * d.sld : hx) * es;
+        }
+    });
+    return out;
+}
+
 SplitList split_small(std::vector<TileDesc> &&all, int es) {
     SplitList out;
     // misaligned tiles go to their own instance of the tile kernel
