@@ -124,7 +124,7 @@ struct Plan {
     std::vector<ProblemHost> probs;
     void *d_mem = nullptr;
     DevList direct;                     // the direct list
-    DevList direct_halves;              // the same with its wide aligned tiles in x-halves (8-byte types)
+    DevList direct_halves;              // the same with its full aligned tiles in x-halves (4- and 8-byte types)
     Scalars *d_scalars = nullptr;
     std::vector<Scalars> cached_scalars;
     int64_t total_tiles = 0, total_cells = 0;
@@ -420,13 +420,18 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     }
     const SplitList split = split_small(std::move(list), es);
     const SplitOffsets off_tiles = arena.add_split(split);
-    // 8-byte types: the aligned tiles also in x-halves of ts / 2, for the
-    // axpby kind with beta = +-2^k, in transposing problems whose A blocks are
-    // at most 256 elements along A's contiguous axis.  Measured on GB300:
-    // block-cyclic targets (blocks of 32 to 256) gain 2-8% on halves (8192^2
-    // f64 T, BC64 -> BC128: 6184 -> 6338 GB/s); targets of whole-panel blocks
-    // (1024 and 4096 rows) lose 2-6%, op = N gains nothing, and the other
-    // kinds lose on halves.
+    // The aligned 32 x 32 tiles also as x-halves (two tiles of at most ts / 2
+    // along A's contiguous axis), for problems whose A blocks are at most 256
+    // elements along that axis: used by every f32 kind, and by the f64 / c64
+    // axpby kind with beta = +-2^k in transposing problems.  Measured on
+    // GB300, same box:
+    //  - f32, 8192^2, BC64 -> BC128: T copy 81 -> 89%, T beta=0.5 88 -> 91%,
+    //    N copy 84 -> 91% of copy; c4 6243 -> 6372 GB/s (its 32 x 16 tiles
+    //    stay whole: halving them cost c4 7%);
+    //  - f64 T, BC64 -> BC128, beta=0.5 (c2) 6184 -> 6338 GB/s; c64 T +8%;
+    //  - lost: the other 8-byte kinds (f64 T copy 91 -> 87%), c128, op = N
+    //    for 8-byte types, and targets of whole panels (1024- and 4096-row
+    //    blocks: 2-6%).
     std::vector<char> halve(static_cast<size_t>(n), 0);
     for (int k = 0; k < n; ++k) {
         const costa_layout_s *a = plan->probs[k].A;
@@ -434,9 +439,10 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
         const std::vector<int64_t> &S = rows_fast ? a->R : a->C;
         int64_t widest = 0;
         for (size_t i = 0; i + 1 < S.size(); ++i) widest = std::max(widest, S[i + 1] - S[i]);
-        halve[k] = plan->probs[k].op != COSTA_OP_N && widest <= 256;
+        halve[k] = widest <= 256 && (es == 4 || plan->probs[k].op != COSTA_OP_N);
     }
-    const std::vector<TileDesc> halves = es == 8 ? split_x_halves(split.big, ts / 2, es, halve) : std::vector<TileDesc>();
+    const std::vector<TileDesc> halves =
+        es <= 8 ? split_x_halves(split.big, ts / 2, es, halve) : std::vector<TileDesc>();
     const size_t off_halves = halves.empty() ? 0 : arena.add_vec(halves);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
@@ -765,7 +771,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     // one launch per combine kind present in the batch
     bool kinds[K_NKINDS] = {};
     for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
-    // halves: the list for K_AXPBY2 (null: the same list)
+    // halves: the list for the kinds that run on x-halves (null: none)
     auto launch_list = [&](const DevList &list, const DevList *halves) -> cudaError_t {
         RemapLaunch l = L;
         l.tiles = list.tiles;
@@ -778,7 +784,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         for (int kind = 0; kind < K_NKINDS; ++kind) {
             if (!kinds[kind]) continue;
             RemapLaunch lk = l;
-            if (kind == K_AXPBY2 && halves) {
+            if (halves && (plan->esize == 4 || kind == K_AXPBY2)) {
                 lk.tiles = halves->tiles;
                 lk.ntiles = halves->ntiles;
             }

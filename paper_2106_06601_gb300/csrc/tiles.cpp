@@ -139,7 +139,7 @@ int cut_pieces(const TileDesc &d, int es, TileDesc *out) {
 std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, int es,
                                      const std::vector<char> &halve) {
     const int64_t n = static_cast<int64_t>(list.size());
-    auto cut = [&](const TileDesc &d) { return d.nx > hx && halve[d.prob]; };
+    auto cut = [&](const TileDesc &d) { return d.nx > hx && d.ny >= 2 * hx && halve[d.prob]; };
     std::vector<int64_t> pos(static_cast<size_t>(n) + 1, 0);
     for (int64_t i = 0; i < n; ++i) pos[i + 1] = pos[i] + (cut(list[i]) ? 2 : 1);
     std::vector<TileDesc> out;

@@ -117,9 +117,10 @@ int cut_pieces(const TileDesc &d, int es, TileDesc *out);
 SplitList split_small(std::vector<TileDesc> &&list, int es);
 
 // The aligned tiles of problems k with halve[k] that are wider than hx
-// along x (A's contiguous axis), cut into [0, hx) and the rest, in list
-// order (the two halves of a tile adjacent); empty when no tile is cut.
-// hx * es must be a multiple of 16, so both halves stay 16-byte aligned.
+// along x (A's contiguous axis) and at least 2 hx high, cut into [0, hx)
+// and the rest along x, in list order (the two halves of a tile adjacent);
+// empty when no tile is cut.  hx * es must be a multiple of 16, so both
+// halves stay 16-byte aligned.
 std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, int es,
                                      const std::vector<char> &halve);
 
