@@ -368,7 +368,7 @@ costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void
  * 16-byte elements, x along A's contiguous axis), which the small-tile
  * kernel moves in groups of up to a full tile's passes; the other tiles stay
  * with the tile kernel (those whose runs are not 16-byte aligned after the
- * others, for its one-element-per-lane instance).  Writes up to cap_tiles full-size tiles to `tiles`
+ * others, for its instance for misaligned tiles).  Writes up to cap_tiles full-size tiles to `tiles`
  * and up to cap_pieces pieces to `pieces` (32-byte descriptors as in
  * costa_debug_tiles), and up to cap_groups group offsets to `groups` (group
  * g covers pieces [groups[g], groups[g + 1]), so there are *ngroups + 1
@@ -377,6 +377,18 @@ costa_status costa_debug_tiles(costa_layout A, costa_layout B, costa_op op, void
 costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
                                void *pieces, int64_t cap_pieces, uint32_t *groups, int64_t cap_groups,
                                int64_t *ntiles, int64_t *npieces, int64_t *ngroups);
+
+/* Diagnostics (host only, no device work): the aligned full-size tiles of
+ * (A, B, op) as x-halves, the list that the f32 kinds and the f64 / c64
+ * axpby kind with beta = +-2^k run on.  A tile at least 32 high and wider
+ * than 16 along A's contiguous axis becomes two tiles, columns [0, 16) and
+ * the rest, adjacent in the list; the others stay as they are.  Writes up
+ * to cap_tiles 32-byte descriptors (as in costa_debug_tiles) to `tiles` and
+ * the total to *ntiles, which is 0 when the pair has no halves list: 16-byte
+ * elements, A blocks longer than 256 along A's contiguous axis, op = N with
+ * 8-byte elements, or no tile to cut. */
+costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
+                                int64_t *ntiles);
 
 /* Frees every cached plan (synchronizes the device). */
 costa_status costa_release_plans(void);

@@ -85,6 +85,7 @@ def _load():
         "costa_scalapack_release": [],
         "costa_debug_tiles": [P, P, I, P, I64, P],
         "costa_debug_split": [P, P, I, P, I64, P, I64, P, I64, P, P, P],
+        "costa_debug_halves": [P, P, I, P, I64, P],
         "costa_phase_timing": [I],
         "costa_phase_times": [P, P],
     }
@@ -455,6 +456,16 @@ def costa_debug_split(A: Layout, B: Layout, op: str):
                                   pieces.ctypes.data, npc.value, groups.ctypes.data, ngo,
                                   ctypes.byref(nt), ctypes.byref(npc), ctypes.byref(ng)))
     return tiles[:nt.value], pieces[:npc.value], groups[:ngo]
+
+
+def costa_debug_halves(A: Layout, B: Layout, op: str) -> np.ndarray:
+    """The aligned tiles as x-halves (empty when the pair has no halves list)."""
+    cnt = ctypes.c_int64()
+    _check(_lib.costa_debug_halves(A.handle, B.handle, OPS[op], None, 0, ctypes.byref(cnt)))
+    out = np.zeros(max(1, cnt.value), dtype=TILE_DTYPE)
+    _check(_lib.costa_debug_halves(A.handle, B.handle, OPS[op], out.ctypes.data, cnt.value,
+                                   ctypes.byref(cnt)))
+    return out[:cnt.value]
 
 
 def costa_debug_tiles(A: Layout, B: Layout, op: str) -> np.ndarray:

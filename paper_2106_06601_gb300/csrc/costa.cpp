@@ -420,29 +420,11 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     }
     const SplitList split = split_small(std::move(list), es);
     const SplitOffsets off_tiles = arena.add_split(split);
-    // The aligned 32 x 32 tiles also as x-halves (two tiles of at most ts / 2
-    // along A's contiguous axis), for problems whose A blocks are at most 256
-    // elements along that axis: used by every f32 kind, and by the f64 / c64
-    // axpby kind with beta = +-2^k in transposing problems.  Measured on
-    // GB300, same box:
-    //  - f32, 8192^2, BC64 -> BC128: T copy 81 -> 89%, T beta=0.5 88 -> 91%,
-    //    N copy 84 -> 91% of copy; c4 6243 -> 6372 GB/s (its 32 x 16 tiles
-    //    stay whole: halving them cost c4 7%);
-    //  - f64 T, BC64 -> BC128, beta=0.5 (c2) 6184 -> 6338 GB/s; c64 T +8%;
-    //  - lost: the other 8-byte kinds (f64 T copy 91 -> 87%), c128, op = N
-    //    for 8-byte types, and targets of whole panels (1024- and 4096-row
-    //    blocks: 2-6%).
+    // The aligned tiles also as x-halves (see use_halves), for the kinds
+    // that run on them (see launch_list in transform_impl).
     std::vector<char> halve(static_cast<size_t>(n), 0);
-    for (int k = 0; k < n; ++k) {
-        const costa_layout_s *a = plan->probs[k].A;
-        const bool rows_fast = a->blocks.empty() || a->blocks[0].order == COSTA_COL_MAJOR;
-        const std::vector<int64_t> &S = rows_fast ? a->R : a->C;
-        int64_t widest = 0;
-        for (size_t i = 0; i + 1 < S.size(); ++i) widest = std::max(widest, S[i + 1] - S[i]);
-        halve[k] = widest <= 256 && (es == 4 || plan->probs[k].op != COSTA_OP_N);
-    }
-    const std::vector<TileDesc> halves =
-        es <= 8 ? split_x_halves(split.big, ts / 2, es, halve) : std::vector<TileDesc>();
+    for (int k = 0; k < n; ++k) halve[k] = use_halves(plan->probs[k], es);
+    const std::vector<TileDesc> halves = split_x_halves(split.big, ts / 2, es, halve);
     const size_t off_halves = halves.empty() ? 0 : arena.add_vec(halves);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
@@ -1200,6 +1182,29 @@ costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void
     if (kt) std::memcpy(tiles, whole.data(), kt * sizeof(TileDesc));
     if (kp) std::memcpy(pieces, sp.pieces.data(), kp * sizeof(TileDesc));
     if (kg) std::memcpy(groups, sp.groups.data(), kg * sizeof(uint32_t));
+    return COSTA_OK;
+}
+
+costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
+                                int64_t *ntiles) {
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    if (!ntiles || (cap_tiles > 0 && !tiles)) return fail(COSTA_ERR_INVALID_ARG, "bad arguments");
+    const int es = esize_of(A->dt), ts = tile_extent(es);
+    ProblemHost ph;
+    ph.A = A;
+    ph.B = B;
+    ph.op = op;
+    ph.rows = cut_pair_axis(A, B, op, 0, ts);
+    ph.cols = cut_pair_axis(A, B, op, 1, ts);
+    std::vector<TileDesc> list;
+    append_direct_tiles(ph, 0, es, ts, list);
+    const SplitList sp = split_small(std::move(list), es);
+    const std::vector<TileDesc> halves =
+        split_x_halves(sp.big, ts / 2, es, std::vector<char>(1, use_halves(ph, es) ? 1 : 0));
+    *ntiles = static_cast<int64_t>(halves.size());
+    const size_t k = static_cast<size_t>(std::min<int64_t>(cap_tiles, *ntiles));
+    if (k) std::memcpy(tiles, halves.data(), k * sizeof(TileDesc));
     return COSTA_OK;
 }
 

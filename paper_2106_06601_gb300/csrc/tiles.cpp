@@ -136,6 +136,24 @@ int cut_pieces(const TileDesc &d, int es, TileDesc *out) {
     return k;
 }
 
+// Measured on GB300, same box, halves against whole 32 x 32 tiles:
+//  - f32, 8192^2, BC64 -> BC128: T copy 81 -> 89%, T beta=0.5 88 -> 91%,
+//    N copy 84 -> 91% of the copy bandwidth; c4 6243 -> 6372 GB/s, with its
+//    32 x 16 tiles left whole (halving them too cost c4 7%);
+//  - f64 T, BC64 -> BC128, beta=0.5 (c2): 6184 -> 6338 GB/s; c64 T +8%;
+//  - lost: the other 8-byte kinds (f64 T copy 91 -> 87%), c128 (95 -> 86%),
+//    op = N for 8-byte types (no gain), and targets of whole panels
+//    (1024- and 4096-row blocks: 2-6%).
+bool use_halves(const ProblemHost &ph, int es) {
+    if (es != 4 && es != 8) return false;
+    const costa_layout_s *a = ph.A;
+    const bool rows_fast = a->blocks.empty() || a->blocks[0].order == COSTA_COL_MAJOR;
+    const std::vector<int64_t> &S = rows_fast ? a->R : a->C;
+    int64_t widest = 0;
+    for (size_t i = 0; i + 1 < S.size(); ++i) widest = std::max(widest, S[i + 1] - S[i]);
+    return widest <= 256 && (es == 4 || ph.op != COSTA_OP_N);
+}
+
 std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, int es,
                                      const std::vector<char> &halve) {
     const int64_t n = static_cast<int64_t>(list.size());

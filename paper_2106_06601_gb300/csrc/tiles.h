@@ -124,4 +124,10 @@ SplitList split_small(std::vector<TileDesc> &&list, int es);
 std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, int es,
                                      const std::vector<char> &halve);
 
+// Whether a problem's aligned tiles are also listed as x-halves: for 4- and
+// 8-byte types, when A's blocks are at most 256 elements along A's
+// contiguous axis, and, for 8-byte types, when op transposes.  Every f32
+// kind runs on the halves, and the f64 / c64 axpby kind with beta = +-2^k.
+bool use_halves(const ProblemHost &ph, int es);
+
 }  // namespace costa

@@ -313,3 +313,73 @@ def test_plan_independent_of_thread_count():
         assert r.returncode == 0, r.stderr
         out.append(r.stdout.strip())
     assert out[0] == out[1] == out[2]
+
+
+def check_halves(p):
+    """The x-halves list: each aligned full-size tile at least 32 high and
+    wider than 16 along x becomes two tiles (x in [0, 16) and the rest,
+    adjacent, on the vector path, inside the buffers); the others stay as
+    they are, in order; no halves list for c128, for A blocks longer than
+    256 along x, or for op = N with 8-byte elements."""
+    es = {"f32": 4, "f64": 8, "c64": 8, "c128": 16}[p.dtype]
+    LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+    try:
+        big, _, _ = costa.costa_debug_split(LA, LB, p.op)
+        halves = costa.costa_debug_halves(LA, LB, p.op)
+    finally:
+        LA.destroy()
+        LB.destroy()
+    aligned = big[(big["flags"] & 2) != 0]
+    rows_fast = p.A.order.flat[0] == L.COL_MAJOR if p.A.order.size else True
+    blocks = np.diff(p.A.rsplit if rows_fast else p.A.csplit)
+    rule = es in (4, 8) and blocks.max(initial=0) <= 256 and (es == 4 or p.op != "N")
+    cut = (aligned["nx"] > 16) & (aligned["ny"] >= 32)
+    if not rule or not cut.any():
+        assert len(halves) == 0
+        return
+    assert len(halves) == len(aligned) + int(cut.sum())
+    k = 0
+    for d, c in zip(aligned, cut):
+        if not c:
+            assert halves[k].tobytes() == d.tobytes()
+            k += 1
+            continue
+        h0, h1 = halves[k], halves[k + 1]
+        k += 2
+        tr = bool(d["flags"] & 1)
+        assert (h0["nx"], h1["nx"]) == (16, d["nx"] - 16)
+        for h in (h0, h1):
+            assert (h["ny"], h["dld"], h["sld"], h["prob"], h["flags"]) == \
+                   (d["ny"], d["dld"], d["sld"], d["prob"], d["flags"])
+            assert h["src"] % 16 == 0 and h["dst"] % 16 == 0
+        assert h0["dst"] == d["dst"] and h0["src"] == d["src"]
+        assert int(h1["dst"]) == int(d["dst"]) + 16 * es
+        assert int(h1["src"]) == int(d["src"]) + (16 * int(d["sld"]) if tr else 16) * es
+    _in_buffers(halves, p.A, es, "dst")
+    _in_buffers(halves, p.B, es, "src")
+
+
+def test_halves():
+    for name in ("c1", "c2", "c3", "c5"):
+        check_halves(C.CONFIGS[name]())
+    for p in C.c4()[:8]:
+        check_halves(p)
+    for case in range(200):
+        check_halves(C.fuzz_problem(case))
+    # block-cyclic pairs with full tiles: every element type, op and storage,
+    # A blocks of 64 and 128 (halves) and 512 (none)
+    n_with = 0
+    for dt in ("f32", "f64", "c64", "c128"):
+        for op in ("N", "T", "C"):
+            for k, (amb, st, pad) in enumerate(((64, "C", 0), (128, "R", 2), (512, "C", 1))):
+                m, n = 520, 392
+                am, an = (m, n) if op == "N" else (n, m)
+                B = L.block_cyclic(m, n, 96, 80, 2, 2, storage="CR"[k % 2])
+                A = L.block_cyclic(am, an, amb, amb, 2, 2, storage=st, ld_pad=pad)
+                p = C.Problem("halves", dt, op, 2.0, 0.5, A, B, "uniform", "uniform", C.SEED0)
+                check_halves(p)
+                LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+                n_with += len(costa.costa_debug_halves(LA, LB, p.op)) > 0
+                LA.destroy()
+                LB.destroy()
+    assert n_with >= 8  # the halves path is exercised
