@@ -114,6 +114,7 @@ struct MessageData {
     bool built = false;
     void *d_mem = nullptr;       // pack, local and unpack tile lists
     DevList pack, local, unpack;
+    DevList local_halves, unpack_halves;  // local and unpack with x-halves (see use_halves)
     void *d_staging = nullptr;
     int64_t staging_bytes = 0;
 };
@@ -613,10 +614,16 @@ costa_status ensure_message(Plan &plan, bool relabel) {
     }
     const SplitList s_pack = split_small(std::move(pack), es), s_local = split_small(std::move(local), es),
                     s_unpack = split_small(std::move(unpack), es);
+    std::vector<char> halve(plan.probs.size(), 0);
+    for (size_t k = 0; k < plan.probs.size(); ++k) halve[k] = use_halves(plan.probs[k], es);
+    const std::vector<TileDesc> h_local = split_x_halves(s_local.big, plan.ts / 2, es, halve),
+                                h_unpack = split_x_halves(s_unpack.big, plan.ts / 2, es, halve);
     Arena arena;
     const SplitOffsets o_pack = arena.add_split(s_pack);
     const SplitOffsets o_local = arena.add_split(s_local);
     const SplitOffsets o_unpack = arena.add_split(s_unpack);
+    const size_t o_hl = h_local.empty() ? 0 : arena.add_vec(h_local);
+    const size_t o_hu = h_unpack.empty() ? 0 : arena.add_vec(h_unpack);
     cudaError_t ce = cudaMalloc(&m.d_mem, arena.host.size());
     if (ce != cudaSuccess) return fail(COSTA_ERR_ALLOC, "cudaMalloc(message tables): %s", cudaGetErrorString(ce));
     ce = cudaMemcpy(m.d_mem, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
@@ -625,6 +632,16 @@ costa_status ensure_message(Plan &plan, bool relabel) {
     m.pack = resolve(db, o_pack, s_pack);
     m.local = resolve(db, o_local, s_local);
     m.unpack = resolve(db, o_unpack, s_unpack);
+    m.local_halves = m.local;
+    m.unpack_halves = m.unpack;
+    if (!h_local.empty()) {
+        m.local_halves.tiles = reinterpret_cast<const TileDesc *>(db + o_hl);
+        m.local_halves.ntiles = static_cast<int64_t>(h_local.size());
+    }
+    if (!h_unpack.empty()) {
+        m.unpack_halves.tiles = reinterpret_cast<const TileDesc *>(db + o_hu);
+        m.unpack_halves.ntiles = static_cast<int64_t>(h_unpack.size());
+    }
     m.built = true;
     plan.stats.staging_bytes = m.staging_bytes;
     return COSTA_OK;
@@ -806,10 +823,10 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     if (ce == cudaSuccess) ce = launch_remap(lp, K_COPY, stream);
     if (ce == cudaSuccess) ce = mark(1);
     if (ce != cudaSuccess) return cuda_fail(ce, "pack kernel launch");
-    ce = launch_list(m.local, nullptr);
+    ce = launch_list(m.local, &m.local_halves);
     if (ce == cudaSuccess) ce = mark(2);
     if (ce != cudaSuccess) return cuda_fail(ce, "local remap kernel launch");
-    ce = launch_list(m.unpack, nullptr);
+    ce = launch_list(m.unpack, &m.unpack_halves);
     if (ce == cudaSuccess) ce = mark(3);
     if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
     if (timer) timer->nphases = 3;
