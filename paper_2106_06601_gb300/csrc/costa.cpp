@@ -73,11 +73,13 @@ struct DevList {
     const TileDesc *pieces = nullptr;
     const uint32_t *groups = nullptr;
     int64_t ngroups = 0;
+    const uint32_t *groups_a = nullptr;  // the groups of the kinds that read A
+    int64_t ngroups_a = 0;
     bool empty() const { return ntiles == 0 && nmtiles == 0 && ngroups == 0; }
 };
 
 struct SplitOffsets {
-    size_t tiles, mtiles, pieces, groups;
+    size_t tiles, mtiles, pieces, groups, groups_a;
 };
 
 // One device allocation holding all tables of a plan, built on the host
@@ -94,7 +96,7 @@ struct Arena {
         return add(v.data(), v.size() * sizeof(V));
     }
     SplitOffsets add_split(const SplitList &l) {
-        return {add_vec(l.big), add_vec(l.mis), add_vec(l.pieces), add_vec(l.groups)};
+        return {add_vec(l.big), add_vec(l.mis), add_vec(l.pieces), add_vec(l.groups), add_vec(l.groups_a)};
     }
 };
 
@@ -107,6 +109,8 @@ DevList resolve(const char *dbase, const SplitOffsets &o, const SplitList &l) {
     d.pieces = reinterpret_cast<const TileDesc *>(dbase + o.pieces);
     d.groups = reinterpret_cast<const uint32_t *>(dbase + o.groups);
     d.ngroups = l.ngroups();
+    d.groups_a = reinterpret_cast<const uint32_t *>(dbase + o.groups_a);
+    d.ngroups_a = l.ngroups_a();
     return d;
 }
 
@@ -419,7 +423,8 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
         costa_status st = check_extents(list, es, "direct");
         if (st != COSTA_OK) return st;
     }
-    const SplitList split = split_small(std::move(list), es);
+    const bool cplx = plan->dtype == COSTA_C64 || plan->dtype == COSTA_C128;
+    const SplitList split = split_small(std::move(list), es, cplx);
     const SplitOffsets off_tiles = arena.add_split(split);
     // The aligned tiles also as x-halves (see use_halves), for the kinds
     // that run on them (see launch_list in transform_impl).
@@ -612,8 +617,10 @@ costa_status ensure_message(Plan &plan, bool relabel) {
         costa_status st = check_extents(*l.first, es, l.second);
         if (st != COSTA_OK) return st;
     }
-    const SplitList s_pack = split_small(std::move(pack), es), s_local = split_small(std::move(local), es),
-                    s_unpack = split_small(std::move(unpack), es);
+    const bool cplx = plan.dtype == COSTA_C64 || plan.dtype == COSTA_C128;
+    const SplitList s_pack = split_small(std::move(pack), es, cplx),
+                    s_local = split_small(std::move(local), es, cplx),
+                    s_unpack = split_small(std::move(unpack), es, cplx);
     std::vector<char> halve(plan.probs.size(), 0);
     for (size_t k = 0; k < plan.probs.size(); ++k) halve[k] = use_halves(plan.probs[k], es);
     const std::vector<TileDesc> h_local = split_x_halves(s_local.big, plan.ts / 2, es, halve),
@@ -786,6 +793,10 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
             if (halves && (plan->esize == 4 || kind == K_AXPBY2)) {
                 lk.tiles = halves->tiles;
                 lk.ntiles = halves->ntiles;
+            }
+            if (kind != K_COPY && kind != K_SCALE) {  // the groups of the kinds that read A
+                lk.groups = list.groups_a;
+                lk.ngroups = list.ngroups_a;
             }
             cudaError_t e = launch_remap(lk, kind, stream);
             if (e != cudaSuccess) return e;
@@ -1187,7 +1198,7 @@ costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void
     ph.cols = cut_pair_axis(A, B, op, 1, ts);
     std::vector<TileDesc> list;
     append_direct_tiles(ph, 0, es, ts, list);
-    const SplitList sp = split_small(std::move(list), es);
+    const SplitList sp = split_small(std::move(list), es, A->dt == COSTA_C64 || A->dt == COSTA_C128);
     std::vector<TileDesc> whole = sp.big;  // the tile kernel's tiles: aligned, then misaligned
     whole.insert(whole.end(), sp.mis.begin(), sp.mis.end());
     *ntiles = static_cast<int64_t>(whole.size());
@@ -1216,7 +1227,7 @@ costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, voi
     ph.cols = cut_pair_axis(A, B, op, 1, ts);
     std::vector<TileDesc> list;
     append_direct_tiles(ph, 0, es, ts, list);
-    const SplitList sp = split_small(std::move(list), es);
+    const SplitList sp = split_small(std::move(list), es, A->dt == COSTA_C64 || A->dt == COSTA_C128);
     const std::vector<TileDesc> halves =
         split_x_halves(sp.big, ts / 2, es, std::vector<char>(1, use_halves(ph, es) ? 1 : 0));
     *ntiles = static_cast<int64_t>(halves.size());

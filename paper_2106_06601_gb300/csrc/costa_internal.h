@@ -170,6 +170,20 @@ COSTA_HD constexpr int tile_passes(int esize) { return tile_extent(esize) * tile
 #define COSTA_GROUP_4 8
 #endif
 COSTA_HD constexpr int group_pieces(int esize) { return esize == 4 ? COSTA_GROUP_4 : tile_passes(esize); }
+// Groups for the kinds that read A, of 8-byte types: smaller (measured on
+// GB300, 8192^2 T, BC8: f64 86 -> 91% of copy at 8 pieces, c64 87 -> 93% at
+// 12; the copy kind loses 10-15% on groups below 16, so it keeps those).
+#ifndef COSTA_GROUP_8A
+#define COSTA_GROUP_8A 8
+#endif
+#ifndef COSTA_GROUP_8CA
+#define COSTA_GROUP_8CA 12
+#endif
+COSTA_HD constexpr int group_pieces_a(int esize, bool cplx) {
+    return esize == 8 ? (cplx ? COSTA_GROUP_8CA : COSTA_GROUP_8A) : group_pieces(esize);
+}
+static_assert(group_pieces_a(8, false) <= group_pieces(8) && group_pieces_a(8, true) <= group_pieces(8),
+              "a group must fit the small-tile kernel's slots");
 
 // Launches the remap kernel for (args.dtype, kind) over a tile list.  With
 // args.per_problem set, the kernel skips the tiles of problems of another kind.

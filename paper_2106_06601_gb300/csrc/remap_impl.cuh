@@ -910,7 +910,9 @@ template <typename T, int KIND> struct SCfg {
     static constexpr int MINB = sizeof(T) == 4 ? COSTA_SMINB_4
                               : sizeof(T) == 16 ? (KCfg<T, KIND>::READS_A ? COSTA_SMINB_16A : COSTA_SMINB_16)
                               : KCfg<T, KIND>::HEAVY ? COSTA_SMINB_8H : COSTA_SMINB_8;
-    static constexpr int NS = group_pieces(static_cast<int>(sizeof(T)));
+    // pieces per group: the host's cap for the groups this kind receives
+    static constexpr int NS = KCfg<T, KIND>::READS_A ? group_pieces_a(static_cast<int>(sizeof(T)), ET<T>::CPLX != 0)
+                                                    : group_pieces(static_cast<int>(sizeof(T)));
     static constexpr int BUF_BYTES = NS * 512 + NS * 32;  // slots, then the group's descriptors
 };
 

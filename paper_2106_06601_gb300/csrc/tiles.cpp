@@ -180,7 +180,7 @@ std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, 
     return out;
 }
 
-SplitList split_small(std::vector<TileDesc> &&all, int es) {
+SplitList split_small(std::vector<TileDesc> &&all, int es, bool cplx) {
     SplitList out;
     // misaligned tiles go to their own instance of the tile kernel
     std::vector<TileDesc> list;
@@ -233,18 +233,21 @@ SplitList split_small(std::vector<TileDesc> &&all, int es) {
         out.big = std::move(list);
         return out;
     }
-    // groups in list order: at most group_pieces(es) pieces of one problem
-    const int cap = group_pieces(es);
-    int in_group = 0, group_prob = -1;
-    for (size_t k = 0; k < out.pieces.size(); ++k) {
-        if (in_group == cap || out.pieces[k].prob != group_prob || out.groups.empty()) {
-            out.groups.push_back(static_cast<uint32_t>(k));
-            in_group = 0;
-            group_prob = out.pieces[k].prob;
+    // groups in list order: at most `cap` pieces of one problem
+    auto make_groups = [&](int cap, std::vector<uint32_t> &g) {
+        int in_group = 0, group_prob = -1;
+        for (size_t k = 0; k < out.pieces.size(); ++k) {
+            if (in_group == cap || out.pieces[k].prob != group_prob || g.empty()) {
+                g.push_back(static_cast<uint32_t>(k));
+                in_group = 0;
+                group_prob = out.pieces[k].prob;
+            }
+            ++in_group;
         }
-        ++in_group;
-    }
-    if (!out.groups.empty()) out.groups.push_back(static_cast<uint32_t>(out.pieces.size()));
+        if (!g.empty()) g.push_back(static_cast<uint32_t>(out.pieces.size()));
+    };
+    make_groups(group_pieces(es), out.groups);
+    make_groups(group_pieces_a(es, cplx), out.groups_a);
     return out;
 }
 

@@ -82,7 +82,9 @@ struct SplitList {
     std::vector<TileDesc> mis;  // misaligned tiles (16-byte windows or single elements)
     std::vector<TileDesc> pieces;
     std::vector<uint32_t> groups;  // group g = pieces [groups[g], groups[g + 1])
+    std::vector<uint32_t> groups_a;  // the same pieces in the groups of the kinds that read A
     int64_t ngroups() const { return groups.empty() ? 0 : static_cast<int64_t>(groups.size()) - 1; }
+    int64_t ngroups_a() const { return groups_a.empty() ? 0 : static_cast<int64_t>(groups_a.size()) - 1; }
 };
 
 // Visits the tiles of a problem in the global super-tile order (see
@@ -114,7 +116,7 @@ int fast_tile_passes(const TileDesc &d, int es);
 int small_limit(int es);
 bool is_small(const TileDesc &d, int es);
 int cut_pieces(const TileDesc &d, int es, TileDesc *out);
-SplitList split_small(std::vector<TileDesc> &&list, int es);
+SplitList split_small(std::vector<TileDesc> &&list, int es, bool cplx);
 
 // The aligned tiles of problems k with halve[k] that are wider than hx
 // along x (A's contiguous axis) and at least 2 hx high, cut into [0, hx)
