@@ -230,3 +230,14 @@ def test_sparse_relabel_is_exact():
                        env=dict(os.environ, COSTA_RELABEL_SPARSE_MIN_P="1"), timeout=600)
     assert r.returncode == 0, r.stderr
     assert r.stdout.strip() == "[]", r.stdout
+
+
+def test_scalar_marshalling_matches_element_type():
+    """The binding hands alpha and beta to the C ABI as one value of A's
+    element type: the bytes must be those of numpy's scalar of that type."""
+    import ctypes
+    for dt, v in (("f32", 0.1), ("f64", 0.1), ("c64", 0.25 - 1.5j), ("c128", 1 / 3 + 2j), ("c64", 2.0)):
+        c = costa._scalar1(dt, v)
+        want = np.asarray(v, dtype={"f32": np.float32, "f64": np.float64, "c64": np.complex64,
+                                    "c128": np.complex128}[dt]).tobytes()
+        assert ctypes.string_at(ctypes.addressof(c), ctypes.sizeof(c)) == want
