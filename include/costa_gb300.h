@@ -378,6 +378,15 @@ costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void
                                void *pieces, int64_t cap_pieces, uint32_t *groups, int64_t cap_groups,
                                int64_t *ntiles, int64_t *npieces, int64_t *ngroups);
 
+/* Diagnostics (host only, no device work): the group offsets over the
+ * pieces of costa_debug_split that the small-tile kernel uses for the copy
+ * and scale kinds (reads_a = 0) or for the kinds that read A (reads_a != 0:
+ * at most 8 pieces per group for f64, 12 for c64, as for copy otherwise).
+ * Writes up to cap_groups offsets to `groups` (group g covers pieces
+ * [groups[g], groups[g + 1])) and the number of groups to *ngroups. */
+costa_status costa_debug_groups(costa_layout A, costa_layout B, costa_op op, int reads_a, uint32_t *groups,
+                                int64_t cap_groups, int64_t *ngroups);
+
 /* Diagnostics (host only, no device work): the aligned full-size tiles of
  * (A, B, op) as x-halves, the list that the f32 kinds and the f64 / c64
  * axpby kind with beta = +-2^k run on.  A tile at least 32 high and wider

@@ -86,6 +86,7 @@ def _load():
         "costa_debug_tiles": [P, P, I, P, I64, P],
         "costa_debug_split": [P, P, I, P, I64, P, I64, P, I64, P, P, P],
         "costa_debug_halves": [P, P, I, P, I64, P],
+        "costa_debug_groups": [P, P, I, I, P, I64, P],
         "costa_phase_timing": [I],
         "costa_phase_times": [P, P],
     }
@@ -456,6 +457,17 @@ def costa_debug_split(A: Layout, B: Layout, op: str):
                                   pieces.ctypes.data, npc.value, groups.ctypes.data, ngo,
                                   ctypes.byref(nt), ctypes.byref(npc), ctypes.byref(ng)))
     return tiles[:nt.value], pieces[:npc.value], groups[:ngo]
+
+
+def costa_debug_groups(A: Layout, B: Layout, op: str, reads_a: bool) -> np.ndarray:
+    """Group offsets of the small-tile pieces for one class of kinds."""
+    cnt = ctypes.c_int64()
+    _check(_lib.costa_debug_groups(A.handle, B.handle, OPS[op], int(reads_a), None, 0, ctypes.byref(cnt)))
+    n = cnt.value + 1 if cnt.value > 0 else 0
+    out = np.zeros(max(1, n), dtype=np.uint32)
+    _check(_lib.costa_debug_groups(A.handle, B.handle, OPS[op], int(reads_a), out.ctypes.data, n,
+                                   ctypes.byref(cnt)))
+    return out[:n]
 
 
 def costa_debug_halves(A: Layout, B: Layout, op: str) -> np.ndarray:

@@ -1213,6 +1213,28 @@ costa_status costa_debug_split(costa_layout A, costa_layout B, costa_op op, void
     return COSTA_OK;
 }
 
+costa_status costa_debug_groups(costa_layout A, costa_layout B, costa_op op, int reads_a, uint32_t *groups,
+                                int64_t cap_groups, int64_t *ngroups) {
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    if (!ngroups || (cap_groups > 0 && !groups)) return fail(COSTA_ERR_INVALID_ARG, "bad arguments");
+    const int es = esize_of(A->dt), ts = tile_extent(es);
+    ProblemHost ph;
+    ph.A = A;
+    ph.B = B;
+    ph.op = op;
+    ph.rows = cut_pair_axis(A, B, op, 0, ts);
+    ph.cols = cut_pair_axis(A, B, op, 1, ts);
+    std::vector<TileDesc> list;
+    append_direct_tiles(ph, 0, es, ts, list);
+    const SplitList sp = split_small(std::move(list), es, A->dt == COSTA_C64 || A->dt == COSTA_C128);
+    const std::vector<uint32_t> &g = reads_a ? sp.groups_a : sp.groups;
+    *ngroups = reads_a ? sp.ngroups_a() : sp.ngroups();
+    const size_t k = static_cast<size_t>(std::min<int64_t>(cap_groups, static_cast<int64_t>(g.size())));
+    if (k) std::memcpy(groups, g.data(), k * sizeof(uint32_t));
+    return COSTA_OK;
+}
+
 costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
                                 int64_t *ntiles) {
     costa_status s = validate_pair(A, B, op);

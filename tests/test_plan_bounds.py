@@ -280,6 +280,37 @@ def test_small_block_split():
         check_split(C.small_block_problem(case), exact=True)
 
 
+def test_groups_of_kinds_that_read_a():
+    """The second grouping of the pieces (kinds that read A): the same pieces
+    in order, one problem per group, at most 8 (f64) or 12 (c64) per group,
+    and the copy grouping unchanged for the other types."""
+    caps = {"f32": 8, "f64": 8, "c64": 12, "c128": 32}
+    seen = set()
+    for case in range(96):
+        p = C.small_block_problem(case)
+        LA, LB = _layout(p.A, p.dtype), _layout(p.B, p.dtype)
+        try:
+            _, pieces, groups = costa.costa_debug_split(LA, LB, p.op)
+            g0 = costa.costa_debug_groups(LA, LB, p.op, False)
+            ga = costa.costa_debug_groups(LA, LB, p.op, True)
+        finally:
+            LA.destroy()
+            LB.destroy()
+        assert np.array_equal(g0, groups)
+        if len(pieces) == 0:
+            assert len(ga) == 0
+            continue
+        ga = ga.astype(np.int64)
+        assert ga[0] == 0 and ga[-1] == len(pieces) and np.all(np.diff(ga) >= 1)
+        assert np.all(np.diff(ga) <= caps[p.dtype])
+        for a, b in zip(ga[:-1], ga[1:]):
+            assert len(np.unique(pieces["prob"][a:b])) == 1
+        if p.dtype in ("f32", "c128"):
+            assert np.array_equal(ga, groups.astype(np.int64))
+        seen.add(p.dtype)
+    assert {"f64", "c64"} <= seen
+
+
 _DUMP = """
 import hashlib, sys
 sys.path.insert(0, %r)
