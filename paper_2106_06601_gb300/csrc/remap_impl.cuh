@@ -128,15 +128,18 @@ template <typename T> struct Cfg {
 // Launch shape per element type and combine kind (measured on GB300): warps
 // per block, resident blocks per SM the registers must allow, and
 // shared-memory buffers per warp (the warp keeps NBUF - 1 tiles' copies in
-// flight ahead of the tile it writes).  8-byte types with the light kinds
-// run more warps without look-ahead; the general kinds (non-power-of-two
-// beta, complex scalars) need the registers of 3 blocks and use a 2-deep
-// ring; in the misaligned-tile instance the light kinds that read A (one
-// element per lane, a whole tile of A in registers) run 4 blocks, which
-// their registers fit without spills.  4-byte kinds that read A run 3
-// blocks without look-ahead, those that do not 2 blocks with a 2-deep ring.  16-byte kinds that read A hold
-// a whole 16 KB tile of A in registers; they run two blocks without
-// look-ahead.  Overridable at build time for tuning.
+// flight ahead of the tile it writes).
+//  - 8-byte types: the light kinds run more warps without look-ahead; the
+//    general kinds (non-power-of-two beta, complex scalars) need the
+//    registers of 3 blocks and use a 2-deep ring; in the misaligned-tile
+//    instance the light kinds that read A (one element per lane, a whole
+//    tile of A in registers) run 4 blocks, which their registers fit
+//    without spills.
+//  - 4-byte types: the kinds that read A run 3 blocks without look-ahead,
+//    the others 2 blocks with a 2-deep ring.
+//  - 16-byte types: the kinds that read A hold a whole 16 KB tile of A in
+//    registers and run two blocks without look-ahead.
+// Overridable at build time for tuning.
 template <typename T, int KIND, bool MIS = false> struct KCfg {
     static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX;
     static constexpr bool READS_A = KIND != K_COPY && KIND != K_SCALE;
