@@ -1,6 +1,8 @@
-"""CPU check of the index arithmetic of the misaligned-tile window path
-(`stage_issue_w`, `stage_drain_w` in the remap kernel source), replayed per
-lane for random tiles before any kernel runs it.
+"""CPU check of the index arithmetic of the misaligned-tile paths: the
+16-byte window path (`stage_issue_w`, `stage_drain_w` in the remap kernel
+source) and the one-element-per-lane path of the kinds that read A
+(`stage_issue_e`, `load_a_e`, `stage_drain_e`), replayed per lane for random
+tiles before any kernel runs them.
 
 For a tile of nx x ny elements (nx, ny <= 32), transposed or not, with any
 element-aligned start addresses and leading dimensions of source and target,
@@ -122,3 +124,61 @@ def test_window_map(es):
     rnd = random.Random(2106066010 + es)
     for _ in range(8000):
         replay(es, rnd)
+
+
+def replay_elements(es, rnd):
+    """The one-element-per-lane path: every staged element lands in the
+    TS x TS buffer at c ^ (r mod TS) of its row, is read back by the lane
+    that writes its target element, and every target element of the tile is
+    loaded and written exactly once."""
+    nx = TS if rnd.random() < 0.3 else rnd.randint(1, TS)
+    ny = TS if rnd.random() < 0.3 else rnd.randint(1, TS)
+    tr = rnd.random() < 0.5
+    runs, ln = (nx, ny) if tr else (ny, nx)
+    sld = ln + rnd.randint(0, 9)
+    dld = nx + rnd.randint(0, 9)
+    src = (1 << 20) + rnd.randrange(64) * es
+    dst = (1 << 24) + rnd.randrange(64) * es
+
+    def slot_e(r, c):
+        assert 0 <= r < TS and 0 <= c < TS
+        return r * TS + (c ^ (r & (TS - 1)))
+
+    smem = {}
+    c, r0, rpp = lane_map(ln, 0)  # the map's shape is the same for every lane
+    assert rpp >= 1
+    for lane in range(32):
+        c, r0, rpp = lane_map(ln, lane)
+        if c >= ln:
+            continue
+        for r in range(r0, runs, rpp):
+            ga = src + (r * sld + c) * es
+            assert src + r * sld * es <= ga < src + (r * sld + ln) * es
+            smem[slot_e(r, c)] = ga
+    written, loaded = set(), set()
+    vec = 16 // es
+    ne = (TS // (32 // (TS // vec))) * vec  # elements per lane of a full tile
+    for lane in range(32):
+        c, r0, rpp = lane_map(nx, lane)
+        if c >= nx:
+            continue
+        npass = (ny + rpp - 1) // rpp
+        assert npass <= ne
+        for p in range(npass):
+            y = p * rpp + r0
+            if y >= ny:
+                continue
+            want = src + ((c * sld + y) if tr else (y * sld + c)) * es
+            assert smem.get(slot_e(c, y) if tr else slot_e(y, c)) == want
+            assert (y, c) not in written
+            written.add((y, c))
+            loaded.add((y, c))
+    every = {(y, x) for y in range(ny) for x in range(nx)}
+    assert written == every and loaded == every
+
+
+@pytest.mark.parametrize("es", [4, 8])
+def test_element_map(es):
+    rnd = random.Random(2106066020 + es)
+    for _ in range(8000):
+        replay_elements(es, rnd)
