@@ -10,6 +10,7 @@ docstring; every function here is pinned by tests/test_oracle_pins.py.
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes
 import os
 import subprocess
@@ -50,31 +51,68 @@ class _OLayout(ctypes.Structure):
                 ("order", ctypes.c_void_p)]
 
 
+def _bind(cdll):
+    P = ctypes.c_void_p
+    cdll.oracle_transform.argtypes = [ctypes.c_int, ctypes.c_int, P, P, P, P, P, P,
+                                      ctypes.c_int64, ctypes.c_int64, ctypes.c_int]
+    cdll.oracle_transform.restype = ctypes.c_int
+    cdll.oracle_volume.argtypes = [ctypes.c_int, P, P, ctypes.c_int, P, ctypes.c_int]
+    cdll.oracle_volume.restype = ctypes.c_int
+    cdll.oracle_locate_many.argtypes = [P, ctypes.c_int64, P, P, P, P]
+    cdll.oracle_combine_many.argtypes = [ctypes.c_int, ctypes.c_int, P, P,
+                                         ctypes.c_int64, P, P, P]
+    cdll.oracle_lap_bruteforce.argtypes = [ctypes.c_int, P, P]
+    cdll.oracle_lap_bruteforce.restype = ctypes.c_int64
+    cdll.oracle_lap_subset_dp.argtypes = [ctypes.c_int, P, P]
+    cdll.oracle_lap_subset_dp.restype = ctypes.c_int64
+    cdll.oracle_lap_greedy.argtypes = [ctypes.c_int, P, P]
+    cdll.oracle_lap_greedy.restype = ctypes.c_int64
+    cdll.oracle_cost_W.argtypes = [ctypes.c_int, P, P, P, P]
+    cdll.oracle_cost_W.restype = ctypes.c_double
+    cdll.oracle_copr_bruteforce_cost.argtypes = [ctypes.c_int, P, P, P, P]
+    cdll.oracle_copr_bruteforce_cost.restype = ctypes.c_double
+    return cdll
+
+
 def lib():
     global _lib
     with _lock:
         if _lib is None:
-            _lib = ctypes.CDLL(build())
-            P = ctypes.c_void_p
-            _lib.oracle_transform.argtypes = [ctypes.c_int, ctypes.c_int, P, P, P, P, P, P,
-                                              ctypes.c_int64, ctypes.c_int64, ctypes.c_int]
-            _lib.oracle_transform.restype = ctypes.c_int
-            _lib.oracle_volume.argtypes = [ctypes.c_int, P, P, ctypes.c_int, P, ctypes.c_int]
-            _lib.oracle_volume.restype = ctypes.c_int
-            _lib.oracle_locate_many.argtypes = [P, ctypes.c_int64, P, P, P, P]
-            _lib.oracle_combine_many.argtypes = [ctypes.c_int, ctypes.c_int, P, P,
-                                                 ctypes.c_int64, P, P, P]
-            _lib.oracle_lap_bruteforce.argtypes = [ctypes.c_int, P, P]
-            _lib.oracle_lap_bruteforce.restype = ctypes.c_int64
-            _lib.oracle_lap_subset_dp.argtypes = [ctypes.c_int, P, P]
-            _lib.oracle_lap_subset_dp.restype = ctypes.c_int64
-            _lib.oracle_lap_greedy.argtypes = [ctypes.c_int, P, P]
-            _lib.oracle_lap_greedy.restype = ctypes.c_int64
-            _lib.oracle_cost_W.argtypes = [ctypes.c_int, P, P, P, P]
-            _lib.oracle_cost_W.restype = ctypes.c_double
-            _lib.oracle_copr_bruteforce_cost.argtypes = [ctypes.c_int, P, P, P, P]
-            _lib.oracle_copr_bruteforce_cost.restype = ctypes.c_double
+            _lib = _bind(ctypes.CDLL(build()))
         return _lib
+
+
+def compile_variant(source_text: str, out_path: str) -> str:
+    """Compiles a modified copy of costa_oracle.c with the oracle's own flags.
+    Test hook: the planted-mistake tests build mutated oracles with it."""
+    src = out_path + ".c"
+    with open(src, "w") as f:
+        f.write(source_text)
+    cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-fno-fast-math",
+           "-fPIC", "-shared", "-o", out_path, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    return out_path
+
+
+def source_text() -> str:
+    with open(_SRC) as f:
+        return f.read()
+
+
+@contextlib.contextmanager
+def loaded(path: str):
+    """Runs this module's functions on another build of the oracle (a mutated
+    copy from compile_variant) inside the block.  Test hook only."""
+    global _lib
+    lib()
+    with _lock:
+        saved = _lib
+        _lib = _bind(ctypes.CDLL(path))
+    try:
+        yield
+    finally:
+        with _lock:
+            _lib = saved
 
 
 def _ptr(a: np.ndarray):

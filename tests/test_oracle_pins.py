@@ -138,8 +138,10 @@ def test_linearity_in_alpha():
     assert np.array_equal(A4, 4.0 * A1)
 
 
-def test_locate_matches_block_views():
-    p = C.fuzz_problem(21)
+@pytest.mark.parametrize("case", [21, 8, 30])
+def test_locate_matches_block_views(case):
+    """Cases 8 and 30 have an empty block row or column."""
+    p = C.fuzz_problem(case)
     spec = p.A
     ij = np.array([(i, j) for i in range(spec.m) for j in range(spec.n)], np.int64)
     owner, buf, off = oracle.locate(spec, ij)
@@ -328,44 +330,183 @@ def test_lemma1_gain_equals_cost_reduction():
 
 
 # ----------------------------------------------------------------------------
-# planted mistakes: each pin must fail on a plausible oracle error
+# cost function, COPR and greedy against hand-worked cases (tests/golden)
 # ----------------------------------------------------------------------------
 
-def test_planted_mistakes_are_caught():
-    p = C.fuzz_problem(40, dtype="c128", op="C")
-    p.alpha, p.beta, p.a_kind = 2.0, 0.5, "uniform"
-    B, A = host_problem(p)
-    good = global_matrix(p.A, run_oracle(p, B, A).buffers())
-    want = expected_global(p, B, A)
-    assert np.array_equal(good, want)
-    GB = global_matrix(p.B, B.buffers())
-    GA = global_matrix(p.A, A.buffers())
-    mutants = {
-        "dropped beta term": 2.0 * np.conj(GB.T),
-        "missing conjugate": 2.0 * GB.T + 0.5 * GA,
-        "sign of beta": 2.0 * np.conj(GB.T) - 0.5 * GA,
-    }
-    for name, bad in mutants.items():
-        assert not np.array_equal(bad, want), name
-    # a transposed operand in the volume count breaks the owner-map pin
-    q = C.fuzz_problem(41, op="T")
-    while q.A.m == q.A.n:
-        q = C.fuzz_problem(q.index + 200, op="T")
-    P = q.A.nranks
-    V = oracle.volume("T", q.A, q.B, P)
-    ob, qa = owner_matrix(q.B), owner_matrix(q.A)
-    # a wrong volume (owner maps swapped) differs from the pinned one
-    Vbad = np.bincount((qa.astype(np.int64) * P + ob.T).ravel(), minlength=P * P).reshape(P, P)
-    assert not np.array_equal(Vbad, V) or np.array_equal(Vbad, Vbad.T)
-    # a scrambled buffer address fails the block-view reconstruction
-    H = HostMatrix(q.A, "f64")
-    scatter_global(q.A, H.buffers(), np.arange(q.A.m * q.A.n, dtype=np.float64).reshape(q.A.m, q.A.n))
-    ij = np.array([(i, j) for i in range(q.A.m) for j in range(q.A.n)])
-    _, buf, off = oracle.locate(q.A, ij)
-    vals = np.array([H.buffer(b)[o] for b, o in zip(buf, off)])
-    assert np.array_equal(vals, np.arange(len(ij), dtype=np.float64))
-    # an off-by-one storage address (a dropped "+ r" term would look alike)
-    size = q.A.bufsize[buf]
-    shifted = np.where(off + 1 < size, off + 1, off - 1)
-    wrong = np.array([H.buffer(b)[o] for b, o in zip(buf, shifted)])
-    assert not np.array_equal(wrong, np.arange(len(ij), dtype=np.float64))
+def _relabel_cases():
+    with open(os.path.join(GOLDEN, "relabel_cases.json")) as f:
+        return json.load(f)
+
+
+def test_cost_W_topology_3x3_by_hand():
+    """W(G_sigma) of every permutation, the COPR optimum (Def. COPR) and the
+    volume-only optimum (Eq. 2) of the hand-worked 3 x 3 case."""
+    g = _relabel_cases()["topology_3x3"]
+    V, lat, bw = np.array(g["V"]), np.array(g["lat"], float), np.array(g["bw"], float)
+    for key, w in g["W"].items():
+        sigma = [int(x) for x in key.split(",")]
+        assert oracle.cost_W(V, lat, bw, sigma) == w, key
+        assert oracle.objective(V, sigma) == g["local"][key], key
+    best, sigma = oracle.copr_bruteforce_cost(V, lat, bw)
+    assert best == g["optimum"] and sigma.tolist() == g["sigma"]
+    vbest, vsig = oracle.lap_bruteforce(V)
+    assert vbest == g["volume_optimum"] and vsig.tolist() == g["volume_sigma"]
+
+
+def test_cost_W_closed_forms():
+    """W(G_sigma) on cases whose totals are derived by hand (golden README)."""
+    g = _relabel_cases()["cost_W_closed_forms"]
+    f = g["all_ones_identity"]
+    for P, want in zip(f["P"], f["values"]):
+        idx = np.arange(P)
+        V = np.ones((P, P), np.int64)
+        lat = 1.0 - np.eye(P)
+        bw = np.abs(idx[:, None] - idx[None, :]).astype(float)
+        assert oracle.cost_W(V, lat, bw, idx) == want == P * (P - 1) + (P ** 3 - P) // 3
+    P = 4
+    idx = np.arange(P)
+    V = np.tile(1 + idx, (P, 1)).astype(np.int64)     # V[i][j] = 1 + j
+    lat = 1.0 - np.eye(P)
+    bw = np.abs(idx[:, None] - idx[None, :]).astype(float)
+    assert oracle.cost_W(V, lat, bw, (idx + 1) % P) == g["shift_4"]["W"]
+    d = g["diagonal_nonzero"]
+    P = d["P"]
+    ones = np.ones((P, P))
+    assert oracle.cost_W(np.ones((P, P), np.int64), ones, ones, np.arange(P)) == d["W"] \
+        == 2 * P * (P - 1)
+
+
+def test_greedy_hand_worked_with_ties():
+    """Sec. 6 greedy: decreasing volume, ties by smaller p then smaller q."""
+    g = _relabel_cases()["greedy_ties_4x4"]
+    V = np.array(g["V"], np.int64)
+    total, sigma = oracle.lap_greedy(V)
+    assert sigma.tolist() == g["greedy_sigma"] and total == g["greedy_local"]
+    assert oracle.lap_bruteforce(V)[0] == g["optimum"]
+
+
+@pytest.mark.parametrize("P", [1, 2, 3, 4, 5, 6, 7])
+def test_copr_reduces_to_volume_relabeling(P):
+    """lat = 0, bw = 1 off the diagonal is the locally-free volume cost
+    (Eq. 2): min W(G_sigma) = total volume - the volume optimum, and the
+    minimizing sigma keeps that optimum (Remark on the gain)."""
+    for s in range(6):
+        V = _rand_V(P, 900 + 10 * P + s, ties=(s % 2 == 0))
+        lat = np.zeros((P, P))
+        bw = 1.0 - np.eye(P)
+        best, sigma = oracle.copr_bruteforce_cost(V, lat, bw)
+        opt, _ = oracle.lap_bruteforce(V)
+        assert best == V.sum() - opt
+        assert oracle.objective(V, sigma) == opt
+
+
+@pytest.mark.parametrize("P", [2, 3, 5, 7])
+def test_copr_latency_only_counts_remote_packages(P):
+    """lat = 1 off the diagonal, bw = 0: W counts the remote non-empty
+    packages, so min W = (non-empty packages) - (largest matching inside
+    the support of V), the matching taken by brute force on V > 0."""
+    for s in range(6):
+        V = _rand_V(P, 700 + 10 * P + s)
+        lat = 1.0 - np.eye(P)
+        bw = np.zeros((P, P))
+        best, _ = oracle.copr_bruteforce_cost(V, lat, bw)
+        match, _ = oracle.lap_bruteforce((V > 0).astype(np.int64))
+        assert best == np.count_nonzero(V) - match
+
+
+# ----------------------------------------------------------------------------
+# planted mistakes: mutated builds of the oracle itself must fail the pins
+# ----------------------------------------------------------------------------
+
+# (name, text in costa_oracle.c, replacement, replace every occurrence)
+MUTANTS = [
+    ("dropped beta term", "{alpha[0], beta[0]}, y[2] = {b[0], a[0]}",
+     "{alpha[0], 0.0}, y[2] = {b[0], a[0]}", False),
+    ("sign of beta", "{alpha[0], beta[0]}, y[2] = {b[0], a[0]}",
+     "{alpha[0], -beta[0]}, y[2] = {b[0], a[0]}", False),
+    ("missing conjugate", "Bbufs[bb], ob, b);\n            if (op == O_C && cplx) b[1] = -b[1];",
+     "Bbufs[bb], ob, b);", False),
+    ("sign of alpha's imaginary part", "double xr[4] = {alpha[0], -alpha[1], beta[0], -beta[1]};",
+     "double xr[4] = {alpha[0], alpha[1], beta[0], -beta[1]};", False),
+    ("product error term dropped", "*e = fma(a, b, -x);", "*e = 0.0;", False),
+    ("beta = 0 reads A", "int beta0 = (beta[0] == 0.0 && beta[1] == 0.0);", "int beta0 = 0;", True),
+    ("off-by-one row offset", "int64_t r = i - L->rsplit[bi], c = j - L->csplit[bj];",
+     "int64_t r = i - L->rsplit[bi] + 1, c = j - L->csplit[bj];", False),
+    ("storage orders swapped", "(L->order[b] == 0 ? r + c * L->ld[b] : r * L->ld[b] + c)",
+     "(L->order[b] == 1 ? r + c * L->ld[b] : r * L->ld[b] + c)", False),
+    ("column block from the row index", "int64_t bj = find_block(L->csplit, L->nbc, j);",
+     "int64_t bj = find_block(L->csplit, L->nbc, i);", False),
+    ("volume indices transposed", "loc[(int64_t)qb * P + qa] += 1;", "loc[(int64_t)qa * P + qb] += 1;",
+     False),
+    ("op ignored in volume", "else oracle_locate(B, j, i, &qb, &bb, &ob);\n                loc",
+     "else oracle_locate(B, i, j, &qb, &bb, &ob);\n                loc", False),
+    ("brute force minimizes", "if (s > best) {", "if (s < best || best == INT64_MIN) {", False),
+    ("subset DP operand transposed", "best[S & ~((size_t)1 << p)] + V[(int64_t)p * P + q];",
+     "best[S & ~((size_t)1 << p)] + V[(int64_t)q * P + p];", False),
+    ("greedy tie rule reversed", "(V[key] == V[a] && key < a)", "(V[key] == V[a] && key > a)", False),
+    ("greedy ascending", "int before = V[key] > V[a] ||", "int before = V[key] < V[a] ||", False),
+    ("cost without latency", "W += lat[(int64_t)i * P + k] + bw", "W += bw", False),
+    ("cost indexed by label", "W += lat[(int64_t)i * P + k] + bw[(int64_t)i * P + k] * (double)v;",
+     "W += lat[(int64_t)i * P + j] + bw[(int64_t)i * P + j] * (double)v;", False),
+    ("empty packages charged", "if (v == 0) continue;\n            int k = sigma[j];",
+     "int k = sigma[j];", False),
+    ("kept packages charged", "if (k == i) continue;\n            W +=", "W +=", False),
+    ("COPR maximizes", "if (first || W < best) {", "if (first || W > best) {", False),
+]
+
+
+def _pins_for(name):
+    """The pins that must catch each mutant (plain calls of the pin tests)."""
+    cases_movement = lambda: [test_pure_movement_matches_numpy_op(c) for c in range(8)]
+    cases_pow2 = lambda: [test_power_of_two_scalars_exact(c) for c in range(40, 52)]
+    return {
+        "dropped beta term": cases_pow2,
+        "sign of beta": cases_pow2,
+        "missing conjugate": lambda: test_conjugate_transpose_round_trip("c128"),
+        "sign of alpha's imaginary part":
+            lambda: test_combine_rounds_exact_value_once("c128", complex(0.2, 0.9), complex(-1.1, 0.4)),
+        "product error term dropped": lambda: test_combine_rounds_exact_value_once("f64", -0.3, 0.7),
+        "beta = 0 reads A": cases_movement,
+        "off-by-one row offset": lambda: test_locate_matches_block_views(21),
+        "storage orders swapped": lambda: test_locate_matches_block_views(21),
+        "column block from the row index": lambda: [test_locate_matches_block_views(c) for c in (21, 8, 30)],
+        "volume indices transposed": lambda: [test_volume_matches_owner_maps(c) for c in range(10)],
+        "op ignored in volume": lambda: [test_volume_matches_owner_maps(c) for c in range(10)],
+        "brute force minimizes": lambda: test_lap_solvers_agree_small(4),
+        "subset DP operand transposed": lambda: test_lap_solvers_agree_small(5),
+        "greedy tie rule reversed": test_greedy_hand_worked_with_ties,
+        "greedy ascending": test_greedy_hand_worked_with_ties,
+        "cost without latency": test_cost_W_closed_forms,
+        "cost indexed by label": test_cost_W_closed_forms,
+        "empty packages charged": test_cost_W_topology_3x3_by_hand,
+        "kept packages charged": test_cost_W_closed_forms,
+        "COPR maximizes": lambda: test_copr_reduces_to_volume_relabeling(4),
+    }[name]
+
+
+@pytest.fixture(scope="module")
+def mutant_libs(tmp_path_factory):
+    from concurrent.futures import ThreadPoolExecutor
+    src = oracle.source_text()
+    d = tmp_path_factory.mktemp("oracle_mutants")
+    jobs = {}
+    for k, (name, old, new, every) in enumerate(MUTANTS):
+        n = src.count(old)
+        assert n >= 1 and (every or n == 1), (name, n)
+        jobs[name] = (src.replace(old, new), str(d / f"mutant{k}.so"))
+    with ThreadPoolExecutor(8) as ex:
+        futs = {name: ex.submit(oracle.compile_variant, text, path)
+                for name, (text, path) in jobs.items()}
+        return {name: f.result() for name, f in futs.items()}
+
+
+@pytest.mark.parametrize("name", [m[0] for m in MUTANTS])
+def test_planted_mistake_fails_a_pin(name, mutant_libs):
+    pin = _pins_for(name)
+    pin()                                   # the pin holds for the real oracle
+    with oracle.loaded(mutant_libs[name]):
+        try:
+            pin()
+        except Exception:
+            return
+    raise AssertionError(f"planted mistake '{name}' passed its pins")
