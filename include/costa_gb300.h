@@ -31,6 +31,14 @@
  *  - Aliasing: A's and B's storage must not overlap; a layout's blocks must
  *    not overlap each other.  Overlap is not detected and gives undefined
  *    results.
+ *  - Arithmetic (Eq. 1): with real alpha and beta each element, or each
+ *    component of a complex element, is fma(alpha, b, beta * a) in the
+ *    element type's precision (alpha * b when beta == 0, b when also
+ *    alpha == 1).  With a complex alpha or beta each component is the
+ *    compensated dot product Dot2 (Ogita, Rump & Oishi 2005) of its 2
+ *    (beta == 0) or 4 products: as if evaluated in twice the precision and
+ *    rounded once.  When beta == 0, A is never read, so NaN or garbage in A
+ *    does not propagate.
  */
 #ifndef COSTA_GB300_H
 #define COSTA_GB300_H

@@ -794,7 +794,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
                 lk.tiles = halves->tiles;
                 lk.ntiles = halves->ntiles;
             }
-            if (kind != K_COPY && kind != K_SCALE) {  // the groups of the kinds that read A
+            if (kind_reads_a(kind)) {  // the groups of the kinds that read A
                 lk.groups = list.groups_a;
                 lk.ngroups = list.ngroups_a;
             }

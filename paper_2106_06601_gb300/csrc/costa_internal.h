@@ -100,14 +100,20 @@ enum : int32_t { SF_BETA0 = 1, SF_ALPHA1 = 2, SF_CPLX = 4, SF_BPOW2 = 8 };
 //   K_COPY  alpha = 1, beta = 0        out = op(b)
 //   K_SCALE real alpha, beta = 0       out = alpha * op(b)
 //   K_AXPBY real alpha, beta != 0      out = fma(alpha, op(b), beta * a)
-//   K_CPLX  complex alpha or beta      complex products as chains of fma
+//   K_CPLX  complex beta (or complex alpha with beta != 0): each component
+//           a compensated sum of its four products (Dot2)
 //   K_AXPBY2 as K_AXPBY with beta = +-2^k: beta * a is formed exactly on the
 //            integer pipes (exponent add), saving one multiply on the scarce
 //            FP64 pipe; same bits as K_AXPBY
-enum : int { K_COPY = 0, K_SCALE = 1, K_AXPBY = 2, K_CPLX = 3, K_AXPBY2 = 4, K_NKINDS = 5 };
+//   K_CSCALE complex alpha, beta = 0   out = alpha * op(b) by Dot2; A is not
+//            read (BLAS convention), so NaN in A does not propagate
+enum : int { K_COPY = 0, K_SCALE = 1, K_AXPBY = 2, K_CPLX = 3, K_AXPBY2 = 4, K_CSCALE = 5, K_NKINDS = 6 };
+
+// The kinds whose output depends on A's old value (beta != 0).
+COSTA_HD constexpr bool kind_reads_a(int kind) { return kind == K_AXPBY || kind == K_CPLX || kind == K_AXPBY2; }
 
 COSTA_HD inline int kind_of(int32_t flags) {
-    if (flags & SF_CPLX) return K_CPLX;
+    if (flags & SF_CPLX) return (flags & SF_BETA0) ? K_CSCALE : K_CPLX;
     if (!(flags & SF_BETA0)) return (flags & SF_BPOW2) ? K_AXPBY2 : K_AXPBY;
     if (!(flags & SF_ALPHA1)) return K_SCALE;
     return K_COPY;

@@ -141,8 +141,8 @@ template <typename T> struct Cfg {
 //    registers and run two blocks without look-ahead.
 // Overridable at build time for tuning.
 template <typename T, int KIND, bool MIS = false> struct KCfg {
-    static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX;
-    static constexpr bool READS_A = KIND != K_COPY && KIND != K_SCALE;
+    static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX || KIND == K_CSCALE;
+    static constexpr bool READS_A = kind_reads_a(KIND);
     static constexpr int WARPS = Cfg<T>::WARPS;
     static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : COSTA_MINB_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
@@ -229,22 +229,61 @@ __device__ __forceinline__ double flip_sign(double v, uint32_t m) {
     return __longlong_as_double(__double_as_longlong(v) ^ (static_cast<unsigned long long>(m) << 32));
 }
 
+// Complex scalars: each component of alpha * b (+ beta * a) is the
+// compensated dot product Dot2 of Ogita, Rump and Oishi ("Accurate sum and
+// dot product", SIAM J. Sci. Comput. 26(6), 2005) over its 2 or 4 products,
+// built on TwoProduct (one fma gives a product's rounding error exactly) and
+// Knuth's TwoSum.  The result lies within u|x| + gamma_n^2 * sum|terms| of
+// the exact component x (u the unit roundoff, n the number of terms): as if
+// computed in twice the working precision and rounded once.  The running sum
+// p is the plain sum of the rounded products; when it is not finite (an
+// infinite or NaN input, an overflow) the error terms are undefined and p
+// itself, the plain IEEE value, is the result.
+__device__ __forceinline__ float addr(float a, float b) { return __fadd_rn(a, b); }
+__device__ __forceinline__ double addr(double a, double b) { return __dadd_rn(a, b); }
+__device__ __forceinline__ float subr(float a, float b) { return __fsub_rn(a, b); }
+__device__ __forceinline__ double subr(double a, double b) { return __dsub_rn(a, b); }
+
+template <typename R> struct Dot2 {
+    R p, s;  // running sum of the rounded products; sum of the error terms
+    __device__ __forceinline__ Dot2(R x, R y) {
+        p = mulr(x, y);
+        s = fmar(x, y, -p);
+    }
+    __device__ __forceinline__ void add(R x, R y) {
+        const R h = mulr(x, y);
+        const R r = fmar(x, y, -h);  // x * y = h + r exactly
+        const R t = addr(p, h);
+        const R z = subr(t, p);
+        const R q = addr(subr(p, subr(t, z)), subr(h, z));  // p + h = t + q exactly
+        p = t;
+        s = addr(s, addr(q, r));
+    }
+    __device__ __forceinline__ R result() const { return isfinite(p) ? addr(p, s) : p; }
+};
+
 template <int KIND, typename C, typename R>
 __device__ __forceinline__ C combine_c(C b, C a, const Sc &s) {
     b.y = flip_sign(b.y, s.conj_mask);
     C o;
-    if (KIND != K_CPLX) {
+    if (KIND != K_CPLX && KIND != K_CSCALE) {
         o.x = comb_real<KIND, R>(b.x, a.x, s);
         o.y = comb_real<KIND, R>(b.y, a.y, s);
         return o;
     }
-    const R ar = R(s.ar), ai = R(s.ai), br = R(s.br), bi = R(s.bi);
-    R t = fmar(br, a.x, -mulr(bi, a.y));
-    t = fmar(-ai, b.y, t);
-    o.x = fmar(ar, b.x, t);
-    R w = fmar(br, a.y, mulr(bi, a.x));
-    w = fmar(ai, b.x, w);
-    o.y = fmar(ar, b.y, w);
+    const R ar = R(s.ar), ai = R(s.ai);
+    Dot2<R> re(ar, b.x), im(ar, b.y);
+    re.add(-ai, b.y);
+    im.add(ai, b.x);
+    if (KIND == K_CPLX) {
+        const R br = R(s.br), bi = R(s.bi);
+        re.add(br, a.x);
+        re.add(-bi, a.y);
+        im.add(br, a.y);
+        im.add(bi, a.x);
+    }
+    o.x = re.result();
+    o.y = im.result();
     return o;
 }
 template <int KIND>
@@ -398,7 +437,7 @@ template <typename T, int KIND>
 __device__ __forceinline__ void load_a(const Geom<T> &g, const Sc &s, Chunk<T> (&av)[Cfg<T>::NPASS],
                                        int lane) {
     using C = Cfg<T>;
-    if (KIND == K_COPY || KIND == K_SCALE) return;
+    if (!kind_reads_a(KIND)) return;
     const int chunks = g.nx / C::VEC;
     const LaneMap m = lane_map(chunks, lane);
     const int x0 = m.c * C::VEC;
@@ -469,7 +508,7 @@ template <int KIND> __device__ __forceinline__ double2 premul(double2 a, const S
 template <typename T, int KIND>
 __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
     using C = Cfg<T>;
-    constexpr bool READ_A = KIND != K_COPY && KIND != K_SCALE;
+    constexpr bool READ_A = kind_reads_a(KIND);
     T *sm = reinterpret_cast<T *>(buf);
     const int n = g.nx * g.ny;
     if (!g.transpose) {
@@ -624,7 +663,7 @@ __device__ __forceinline__ void drain_window(const Geom<T> &g, const Sc &s, unsi
 template <typename T, int KIND>
 __device__ __forceinline__ void stage_drain_w(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
     using C = Cfg<T>;
-    static_assert(KIND == K_COPY || KIND == K_SCALE, "the window path does not read A");
+    static_assert(!kind_reads_a(KIND), "the window path does not read A");
     const int cm = wmain<T>(g.nx);
     const LaneMap m = lane_map(cm, lane);
     const int x0 = m.c * C::VEC - phase<T>(g.dst, g.dld, m.r0);  // first tile column of the lane's chunk
@@ -674,7 +713,7 @@ template <typename T> __device__ __forceinline__ T &elem(Chunk<T> (&av)[Cfg<T>::
 template <typename T, int KIND>
 __device__ __forceinline__ void load_a_e(const Geom<T> &g, const Sc &s, Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
     using C = Cfg<T>;
-    if (KIND == K_COPY || KIND == K_SCALE) return;
+    if (!kind_reads_a(KIND)) return;
     constexpr int NE = C::NPASS * C::VEC;  // elements per lane, full tile
     const LaneMap m = lane_map(g.nx, lane);
     const bool on = m.c < g.nx;
@@ -1160,7 +1199,8 @@ cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     return e;
 }
 
-// Kernel for (element type, combine kind).  Real types never take K_CPLX.
+// Kernel for (element type, combine kind).  Real types never take K_CPLX or
+// K_CSCALE.
 template <typename T>
 cudaError_t launch_remap_t(const RemapLaunch &a, int kind, cudaStream_t st) {
     switch (kind) {
@@ -1168,8 +1208,13 @@ cudaError_t launch_remap_t(const RemapLaunch &a, int kind, cudaStream_t st) {
     case K_SCALE: return launch_t<T, K_SCALE>(a, st);
     case K_AXPBY: return launch_t<T, K_AXPBY>(a, st);
     case K_AXPBY2: return launch_t<T, K_AXPBY2>(a, st);
-    default:
+    case K_CPLX:
         if constexpr (ET<T>::CPLX) return launch_t<T, K_CPLX>(a, st);
+        return cudaErrorInvalidValue;
+    case K_CSCALE:
+        if constexpr (ET<T>::CPLX) return launch_t<T, K_CSCALE>(a, st);
+        return cudaErrorInvalidValue;
+    default:
         return cudaErrorInvalidValue;
     }
 }

@@ -320,3 +320,86 @@ def test_misaligned_runs(dtype, op, dev):
             p = C.Problem("misaligned", dtype, op, alpha, beta, A, B, "uniform",
                           "nan" if beta == 0 else "uniform", C.SEED0 + 11 + k)
             check_problem(p, dev, guard=guard)
+
+
+def _complex_layouts(op):
+    """Aligned multi-tile grid with a ragged tail, odd leading dimensions
+    (misaligned runs) and 8 x 8 blocks (the small-tile kernel)."""
+    m, n = 150, 171
+    am, an = (m, n) if op == "N" else (n, m)
+    yield L.block_cyclic(m, n, 40, 24, 2, 3), L.block_cyclic(am, an, 33, 64, 3, 2, grid_order="C")
+    yield (L.block_cyclic(m, n, 13, 37, 2, 3, storage="R", ld_pad=1),
+           L.block_cyclic(am, an, 29, 7, 3, 2, ld_pad=3))
+    yield L.block_cyclic(m, n, 8, 8, 2, 3), L.block_cyclic(am, an, 8, 8, 3, 2, grid_order="C")
+
+
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("op", ["N", "T", "C"])
+@pytest.mark.parametrize("alpha,beta", [(complex(-0.6, 0.3), 0.0),
+                                        (complex(0.5, -0.75), 1.0),
+                                        (1.0, complex(0.25, 2.0)),
+                                        (complex(0.2, 0.9), complex(-1.1, 0.4))])
+def test_complex_scalars_within_2ulp(dtype, op, alpha, beta, dev):
+    """Complex scalars: each component within 2 ulp(M) of the oracle, M the
+    largest of its product terms and of the oracle's value (tests/_util
+    tolerance).  A third of A's elements are set to -alpha op(B) / beta, so
+    the two halves of each component cancel.  With beta = 0, A is pre-filled
+    with NaN and must not be read."""
+    from tests._util import global_matrix, max_ulps, op_apply, scatter_global
+    for k, (B, A) in enumerate(_complex_layouts(op)):
+        p = C.Problem("cplx", dtype, op, alpha, beta, A, B, "uniform",
+                      "nan" if beta == 0 else "uniform", C.SEED0 + 40 + k)
+        g = OnDevice(p, dev, guard=2)
+        try:
+            if beta != 0:
+                al, be = oracle.scalar(dtype, alpha), oracle.scalar(dtype, beta)
+                X = op_apply(op, global_matrix(p.B, g.Bh.buffers())).astype(np.complex128)
+                G = global_matrix(p.A, g.Ah.buffers())
+                sel = (np.arange(G.size).reshape(G.shape) % 3) == 0
+                G[sel] = (-(al * X) / be)[sel].astype(G.dtype)
+                scatter_global(p.A, g.Ah.buffers(), G)
+                g.Ad.upload(g.Ah)
+            g.run()
+            got, want = g.Ad.download(), g.oracle_result()
+            compare(p, got, want, g.Ah, g.Bh)
+            assert np.array_equal(g.Bd.download().arena, g.Bh.arena, equal_nan=True)
+            if beta == 0:
+                assert not np.isnan(global_matrix(p.A, got.buffers())).any()
+            al, be = oracle.scalar(dtype, alpha), oracle.scalar(dtype, beta)
+            X = op_apply(op, global_matrix(p.B, g.Bh.buffers()))
+            worst = max_ulps(dtype, global_matrix(p.A, got.buffers()),
+                             global_matrix(p.A, want.buffers()), al, be, X,
+                             global_matrix(p.A, g.Ah.buffers()))
+            assert worst <= 2.0, worst
+        finally:
+            g.close()
+
+
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("alpha,beta", [(complex(-0.6, 0.3), 0.0), (complex(0.2, 0.9), complex(-1.1, 0.4))])
+def test_special_values_complex_scalars(dtype, alpha, beta, dev):
+    """Zeros, subnormals, infinities and NaNs with complex scalars: where the
+    plain sum of the rounded products is not finite, both sides return that
+    plain IEEE value; elsewhere the 2 ulp(M) bound holds.  (Magnitudes stay
+    below max/16, so that no product or partial sum overflows.)"""
+    rng = np.random.default_rng(9)
+    B = L.block_cyclic(64, 48, 16, 16, 2, 2)
+    A = L.block_cyclic(48, 64, 8, 32, 2, 2)
+    p = C.Problem("special-c", dtype, "C", alpha, beta, A, B, "uniform", "uniform", C.SEED0)
+    g = OnDevice(p, dev)
+    try:
+        real = np.float64 if dtype == "c128" else np.float32
+        fi = np.finfo(real)
+        specials = np.array([0.0, -0.0, fi.tiny, -fi.tiny, fi.tiny / 4, -fi.smallest_subnormal,
+                             fi.max / 16, -fi.max / 32, np.inf, -np.inf, np.nan, 1.5, -3.0],
+                            dtype=real)
+        for h in (g.Ah, g.Bh):
+            v = h.arena.view(real)
+            idx = rng.integers(0, v.size, v.size // 4)
+            v[idx] = specials[rng.integers(0, specials.size, idx.size)]
+        g.Bd.upload(g.Bh)
+        g.Ad.upload(g.Ah)
+        g.run(relabel=False)
+        compare(p, g.Ad.download(), g.oracle_result(), g.Ah, g.Bh)
+    finally:
+        g.close()
