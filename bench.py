@@ -1,20 +1,23 @@
 """Benchmark of the reshuffle A = alpha * op(B) + beta * A on GB300.
 
-Default workload (the metric's configuration): 8192 x 8192 f64, B block-cyclic
-64x64 on a 4x4 grid -> A block-cyclic 128x128 on a 4x4 grid with a seeded
-rank permutation, op = T, alpha = 2, beta = 0.5, P = 16 virtual ranks,
-relabeling on.  One step = one costa_transform call (direct mode) through the
-C ABI; its plan (overlay, volume kernel, relabeling, tile lists) is built once
-before the timed region and reported separately, like a reused transformer.
+Headline workload: c5, the largest single-GPU configuration (12.9 GB moved per
+call): B 131072 x 4096 f64 normal(0, 1), block-cyclic 32x32 on a 16x16 grid ->
+A 4096 x 131072 in 256 row panels of 16 rows (a COSMA-style blocked layout,
+one panel per rank), op = T, alpha = beta = 1, P = 256 virtual ranks,
+relabeling on.  The same line carries c2, c3 and c4 under `per_config`, each
+with the headline's fields.  One step = one costa_transform (or
+costa_transform_batched) call in direct mode through the C ABI; its plan
+(overlay, volume kernel, relabeling, tile lists) is built once before the
+timed region and reported separately, like a reused transformer.
 
 Prints one JSON line.  `value` = algorithmic bytes (read B + read A if
 beta != 0 + write A) of all ranks / max-over-ranks device time.  `e2e` = the
-same metric through the same call with the inputs in pinned host memory:
-every step copies B (and A when beta != 0) host->device, transforms, and
-copies A back.
+same metric through the same call with the matrices in pinned host memory
+(the kernels read and write them over the host link), and under `copies`
+with explicit host->device and device->host copies around the call.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2|c3|c4|c5|c1]
-                  [--mode direct|message] [--impl gb300|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5|c2|c3|c4|c1|...]
+                  [--also c2,c3,c4|none] [--mode direct|message] [--impl gb300|reference]
 
 Multi-GPU (torchrun): one independent replica per GPU (the reshuffle of one
 problem uses one GPU here), scaling "weak".
@@ -54,9 +57,12 @@ KERNEL_SOURCES = ["paper_2106_06601_gb300/csrc/remap_impl.cuh",
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--workload", default="c2", choices=list(C.CONFIGS) + list(C.EXTRA_WORKLOADS))
+    ap.add_argument("--workload", default="c5", choices=list(C.CONFIGS) + list(C.EXTRA_WORKLOADS))
+    ap.add_argument("--also", default="auto",
+                    help="comma-separated workloads measured after the headline and reported "
+                         "under per_config ('auto': c2,c3,c4 when the headline is c5; 'none')")
     ap.add_argument("--mode", default="direct", choices=["direct", "message"])
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=20)
@@ -214,13 +220,13 @@ def algorithmic_bytes(probs) -> int:
     return sum(p.algorithmic_bytes() for p in probs)
 
 
-def run_gpu(args, rank, world, local_rank):
+def run_gpu(args, workload, rank, world, local_rank):
     import torch
     import paper_2106_06601_gb300 as costa
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    probs = problems(args.workload, args.small)
+    probs = problems(workload, args.small)
     mats = []
     for p in probs:
         Bd = DeviceMatrix(p.B, p.dtype, dev).fill(p.b_kind, p.seed, p.src_stream)
@@ -303,7 +309,7 @@ def run_gpu(args, rank, world, local_rank):
     peak, peak_kind = measured_peaks()
     avg_launch_ms = statistics.mean(per)
     achieved = nbytes / (avg_launch_ms * 1e-3) / 1e9
-    traffic = recorded_traffic(args.workload) if args.mode == "direct" else None
+    traffic = recorded_traffic(workload) if args.mode == "direct" else None
     return dict(value=value, ms_per_step=ms_per_step, total_ms=total_ms, per=per,
                 launches=launches, clocks=clk, e2e=e2e, plan_s=plan_s, stats=stats,
                 nbytes=nbytes, achieved=achieved, peak=peak, peak_kind=peak_kind,
@@ -490,7 +496,7 @@ def cpu_model() -> str:
     return platform.machine()
 
 
-def run_cpu_oracle(args, probs, seconds_target: float, threads: int | None = None):
+def run_cpu_oracle(probs, seconds_target: float, threads: int | None = None):
     """The oracle, as it stands, on a bounded row slab of the first instance
     (the same layouts and values); returns (GB/s, threads, description)."""
     import oracle
@@ -524,13 +530,13 @@ def run_cpu_oracle(args, probs, seconds_target: float, threads: int | None = Non
     return gbs, threads, desc, rows2, dt2
 
 
-def workload_config(args, probs, world):
+def workload_config(args, workload, probs, world):
     p = probs[0]
     nbytes = algorithmic_bytes(probs)
-    text = C.WORKLOAD_TEXT[args.workload]
+    text = C.WORKLOAD_TEXT[workload]
     if args.small:
-        text = f"{args.workload} layouts at reduced size ({p.A.m}x{p.A.n} per instance)"
-    return {"workload": f"{args.workload}: {text}",
+        text = f"{workload} layouts at reduced size ({p.A.m}x{p.A.n} per instance)"
+    return {"workload": f"{workload}: {text}",
             "dtype": p.dtype, "op": p.op, "alpha": str(p.alpha), "beta": str(p.beta),
             "P": p.A.nranks, "instances": len(probs), "relabel": True, "mode": args.mode,
             "bytes_per_step_per_gpu": nbytes,
@@ -539,86 +545,127 @@ def workload_config(args, probs, world):
             "parallelism": f"replicas x{world}"}
 
 
+METRIC = "reshuffle GB/s and % of GB300 HBM peak for A=alpha*op(B)+beta*A, 1 GPU"
+
+
+def also_list(args):
+    if args.also == "none":
+        return []
+    if args.also == "auto":
+        return ["c2", "c3", "c4"] if args.workload == "c5" and not args.small else []
+    names = [w for w in args.also.split(",") if w and w != args.workload]
+    for w in names:
+        if w not in C.CONFIGS and w not in C.EXTRA_WORKLOADS:
+            raise SystemExit(f"unknown workload {w}")
+    return names
+
+
+def reference_arm(args, probs):
+    """The oracle, as it stands, on the host cores: each step a bounded row
+    slab of the headline workload (the same layouts and values)."""
+    steps, warmup = max(1, args.steps), max(0, args.warmup)
+    # each step sized so that the whole run stays within a few minutes
+    per_step = max(0.5, min(10.0, 150.0 / (steps + warmup)))
+    import oracle
+    threads = oracle.default_threads()
+    gbs, threads, desc, rows, dt = run_cpu_oracle(probs, per_step)
+    p = probs[0]
+    per_row_bytes = p.A.n * p.esize * (3 if p.beta != 0 else 2)
+    Bh = HostMatrix(p.B, p.dtype).fill(p.b_kind, p.seed, p.src_stream)
+    Ah = HostMatrix(p.A, p.dtype).fill(p.a_kind, p.seed, p.tgt_stream)
+    for _ in range(warmup):
+        oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
+                         Bh.buffers(), rows=(0, rows), threads=threads)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
+                         Bh.buffers(), rows=(0, rows), threads=threads)
+    dt = time.perf_counter() - t0
+    value = rows * per_row_bytes * steps / dt / 1e9
+    return {
+        "impl": "reference", "metric": METRIC,
+        "value": round(value, 4), "unit": "GB/s", "n_gpus": args.gpus, "steps": steps,
+        "warmup": warmup, "ms_per_step": round(dt / steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": p.dtype, "data": "synthetic (seeded counter-based generator)",
+        "config": workload_config(args, args.workload, probs, 1),
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads,
+                         "kind": "oracle", "sample": f"each step: {desc.split(',')[0]}",
+                         "cpu_model": cpu_model()},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0}}
+
+
+def measure(args, workload, rank, world, local_rank):
+    """One workload on this rank's GPU; on rank 0 the fields of its JSON
+    entry (None elsewhere)."""
+    import gc
+    import torch
+    probs = problems(workload, args.small)
+    r = run_gpu(args, workload, rank, world, local_rank)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        gbs, threads, desc, _, _ = run_cpu_oracle(probs, args.cpu_seconds)
+        cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+               "sample": desc, "cpu_model": cpu_model()}
+        if workload in ("c1", "c2"):  # the single-threaded figure as well
+            gbs1, _, desc1, _, _ = run_cpu_oracle(probs, min(3.0, args.cpu_seconds), threads=1)
+            cpu["single_thread"] = {"value": round(gbs1, 4), "unit": "GB/s", "sample": desc1}
+    gc.collect()
+    torch.cuda.empty_cache()
+    if rank != 0:
+        return None
+    st = r["stats"]
+    out = {
+        "value": round(r["value"], 3), "unit": "GB/s",
+        "ms_per_step": round(r["ms_per_step"], 5), "dtype": probs[0].dtype,
+        "config": workload_config(args, workload, probs, world),
+        "elements_per_s": round(sum(p.A.m * p.A.n for p in probs) * world / (r["ms_per_step"] * 1e-3), 1),
+        "pct_of_hbm_peak": {"measured": round(100 * r["value"] / world / r["peak"], 2),
+                            "nominal_8TBs": round(100 * r["value"] / world / 8000.0, 2)},
+        "roofline": roofline(args, r),
+        "plan": {"ms": round(r["plan_s"] * 1e3, 2), "volume_ms": round(st["volume_ms"], 3),
+                 "relabel_ms": round(st["relabel_ms"], 3), "cells": st["n_cells"],
+                 "tiles": st["n_tiles"], "total_volume": st["total_volume"],
+                 "local_identity": st["local_identity"],
+                 "local_relabeled": st["local_relabeled"],
+                 "staging_bytes": st["staging_bytes"]},
+        "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
+        "cpu_baseline": cpu,
+    }
+    if r["phases"] is not None:
+        out["message_phases"] = r["phases"]
+    return out
+
+
 def main():
     args = parse()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    probs = problems(args.workload, args.small)
 
     if args.impl == "reference":
         if rank != 0:
             return
-        steps, warmup = max(1, args.steps), max(0, args.warmup)
-        # each step: the oracle on a bounded sample sized so the whole run
-        # stays within a few minutes
-        per_step = max(0.5, min(10.0, 150.0 / (steps + warmup)))
-        import oracle
-        threads = oracle.default_threads()
-        gbs, threads, desc, rows, dt = run_cpu_oracle(args, probs, per_step)
-        p = probs[0]
-        per_row_bytes = p.A.n * p.esize * (3 if p.beta != 0 else 2)
-        Bh = HostMatrix(p.B, p.dtype).fill(p.b_kind, p.seed, p.src_stream)
-        Ah = HostMatrix(p.A, p.dtype).fill(p.a_kind, p.seed, p.tgt_stream)
-        for _ in range(warmup):
-            oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
-                             Bh.buffers(), rows=(0, rows), threads=threads)
-        t0 = time.perf_counter()
-        for _ in range(steps):
-            oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
-                             Bh.buffers(), rows=(0, rows), threads=threads)
-        dt = time.perf_counter() - t0
-        value = rows * per_row_bytes * steps / dt / 1e9
-        print(json.dumps({
-            "impl": "reference", "metric": "reshuffle GB/s (A = alpha*op(B) + beta*A)",
-            "value": round(value, 4), "unit": "GB/s", "n_gpus": args.gpus, "steps": steps,
-            "warmup": warmup, "ms_per_step": round(dt / steps * 1e3, 3),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": p.dtype, "data": "synthetic (seeded counter-based generator)",
-            "config": workload_config(args, probs, 1),
-            "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads,
-                             "kind": "oracle", "sample": f"each step: {desc.split(',')[0]}"},
-            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
-                    "d2h_bytes_per_step": 0}}), flush=True)
+        print(json.dumps(reference_arm(args, problems(args.workload, args.small))), flush=True)
         return
 
     import torch
     if world > 1:
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    r = run_gpu(args, rank, world, local_rank)
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        gbs, threads, desc, _, _ = run_cpu_oracle(args, probs, args.cpu_seconds)
-        cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
-               "sample": desc, "cpu_model": cpu_model()}
-        if args.workload in ("c1", "c2"):  # the single-threaded figure as well
-            gbs1, _, desc1, _, _ = run_cpu_oracle(args, probs, min(3.0, args.cpu_seconds), threads=1)
-            cpu["single_thread"] = {"value": round(gbs1, 4), "unit": "GB/s", "sample": desc1}
+    head = measure(args, args.workload, rank, world, local_rank)
+    others = {w: measure(args, w, rank, world, local_rank) for w in also_list(args)}
     if rank == 0:
-        st = r["stats"]
-        out = {
-            "metric": "reshuffle GB/s (A = alpha*op(B) + beta*A), % of GB300 HBM peak",
-            "value": round(r["value"], 3), "unit": "GB/s", "n_gpus": world,
-            "steps": args.steps, "warmup": max(3, args.warmup),
-            "ms_per_step": round(r["ms_per_step"], 5), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": probs[0].dtype,
-            "data": "synthetic (seeded counter-based generator, values per the workload)",
-            "config": workload_config(args, probs, world),
-            "elements_per_s": round(sum(p.A.m * p.A.n for p in probs) * world / (r["ms_per_step"] * 1e-3), 1),
-            "pct_of_hbm_peak": {"measured": round(100 * r["value"] / world / r["peak"], 2),
-                                "nominal_8TBs": round(100 * r["value"] / world / 8000.0, 2)},
-            "roofline": roofline(args, r),
-            "plan": {"ms": round(r["plan_s"] * 1e3, 2), "volume_ms": round(st["volume_ms"], 3),
-                     "relabel_ms": round(st["relabel_ms"], 3), "cells": st["n_cells"],
-                     "tiles": st["n_tiles"], "total_volume": st["total_volume"],
-                     "local_identity": st["local_identity"],
-                     "local_relabeled": st["local_relabeled"],
-                     "staging_bytes": st["staging_bytes"]},
-            "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
-            "cpu_baseline": cpu,
-        }
-        if r["phases"] is not None:
-            out["message_phases"] = r["phases"]
+        out = {"metric": METRIC, "value": head.pop("value"), "unit": head.pop("unit"),
+               "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
+               "ms_per_step": head.pop("ms_per_step"), "higher_is_better": True,
+               "scaling": "weak", "vs_baseline": None, "dtype": head.pop("dtype"),
+               "data": "synthetic (seeded counter-based generator, values per the workload)"}
+        out.update(head)
+        if others:
+            for o in others.values():
+                o["steps"] = args.steps
+            out["per_config"] = others
         print(json.dumps(out), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
