@@ -28,6 +28,16 @@
  *    costa_plan_stats) and caches it.  Building a plan synchronizes `stream`.
  *    Plans are freed when one of their layouts is destroyed or by
  *    costa_release_plans().
+ *  - Concurrency: every call on one layout pair (A, B) uses the same cached
+ *    plan.  The calls that use its device scratch (message mode's staging
+ *    buffer; the per-problem scalars of a batch whose scalars differ) run
+ *    one after another in call order: a call on another stream than the
+ *    previous such call makes its stream wait for that call's completion
+ *    event.  Other calls on one pair are not ordered by the library; they
+ *    write the same A, so the caller orders them.  Under stream capture the
+ *    library adds no wait: the caller orders captured work.  The library's
+ *    host state is guarded by one mutex, so calls may come from several
+ *    host threads.
  *  - Aliasing: A's and B's storage must not overlap; a layout's blocks must
  *    not overlap each other.  Overlap is not detected and gives undefined
  *    results.
@@ -347,13 +357,17 @@ costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op
  *    arrays (8 bytes per split, 4 per block of A and of B, each section
  *    rounded up to 256 bytes); more than 4 MiB is rejected with
  *    COSTA_ERR_INVALID_ARG and a message giving both sizes.
- *  - Set-up: the first call on a device, with that device current, looks up
- *    the array's device address (cudaGetSymbolAddress).  Make that first call
- *    before any stream capture.
+ *  - Set-up: every call, with the calling device current, looks up the
+ *    array's device address (cudaGetSymbolAddress, which allocates
+ *    nothing), so the address stays valid when the device's context is
+ *    created again (after cudaDeviceReset).  The first lookup on a device
+ *    may load the library's device code: make the first call before any
+ *    stream capture.
  *  - Sharing: every call uses the same array, which keeps the last call's
  *    contents (V is zeroed on the stream at the start of each call).  Calls
  *    that overlap on the GPU would race; this entry point is synchronous and
- *    serializes its own calls, so they do not overlap within one process.
+ *    serializes its own calls (also on its error paths, which wait for the
+ *    work already queued), so they do not overlap within one process.
  *  - Synchronization: runs on `stream` and synchronizes it before returning.
  * V: host array of P * P int64, as in costa_volume.  Errors: INVALID_ARG,
  * SHAPE, DTYPE, CUDA. */

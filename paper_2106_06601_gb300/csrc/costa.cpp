@@ -138,6 +138,13 @@ struct Plan {
     std::vector<int> sigma;      // optimal relabeling
     costa_plan_stats stats{};
     MessageData msg[2];          // [relabel]
+    // Calls that use the plan's device scratch (message mode's staging, the
+    // per-problem scalars of a batch) run one after another in call order:
+    // a call on another stream than the previous such call first makes its
+    // stream wait for that call's completion event.
+    cudaEvent_t scratch_done = nullptr;
+    cudaStream_t scratch_stream = nullptr;
+    bool scratch_used = false;
 
     ~Plan() {
         for (auto &m : msg) {
@@ -145,8 +152,43 @@ struct Plan {
             if (m.d_staging) cudaFree(m.d_staging);
         }
         if (d_mem) cudaFree(d_mem);
+        if (scratch_done) cudaEventDestroy(scratch_done);
     }
 };
+
+// Orders a call that uses `plan`'s device scratch after the previous such
+// call (see Plan::scratch_done).  Under stream capture nothing is added:
+// the caller orders captured work itself.  `capturing` is set for
+// scratch_release.
+costa_status scratch_acquire(Plan &plan, cudaStream_t stream, bool &capturing) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaError_t ce = cudaStreamIsCapturing(stream, &cs);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaStreamIsCapturing");
+    capturing = cs != cudaStreamCaptureStatusNone;
+    if (capturing) return COSTA_OK;
+    if (!plan.scratch_done) {
+        ce = cudaEventCreateWithFlags(&plan.scratch_done, cudaEventDisableTiming);
+        if (ce != cudaSuccess) {
+            plan.scratch_done = nullptr;
+            return cuda_fail(ce, "cudaEventCreate");
+        }
+    }
+    if (plan.scratch_used && plan.scratch_stream != stream) {
+        ce = cudaStreamWaitEvent(stream, plan.scratch_done, 0);
+        if (ce != cudaSuccess) return cuda_fail(ce, "cudaStreamWaitEvent");
+    }
+    return COSTA_OK;
+}
+
+// Marks the end of a call that used the plan's scratch on `stream`.
+costa_status scratch_release(Plan &plan, cudaStream_t stream, bool capturing) {
+    if (capturing) return COSTA_OK;
+    cudaError_t ce = cudaEventRecord(plan.scratch_done, stream);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaEventRecord");
+    plan.scratch_used = true;
+    plan.scratch_stream = stream;
+    return COSTA_OK;
+}
 
 std::mutex g_mu;
 std::map<std::vector<uint64_t>, std::unique_ptr<Plan>> g_plans;
@@ -761,6 +803,17 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         sc[k] = make_scalars(plan->dtype, alphas, betas, k);
         if (!same_scalars(sc[k], sc[0])) uniform = false;
     }
+    // the calls that use the plan's scratch are ordered (Plan::scratch_done)
+    const bool uses_scratch = !uniform || mode == COSTA_MODE_MESSAGE;
+    bool capturing = false;
+    if (uses_scratch) {
+        s = scratch_acquire(*plan, stream, capturing);
+        if (s != COSTA_OK) return s;
+    }
+    auto done = [&](costa_status st) -> costa_status {
+        if (st != COSTA_OK || !uses_scratch) return st;
+        return scratch_release(*plan, stream, capturing);
+    };
     if (!uniform) {
         bool same = plan->cached_scalars.size() == sc.size();
         for (int k = 0; same && k < n; ++k) same = same_scalars(sc[k], plan->cached_scalars[k]);
@@ -769,7 +822,10 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
             // stream order places it after earlier kernels of this stream
             cudaError_t ce = cudaMemcpyAsync(plan->d_scalars, sc.data(), sizeof(Scalars) * n,
                                              cudaMemcpyHostToDevice, stream);
-            if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpyAsync(scalars)");
+            if (ce != cudaSuccess) {
+                plan->cached_scalars.clear();
+                return cuda_fail(ce, "cudaMemcpyAsync(scalars)");
+            }
             plan->cached_scalars = sc;
         }
         L.per_problem = plan->d_scalars;
@@ -810,7 +866,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         if (ce == cudaSuccess) ce = mark(1);
         if (ce != cudaSuccess) return cuda_fail(ce, "remap kernel launch");
         if (timer) timer->nphases = 1;
-        return COSTA_OK;
+        return done(COSTA_OK);
     }
     s = ensure_message(*plan, relabel != 0);
     if (s != COSTA_OK) return s;
@@ -841,7 +897,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     if (ce == cudaSuccess) ce = mark(3);
     if (ce != cudaSuccess) return cuda_fail(ce, "unpack kernel launch");
     if (timer) timer->nphases = 3;
-    return COSTA_OK;
+    return done(COSTA_OK);
 }
 
 costa_status create_layout(costa_layout *out, int dt, int nranks, int nbr, const int64_t *R, int nbc,
