@@ -11,8 +11,11 @@
 // loads the library holds until the process exits.
 //
 // Host code must not use the array's name as a device address (on the host
-// it names a stand-in); the address comes from cudaGetSymbolAddress, taken
-// once per device, with that device current, on the first call made on it.
+// it names a stand-in); the address comes from cudaGetSymbolAddress, looked
+// up by every call with the calling device current.  The lookup allocates
+// nothing, and a fresh lookup stays right when the device's context has
+// been created again (after cudaDeviceReset), which a cached address would
+// not.
 //
 // Unlike costa_volume it builds no plan: one thread block per block of A
 // finds, by binary search, the blocks of op(B) that overlap it, and its
@@ -29,12 +32,10 @@ namespace costa {
 namespace {
 
 constexpr size_t kScratchBytes = size_t(4) << 20;  // 4 MiB
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
 std::mutex g_noalloc_mu;
-void *g_scratch_addr[kMaxDevices] = {};
 
 // Last index k in [0, nb) with split[k] <= x (the block holding x; blocks
 // that are empty share their start with the next one and are skipped).
@@ -82,6 +83,14 @@ costa_status cuda_error(cudaError_t e, const char *what) {
     return report_error(COSTA_ERR_CUDA, msg);
 }
 
+// An error after work was queued on `st`: wait for that work first, so that
+// the next call (which may use another stream) cannot overlap it in the
+// shared array; the wait's own status is not reported over the first error.
+costa_status cuda_error_queued(cudaError_t e, const char *what, cudaStream_t st) {
+    (void)cudaStreamSynchronize(st);
+    return cuda_error(e, what);
+}
+
 }  // namespace
 }  // namespace costa
 
@@ -118,18 +127,11 @@ extern "C" costa_status costa_volume_noalloc(costa_layout A, costa_layout B, cos
     }
 
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
-    if (dev < 0 || dev >= kMaxDevices)
-        return report_error(COSTA_ERR_INVALID_ARG, "costa_volume_noalloc: device index out of range");
-    if (!g_scratch_addr[dev]) {  // set-up: once per device, with that device current
-        void *addr = nullptr;
-        e = cudaGetSymbolAddress(&addr, g_noalloc_scratch);
-        if (e != cudaSuccess) return cuda_error(e, "cudaGetSymbolAddress");
-        g_scratch_addr[dev] = addr;
-    }
-    char *base = static_cast<char *>(g_scratch_addr[dev]);
+    // the array's address on the current device (in its current context)
+    void *addr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&addr, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_error(e, "cudaGetSymbolAddress");
+    char *base = static_cast<char *>(addr);
     cudaStream_t st = static_cast<cudaStream_t>(stream_v);
     unsigned long long *dV = reinterpret_cast<unsigned long long *>(base + oV);
 
@@ -147,7 +149,7 @@ extern "C" costa_status costa_volume_noalloc(costa_layout A, costa_layout B, cos
     for (const Up &u : ups) {
         if (!u.bytes) continue;
         e = cudaMemcpyAsync(base + u.off, u.src, u.bytes, cudaMemcpyHostToDevice, st);
-        if (e != cudaSuccess) return cuda_error(e, "cudaMemcpyAsync");
+        if (e != cudaSuccess) return cuda_error_queued(e, "cudaMemcpyAsync", st);
     }
     if (nblkA > 0) {
         volume_noalloc_kernel<<<static_cast<unsigned>(nblkA), 128, 0, st>>>(
@@ -158,10 +160,10 @@ extern "C" costa_status costa_volume_noalloc(costa_layout A, costa_layout B, cos
             reinterpret_cast<const int32_t *>(base + oOB), B->nbc, tr ? 1 : 0, P, dV);
         count_launch();
         e = cudaGetLastError();
-        if (e != cudaSuccess) return cuda_error(e, "kernel launch");
+        if (e != cudaSuccess) return cuda_error_queued(e, "kernel launch", st);
     }
     e = cudaMemcpyAsync(V, dV, sizeof(int64_t) * P * P, cudaMemcpyDeviceToHost, st);
-    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpyAsync(V)");
+    if (e != cudaSuccess) return cuda_error_queued(e, "cudaMemcpyAsync(V)", st);
     e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return cuda_error(e, "volume kernel");
     return COSTA_OK;
