@@ -127,10 +127,13 @@ def test_window_map(es):
 
 
 def replay_elements(es, rnd):
-    """The one-element-per-lane path: every staged element lands in the
-    TS x TS buffer at c ^ (r mod TS) of its row, is read back by the lane
-    that writes its target element, and every target element of the tile is
-    loaded and written exactly once."""
+    """The one-element-per-lane path.  Staging: every source element lands in
+    the TS x TS buffer at c ^ (r mod TS) of its row, read from inside its
+    run.  load_a_e: the A elements a lane loads are the target elements it
+    later writes, each at dst + (y * dld + x) * es inside the tile's target
+    rows, and only whole-chunk padding slots beyond the tile are left at
+    zero.  stage_drain_e: each target element is written exactly once, at
+    its own address, with the source element staged for it."""
     nx = TS if rnd.random() < 0.3 else rnd.randint(1, TS)
     ny = TS if rnd.random() < 0.3 else rnd.randint(1, TS)
     tr = rnd.random() < 0.5
@@ -139,14 +142,22 @@ def replay_elements(es, rnd):
     dld = nx + rnd.randint(0, 9)
     src = (1 << 20) + rnd.randrange(64) * es
     dst = (1 << 24) + rnd.randrange(64) * es
+    vec = 16 // es
+    ne = (TS // (32 // (TS // vec))) * vec  # NPASS * VEC: elements per lane of a full tile
 
     def slot_e(r, c):
         assert 0 <= r < TS and 0 <= c < TS
         return r * TS + (c ^ (r & (TS - 1)))
 
+    def target(y, x):
+        """Address of target element (y, x); inside the tile's rows."""
+        a = dst + (y * dld + x) * es
+        assert 0 <= y < ny and 0 <= x < nx
+        assert dst + y * dld * es <= a < dst + (y * dld + nx) * es
+        return a
+
+    # stage_issue_e
     smem = {}
-    c, r0, rpp = lane_map(ln, 0)  # the map's shape is the same for every lane
-    assert rpp >= 1
     for lane in range(32):
         c, r0, rpp = lane_map(ln, lane)
         if c >= ln:
@@ -155,26 +166,40 @@ def replay_elements(es, rnd):
             ga = src + (r * sld + c) * es
             assert src + r * sld * es <= ga < src + (r * sld + ln) * es
             smem[slot_e(r, c)] = ga
-    written, loaded = set(), set()
-    vec = 16 // es
-    ne = (TS // (32 // (TS // vec))) * vec  # elements per lane of a full tile
+
+    every = {target(y, x) for y in range(ny) for x in range(nx)}
+    loaded, stored = [], []
     for lane in range(32):
         c, r0, rpp = lane_map(nx, lane)
-        if c >= nx:
-            continue
+        on = c < nx
         npass = (ny + rpp - 1) // rpp
-        assert npass <= ne
-        for p in range(npass):
+        npad = (npass + vec - 1) // vec * vec
+        assert npass <= ne and npad <= ne
+        # load_a_e: register slot p holds A's element of pass p, or zero
+        regs = {}
+        for p in range(ne):
+            if p >= npad:
+                break
+            y = p * rpp + r0
+            regs[p] = target(y, c) if (on and p < npass and y < ny) else None
+            if regs[p] is not None:
+                loaded.append(regs[p])
+        # stage_drain_e: writes pass p's element, combined with register slot p
+        if not on:
+            continue
+        for p in range(ne):
+            if p >= npass:
+                break
             y = p * rpp + r0
             if y >= ny:
                 continue
+            a = target(y, c)
+            assert regs[p] == a                     # the A value it combines is its own
             want = src + ((c * sld + y) if tr else (y * sld + c)) * es
             assert smem.get(slot_e(c, y) if tr else slot_e(y, c)) == want
-            assert (y, c) not in written
-            written.add((y, c))
-            loaded.add((y, c))
-    every = {(y, x) for y in range(ny) for x in range(nx)}
-    assert written == every and loaded == every
+            stored.append(a)
+    assert len(stored) == len(set(stored)) and set(stored) == every
+    assert len(loaded) == len(set(loaded)) and set(loaded) == every
 
 
 @pytest.mark.parametrize("es", [4, 8])
