@@ -19,8 +19,11 @@ with explicit host->device and device->host copies around the call.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5|c2|c3|c4|c1|...]
                   [--also c2,c3,c4|none] [--mode direct|message] [--impl gb300|reference]
 
-Multi-GPU (torchrun): one independent replica per GPU (the reshuffle of one
-problem uses one GPU here), scaling "weak".
+Multi-GPU (torchrun, N > 1): a single-problem workload is split over the N
+GPUs (the multi-GPU exchange: ranks in blocks of P / N per GPU, A's owners
+relabeled for that placement, pack -> NCCL all-to-all-v -> unpack), total work
+fixed ("strong"); the batched c4 runs one independent replica per GPU
+("weak").  --exchange runs the exchange path on one GPU too.
 """
 from __future__ import annotations
 
@@ -64,6 +67,9 @@ def parse():
                     help="comma-separated workloads measured after the headline and reported "
                          "under per_config ('auto': c2,c3,c4 when the headline is c5; 'none')")
     ap.add_argument("--mode", default="direct", choices=["direct", "message"])
+    ap.add_argument("--exchange", action="store_true",
+                    help="run the multi-GPU exchange path also on one GPU (it is the path "
+                         "for every single-problem workload when N > 1)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -316,6 +322,210 @@ def run_gpu(args, workload, rank, world, local_rank):
                 traffic=traffic, probs=probs, phases=phases, kernels=kernels)
 
 
+def run_exchange(args, workload, rank, world, local_rank):
+    """The reshuffle split over the job's GPUs (Sec. 6 "Implementation", Alg.
+    3): the P ranks in blocks of about P / N per GPU, A's owners relabeled for
+    that placement (costa_relabel_placement), and every step = pack, local
+    remap, an NCCL all-to-all-v of the packed segments, unpack.  value = the
+    algorithmic bytes of the whole matrix (all GPUs) / the slowest rank's
+    time: total work fixed as N grows ("strong")."""
+    import dataclasses
+    import torch
+    import torch.distributed as dist
+    import paper_2106_06601_gb300 as costa
+    from workloads.materialize import block_element_offsets
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    probs = problems(workload, args.small)
+    assert len(probs) == 1
+    p = probs[0]
+    P, G, g = p.A.nranks, world, rank
+    place = np.array([r * G // P for r in range(P)], dtype=np.int32)
+    t0 = time.perf_counter()
+    Bd = DeviceMatrix(p.B, p.dtype, dev).fill(p.b_kind, p.seed, p.src_stream)
+
+    def ptrs(spec, dm):  # NULL for the blocks of ranks on other GPUs
+        off = block_element_offsets(spec, dm.starts)
+        ptr = (dm.arena.data_ptr() + off * dm.esize).astype(np.uint64)
+        return np.where(place[spec.owner] == g, ptr, np.uint64(0))
+
+    # relabeling for the placement: label q's blocks go to process sigma(q)
+    LA0 = costa.costa_layout_from_spec(p.A, p.dtype, np.zeros(p.A.owner.size, np.uint64))
+    LB = costa.costa_layout_from_spec(p.B, p.dtype, ptrs(p.B, Bd))
+    tv = time.perf_counter()
+    V = costa.costa_volume_noalloc(LA0, LB, p.op, 0)
+    volume_ms = (time.perf_counter() - tv) * 1e3
+    tr = time.perf_counter()
+    sigma, cross0, cross1 = costa.costa_relabel_placement(V, G, place, 0.0)
+    relabel_ms = (time.perf_counter() - tr) * 1e3
+    LA0.destroy()
+    A = dataclasses.replace(p.A, owner=sigma[p.A.owner].astype(np.int32))
+    Ad = DeviceMatrix(A, p.dtype, dev).fill(p.a_kind, p.seed, p.tgt_stream)
+    LA = costa.costa_layout_from_spec(A, p.dtype, ptrs(A, Ad))
+    sb, rb = costa.costa_exchange_sizes(LA, LB, p.op, G, place, g)
+    if world > 1:  # sends and receives must pair up before any NCCL call
+        allc = [torch.zeros(2 * G, dtype=torch.int64, device=dev) for _ in range(G)]
+        dist.all_gather(allc, torch.from_numpy(np.concatenate([sb, rb])).to(dev))
+        allc = torch.stack(allc).cpu().numpy()
+        if not all(allc[a, b] == allc[b, G + a] for a in range(G) for b in range(G)):
+            raise RuntimeError("exchange segment sizes do not pair up across ranks")
+    send = torch.empty(max(16, int(sb.sum())), dtype=torch.uint8, device=dev)
+    recv = torch.empty(max(16, int(rb.sum())), dtype=torch.uint8, device=dev)
+    x = costa.Exchange(LA, LB, p.op, G, place, g, send.data_ptr(), recv.data_ptr())
+    plan_s = time.perf_counter() - t0
+    stream = torch.cuda.Stream(dev)
+    sh = stream.cuda_stream
+    sbl, rbl = sb.tolist(), rb.tolist()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        x.pack(sh)
+        x.local(p.alpha, p.beta, sh)
+        if ev is not None:
+            ev[1].record(stream)
+        if world > 1:
+            dist.all_to_all_single(recv, send, rbl, sbl)
+        if ev is not None:
+            ev[2].record(stream)
+        x.unpack(p.alpha, p.beta, sh)
+        if ev is not None:
+            ev[3].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            step()
+    torch.cuda.synchronize(dev)
+    clocks = ClockSampler(local_rank)
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    n0 = costa.costa_kernel_launch_count()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        end.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    launches = costa.costa_kernel_launch_count() - n0
+    total_ms = max_over_ranks(start.elapsed_time(end), dev)
+    per = [a.elapsed_time(b) for a, b in ev]
+    clocks.stop()
+    clk = clocks.summary(t_wall0, t_wall1)
+    nbytes = p.algorithmic_bytes()
+    # phases (after the timed region): pack + local, the exchange, unpack
+    n = max(10, min(args.steps, 100))
+    pev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n)]
+    with torch.cuda.stream(stream):
+        for k in range(n):
+            step(pev[k])
+    torch.cuda.synchronize(dev)
+    es = p.esize
+    ra = 1 if p.beta != 0 else 0
+    phase = {}
+    for name, a, b in (("pack+local", 0, 1), ("exchange", 1, 2), ("unpack", 2, 3)):
+        phase[name] = statistics.mean(e[a].elapsed_time(e[b]) for e in pev)
+    send_b, recv_b = int(sb.sum()), int(rb.sum())
+    # elements of this GPU's tiles, from V and the relabeling: source rank p
+    # on GPU place[p], target label q on GPU place[sigma[q]]
+    src_here = place == g
+    tgt_here = place[sigma] == g
+    local_el = int(V[np.ix_(src_here, tgt_here)].sum())
+    sent_el = int(V[np.ix_(src_here, ~tgt_here)].sum())
+    recv_el = int(V[np.ix_(~src_here, tgt_here)].sum())
+    # algorithmic bytes of this GPU's kernels: pack reads and writes each sent
+    # element; local and unpack read the source, A when beta != 0, write A
+    kernel_bytes = es * (2 * sent_el + (2 + ra) * (local_el + recv_el))
+    e2e = run_exchange_e2e(args, step, stream, dev, world, nbytes, Bd, Ad, p, A, place, g)
+    x.destroy()
+    LA.destroy()
+    LB.destroy()
+    peak, peak_kind = measured_peaks()
+    value = job_throughput(nbytes, 1, args.steps, total_ms)
+    stats = {"total_volume": p.A.m * p.A.n, "local_identity": int(np.trace(V)),
+             "local_relabeled": int(sum(int(V[sigma[q], q]) for q in range(P))),
+             "n_cells": None, "n_tiles": None, "staging_bytes": send_b + recv_b,
+             "volume_ms": volume_ms, "relabel_ms": relabel_ms}
+    xinfo = {"gpus": G, "placement": f"ranks in blocks of {P // G}" + ("" if P % G == 0 else " or so"),
+             "cross_gpu_elements_identity": int(round(cross0)),
+             "cross_gpu_elements_relabeled": int(round(cross1)),
+             "send_bytes": send_b, "recv_bytes": recv_b,
+             "phase_ms": {k: round(v, 5) for k, v in phase.items()},
+             "exchange_gbs_per_gpu": None if phase["exchange"] <= 0 or world == 1
+             else round((send_b + recv_b) / (phase["exchange"] * 1e-3) / 1e9, 2)}
+    kernel_ms = phase["pack+local"] + phase["unpack"]
+    return dict(value=value, ms_per_step=total_ms / args.steps, total_ms=total_ms, per=per,
+                launches=launches, clocks=clk, e2e=e2e, plan_s=plan_s, stats=stats,
+                nbytes=nbytes, achieved=kernel_bytes / (kernel_ms * 1e-3) / 1e9 if kernel_ms > 0 else 0.0,
+                kernel_ms=kernel_ms, kernel_bytes=kernel_bytes,
+                peak=peak, peak_kind=peak_kind, traffic=None, probs=probs, phases=None,
+                kernels="remap_kernel / remap_small_kernel over the exchange's pack, local and unpack lists",
+                exchange=xinfo)
+
+
+def run_exchange_e2e(args, step, stream, dev, world, nbytes, Bd, Ad, p, A, place, g):
+    """End to end for the exchange: every step copies this GPU's rank buffers
+    of B (and of A when beta != 0) from pinned host memory, runs the step,
+    and copies its rank buffers of A back."""
+    import torch
+    if args.e2e_steps <= 0:
+        return None
+    own_a = sorted({int(A.buf[i, j]) for i in range(A.nbr) for j in range(A.nbc)
+                    if place[A.owner[i, j]] == g})
+    own_b = sorted({int(p.B.buf[i, j]) for i in range(p.B.nbr) for j in range(p.B.nbc)
+                    if place[p.B.owner[i, j]] == g})
+    hb = {r: torch.empty(Bd.buffer(r).shape, dtype=Bd.arena.dtype, pin_memory=True) for r in own_b}
+    ha = {r: torch.empty(Ad.buffer(r).shape, dtype=Ad.arena.dtype, pin_memory=True) for r in own_a}
+    for r, t in hb.items():
+        t.copy_(Bd.buffer(r))
+    for r, t in ha.items():
+        t.copy_(Ad.buffer(r))
+    torch.cuda.synchronize(dev)
+
+    def e2e_step():
+        with torch.cuda.stream(stream):
+            for r, t in hb.items():
+                Bd.buffer(r).copy_(t, non_blocking=True)
+            if p.beta != 0:
+                for r, t in ha.items():
+                    Ad.buffer(r).copy_(t, non_blocking=True)
+            step()
+            for r, t in ha.items():
+                t.copy_(Ad.buffer(r), non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s2.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e2.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = max_over_ranks(s2.elapsed_time(e2), dev)
+    h2d = sum(t.numel() * t.element_size() for t in hb.values())
+    if p.beta != 0:
+        h2d += sum(t.numel() * t.element_size() for t in ha.values())
+    d2h = sum(t.numel() * t.element_size() for t in ha.values())
+    return {"value": round(job_throughput(nbytes, 1, args.e2e_steps, ms), 3), "unit": "GB/s",
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "ms_per_step": round(ms / args.e2e_steps, 4), "steps": args.e2e_steps,
+            "path": "this GPU's rank buffers copied in from pinned host memory, exchange step, "
+                    "A's rank buffers copied out (bytes per GPU)"}
+
+
 def run_e2e(args, costa, mats, step, stream, dev, world, nbytes):
     """The metric end to end with every step's data in pinned host memory.
 
@@ -457,6 +667,14 @@ def roofline(args, r):
     step for a uniform batch), or in message mode the longest phase."""
     base = {"bound": "hbm", "peak": r["peak"], "unit": "GB/s",
             "peak_source": f"{r['peak_kind']} (MEASURED_PEAKS.json hbm_gbs)"}
+    if "exchange" in r:
+        ach = r["achieved"]
+        base.update({"achieved": round(ach, 2), "frac": round(ach / r["peak"], 4), "traffic": None,
+                     "kernel": r["kernels"] + " (per GPU, the collective excluded)",
+                     "algorithmic_bytes_per_step": r["kernel_bytes"],
+                     "kernel_ms_per_step": round(r["kernel_ms"], 5),
+                     "timing": "phase events after the timed region"})
+        return base
     ph = r["phases"]
     if ph is not None:
         top = max(ph["phases"], key=lambda x: x["ms"])
@@ -602,7 +820,8 @@ def measure(args, workload, rank, world, local_rank):
     import gc
     import torch
     probs = problems(workload, args.small)
-    r = run_gpu(args, workload, rank, world, local_rank)
+    use_x = len(probs) == 1 and (world > 1 or args.exchange)
+    r = (run_exchange if use_x else run_gpu)(args, workload, rank, world, local_rank)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         gbs, threads, desc, _, _ = run_cpu_oracle(probs, args.cpu_seconds)
@@ -632,7 +851,12 @@ def measure(args, workload, rank, world, local_rank):
                  "staging_bytes": st["staging_bytes"]},
         "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
         "cpu_baseline": cpu,
+        "scaling": "strong" if use_x else "weak",
     }
+    if use_x:
+        out["config"]["parallelism"] = f"exchange over {world} GPU(s): pack, NCCL all-to-all-v, unpack"
+        out["config"]["mode"] = "exchange"
+        out["exchange"] = r["exchange"]
     if r["phases"] is not None:
         out["message_phases"] = r["phases"]
     return out
@@ -652,14 +876,16 @@ def main():
 
     import torch
     if world > 1:
-        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+        import datetime
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank),
+                                             timeout=datetime.timedelta(minutes=3))
     head = measure(args, args.workload, rank, world, local_rank)
     others = {w: measure(args, w, rank, world, local_rank) for w in also_list(args)}
     if rank == 0:
         out = {"metric": METRIC, "value": head.pop("value"), "unit": head.pop("unit"),
                "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
                "ms_per_step": head.pop("ms_per_step"), "higher_is_better": True,
-               "scaling": "weak", "vs_baseline": None, "dtype": head.pop("dtype"),
+               "scaling": head.pop("scaling"), "vs_baseline": None, "dtype": head.pop("dtype"),
                "data": "synthetic (seeded counter-based generator, values per the workload)"}
         out.update(head)
         if others:

@@ -103,6 +103,10 @@ typedef enum { COSTA_MODE_DIRECT = 0, COSTA_MODE_MESSAGE = 1 } costa_mode;
  *          read in whole aligned 16-byte chunks: up to 15 bytes before and
  *          after it, in the same aligned chunks (so on the same page), are
  *          read and not used.  Nothing outside A's blocks is written.
+ *          NULL marks a block whose rank keeps its storage in another
+ *          process (the multi-GPU exchange, costa_exchange_create); calls
+ *          that read or write the block reject it with COSTA_ERR_LAYOUT
+ *          before any kernel runs.
  *  ld    - leading dimension in elements: the distance between consecutive
  *          columns (column-major) or rows (row-major); ld >= rows
  *          (column-major) or ld >= cols (row-major); ld < 2^31.
@@ -143,7 +147,7 @@ typedef struct {
  * The layout copies all host arrays; device pointers are borrowed.
  * Errors: COSTA_ERR_INVALID_ARG (null pointer, counts), COSTA_ERR_LAYOUT
  * (unsorted splits, owner out of range, ld too small or too large, misaligned
- * or null block pointer, bad order). */
+ * block pointer, bad order). */
 costa_status costa_layout_create(costa_layout *out, costa_dtype dt, int nranks,
                                  int nbr, const int64_t *row_splits,
                                  int nbc, const int64_t *col_splits,
@@ -157,7 +161,8 @@ costa_status costa_layout_create(costa_layout *out, costa_dtype dt, int nranks,
  * NUMROC cols) column-major at rank_ptrs[o] with leading dimension lld[o]
  * (>= local rows), so block (bi, bj) starts at local row (bi div pr)*mb and
  * local column (bj div pc)*nb.  rank_ptrs and lld are host arrays of pr*pc
- * entries indexed by owner.  Errors as costa_layout_create. */
+ * entries indexed by owner; a NULL rank_ptrs[o] gives rank o's blocks NULL
+ * pointers (storage in another process).  Errors as costa_layout_create. */
 costa_status costa_layout_create_block_cyclic(costa_layout *out, costa_dtype dt,
                                               int64_t m, int64_t n, int64_t mb, int64_t nb,
                                               int pr, int pc, char grid_order,
@@ -334,6 +339,74 @@ costa_status costa_pxtran(costa_dtype dt, int conjugate, int64_t m, int64_t n, c
 /* Frees the layouts (and plans) cached by costa_pxgemr2d / costa_pxtran. */
 costa_status costa_scalapack_release(void);
 
+/* ---- Multi-GPU exchange (Sec. 6 "Implementation", Alg. 3) ----
+ *
+ * The reshuffle with the P ranks placed on G GPUs, one process per GPU:
+ * rank r's blocks (of A and of B) live on GPU place[r].  Process g (on GPU
+ * g, the current device) runs, for A = alpha * op(B) + beta * A:
+ *   costa_exchange_pack    - copies each tile whose source rank is on g and
+ *                            whose target rank is on another GPU h into h's
+ *                            segment of g's send buffer (exactly: the
+ *                            transform comes after the transfer, Sec. 6);
+ *   costa_exchange_local   - the tiles with both ranks on g, B -> A directly;
+ *   the caller's exchange  - an all-to-all-v of the segments: g's segment for
+ *                            h goes to g's segment of h's receive buffer
+ *                            (e.g. NCCL grouped send/receive); the library
+ *                            never touches another GPU's memory;
+ *   costa_exchange_unpack  - each received tile into A with op, alpha, beta.
+ * pack and local may run together; unpack needs the whole receive buffer.
+ * The result equals costa_transform on one device bit for bit.
+ *
+ * Every process builds the same tiles from the layouts (splits, owners and
+ * storage orders, which must be identical in all processes) in one fixed
+ * canonical order, so the package contents and offsets agree without any
+ * coordination.  Segments are ordered by peer GPU: segment h starts at the
+ * sum of the sizes of segments 0 .. h-1 (the all-to-all-v displacements).
+ * Layouts may give NULL pointers for the blocks of ranks on other GPUs
+ * (costa_block); the blocks of ranks on g must be addressable by g.
+ * Relabeling (costa_relabel_placement) is a planning step before this: the
+ * caller moves label q's target blocks to process sigma[q], i.e. builds A's
+ * layout with owner sigma[q] in place of q. */
+typedef struct costa_exchange_s *costa_exchange;
+
+/* Bytes of g's send segments (send_bytes[h]: to GPU h) and receive segments
+ * (recv_bytes[h]: from GPU h); [g] is 0 in both.  Host only.  place: host,
+ * P ints in [0, G).  Errors: INVALID_ARG, SHAPE, DTYPE. */
+costa_status costa_exchange_sizes(costa_layout A, costa_layout B, costa_op op, int G, const int *place,
+                                  int g, int64_t *send_bytes, int64_t *recv_bytes);
+
+/* Builds process g's pack, local and unpack tile lists for the send and
+ * receive buffers send_buf and recv_buf (device memory of the current device,
+ * 16-byte aligned, of at least the sum of costa_exchange_sizes' send_bytes /
+ * recv_bytes; the caller owns them and keeps them alive with the exchange).
+ * The exchange owns one device allocation for its tables, freed by
+ * costa_exchange_destroy.  Errors: INVALID_ARG (placement, buffers), SHAPE,
+ * DTYPE, LAYOUT (a block of a rank on g that g cannot address), ALLOC, CUDA. */
+costa_status costa_exchange_create(costa_exchange *out, costa_layout A, costa_layout B, costa_op op, int G,
+                                   const int *place, int g, void *send_buf, void *recv_buf);
+
+/* The exchange's segment sizes in bytes (host arrays of G), as
+ * costa_exchange_sizes. */
+costa_status costa_exchange_counts(costa_exchange x, int64_t *send_bytes, int64_t *recv_bytes);
+
+/* Enqueue the phases on `stream` (asynchronous; the current device must be
+ * the exchange's).  alpha, beta: host scalars of the element type, as
+ * costa_transform; with beta == 0, A is not read. */
+costa_status costa_exchange_pack(costa_exchange x, void *stream);
+costa_status costa_exchange_local(costa_exchange x, const void *alpha, const void *beta, void *stream);
+costa_status costa_exchange_unpack(costa_exchange x, const void *alpha, const void *beta, void *stream);
+
+costa_status costa_exchange_destroy(costa_exchange x);
+
+/* Relabeling for a placement (Sec. 3 network-topology cost, Def. COPR):
+ * sigma minimizes W(G_sigma) where a package of v elements kept on its
+ * process costs 0, one between two ranks on the same GPU intra * v, and one
+ * between GPUs v (the bytes that cross the GPU link, weighted 1).  Solved
+ * as costa_relabel_cost.  cost_identity / cost_relabeled (nullable) receive
+ * W(G) and W(G_sigma).  Host only.  Errors: INVALID_ARG. */
+costa_status costa_relabel_placement(int P, const int64_t *V, int G, const int *place, double intra, int *sigma,
+                                     double *cost_identity, double *cost_relabeled);
+
 /* Diagnostics (host only, no device work): the pieces into which the plan
  * cuts one axis of A (axis 0 = rows, 1 = columns) for the pair (A, B, op).
  * Each piece is 6 int32: {A block index, op(B) block index, offset in A's
@@ -420,6 +493,16 @@ costa_status costa_debug_groups(costa_layout A, costa_layout B, costa_op op, int
  * 8-byte elements, or no tile to cut. */
 costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, void *tiles, int64_t cap_tiles,
                                 int64_t *ntiles);
+
+/* Diagnostics (host only, no device work): process g's exchange lists for
+ * buffers at the addresses send_base / recv_base: which = 0 pack, 1 local,
+ * 2 unpack, unsplit, in the canonical order (32-byte descriptors as in
+ * costa_debug_tiles).  Writes min(*count, cap) descriptors to out and the
+ * total to *count; volumes (nullable, 2 * G int64): the elements of A that g
+ * sends to each GPU h, then those it receives from each h. */
+costa_status costa_debug_exchange(costa_layout A, costa_layout B, costa_op op, int G, const int *place, int g,
+                                  uint64_t send_base, uint64_t recv_base, int which, void *out, int64_t cap,
+                                  int64_t *count, int64_t *volumes);
 
 /* Frees every cached plan (synchronizes the device). */
 costa_status costa_release_plans(void);

@@ -89,6 +89,15 @@ def _load():
         "costa_debug_groups": [P, P, I, I, P, I64, P],
         "costa_phase_timing": [I],
         "costa_phase_times": [P, P],
+        "costa_exchange_sizes": [P, P, I, I, P, I, P, P],
+        "costa_exchange_create": [P, P, P, I, I, P, I, P, P],
+        "costa_exchange_counts": [P, P, P],
+        "costa_exchange_pack": [P, P],
+        "costa_exchange_local": [P, P, P, P],
+        "costa_exchange_unpack": [P, P, P, P],
+        "costa_exchange_destroy": [P],
+        "costa_relabel_placement": [I, P, I, P, ctypes.c_double, P, P, P],
+        "costa_debug_exchange": [P, P, I, I, P, I, ctypes.c_uint64, ctypes.c_uint64, I, P, I64, P, P],
     }
     for name, args in sigs.items():
         f = getattr(lib, name)
@@ -245,6 +254,89 @@ def costa_relabel_cost(V, lat, bw):
     _check(_lib.costa_relabel_cost(P, _p(V), _p(lat), _p(bw), _p(sigma), ctypes.byref(c0),
                                    ctypes.byref(c1)))
     return sigma, c0.value, c1.value
+
+
+def costa_relabel_placement(V, G: int, place, intra: float = 0.0):
+    """(sigma, W(G), W(G_sigma)) for ranks placed on G GPUs: packages kept
+    on their process cost 0, between ranks of one GPU intra * v, between
+    GPUs v."""
+    V = _i64(V)
+    P = V.shape[0]
+    pl = _i32(place)
+    assert pl.size == P
+    sigma = np.zeros(P, dtype=np.int32)
+    c0, c1 = ctypes.c_double(), ctypes.c_double()
+    _check(_lib.costa_relabel_placement(P, _p(V), G, _p(pl), float(intra), _p(sigma),
+                                        ctypes.byref(c0), ctypes.byref(c1)))
+    return sigma, c0.value, c1.value
+
+
+def costa_exchange_sizes(A: Layout, B: Layout, op: str, G: int, place, g: int):
+    """(send_bytes[G], recv_bytes[G]) of process g's exchange segments."""
+    pl = _i32(place)
+    sb, rb = np.zeros(G, np.int64), np.zeros(G, np.int64)
+    _check(_lib.costa_exchange_sizes(A.handle, B.handle, OPS[op], G, _p(pl), g, _p(sb), _p(rb)))
+    return sb, rb
+
+
+class Exchange:
+    """Owning handle of a costa_exchange: process g's part of the reshuffle
+    with the ranks placed on G GPUs.  send_ptr / recv_ptr: device addresses
+    of the caller's send and receive buffers."""
+
+    def __init__(self, A: Layout, B: Layout, op: str, G: int, place, g: int, send_ptr: int,
+                 recv_ptr: int):
+        self.dtype = A.dtype
+        self.G = G
+        pl = _i32(place)
+        out = ctypes.c_void_p()
+        _check(_lib.costa_exchange_create(ctypes.byref(out), A.handle, B.handle, OPS[op], G, _p(pl),
+                                          g, ctypes.c_void_p(send_ptr), ctypes.c_void_p(recv_ptr)))
+        self.handle = out
+
+    def counts(self):
+        sb, rb = np.zeros(self.G, np.int64), np.zeros(self.G, np.int64)
+        _check(_lib.costa_exchange_counts(self.handle, _p(sb), _p(rb)))
+        return sb, rb
+
+    def pack(self, stream: int = 0) -> None:
+        _check(_lib.costa_exchange_pack(self.handle, ctypes.c_void_p(stream)))
+
+    def local(self, alpha, beta, stream: int = 0) -> None:
+        al, be = _scalar1(self.dtype, alpha), _scalar1(self.dtype, beta)
+        _check(_lib.costa_exchange_local(self.handle, ctypes.byref(al), ctypes.byref(be),
+                                         ctypes.c_void_p(stream)))
+
+    def unpack(self, alpha, beta, stream: int = 0) -> None:
+        al, be = _scalar1(self.dtype, alpha), _scalar1(self.dtype, beta)
+        _check(_lib.costa_exchange_unpack(self.handle, ctypes.byref(al), ctypes.byref(be),
+                                          ctypes.c_void_p(stream)))
+
+    def destroy(self) -> None:
+        if self.handle:
+            _check(_lib.costa_exchange_destroy(self.handle))
+            self.handle = ctypes.c_void_p(0)
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def costa_debug_exchange(A: Layout, B: Layout, op: str, G: int, place, g: int, send_base: int,
+                         recv_base: int, which: str):
+    """(descriptors, volumes[2, G]) of process g's pack, local or unpack list."""
+    pl = _i32(place)
+    w = {"pack": 0, "local": 1, "unpack": 2}[which]
+    cnt = ctypes.c_int64()
+    vol = np.zeros(2 * G, np.int64)
+    _check(_lib.costa_debug_exchange(A.handle, B.handle, OPS[op], G, _p(pl), g, send_base,
+                                     recv_base, w, None, 0, ctypes.byref(cnt), _p(vol)))
+    out = np.zeros(max(1, cnt.value), dtype=TILE_DTYPE)
+    _check(_lib.costa_debug_exchange(A.handle, B.handle, OPS[op], G, _p(pl), g, send_base,
+                                     recv_base, w, _p(out), cnt.value, ctypes.byref(cnt), None))
+    return out[:cnt.value], vol.reshape(2, G)
 
 
 class _BlacsGrid(ctypes.Structure):

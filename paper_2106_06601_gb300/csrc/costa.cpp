@@ -21,6 +21,7 @@
 #include <cuda_runtime_api.h>
 
 #include "costa_internal.h"
+#include "plan_lists.h"
 #include "tiles.h"
 
 namespace costa {
@@ -52,66 +53,6 @@ costa_status cuda_fail(cudaError_t e, const char *what) {
 
 double ms_since(std::chrono::steady_clock::time_point t0) {
     return std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
-}
-
-// Every tile of a list fits the kernel's tile extent along both axes (the
-// kernel's shared-memory buffers and register passes are sized by it).
-costa_status check_extents(const std::vector<TileDesc> &list, int es, const char *what) {
-    const int ts = tile_extent(es);
-    for (const TileDesc &d : list)
-        if (d.nx < 1 || d.ny < 1 || d.nx > ts || d.ny > ts)
-            return fail(COSTA_ERR_INTERNAL, "%s tile %d x %d exceeds the tile extent %d", what, d.nx, d.ny, ts);
-    return COSTA_OK;
-}
-
-// Device copies of a split list inside a plan's arena.
-struct DevList {
-    const TileDesc *tiles = nullptr;
-    int64_t ntiles = 0;
-    const TileDesc *mtiles = nullptr;
-    int64_t nmtiles = 0;
-    const TileDesc *pieces = nullptr;
-    const uint32_t *groups = nullptr;
-    int64_t ngroups = 0;
-    const uint32_t *groups_a = nullptr;  // the groups of the kinds that read A
-    int64_t ngroups_a = 0;
-    bool empty() const { return ntiles == 0 && nmtiles == 0 && ngroups == 0; }
-};
-
-struct SplitOffsets {
-    size_t tiles, mtiles, pieces, groups, groups_a;
-};
-
-// One device allocation holding all tables of a plan, built on the host
-// with 256-byte aligned sections and copied once.
-struct Arena {
-    std::vector<char> host;
-    size_t add(const void *p, size_t bytes) {
-        const size_t off = (host.size() + 255) & ~size_t(255);
-        host.resize(off + std::max<size_t>(bytes, 1));
-        if (bytes) std::memcpy(host.data() + off, p, bytes);
-        return off;
-    }
-    template <typename V> size_t add_vec(const std::vector<V> &v) {
-        return add(v.data(), v.size() * sizeof(V));
-    }
-    SplitOffsets add_split(const SplitList &l) {
-        return {add_vec(l.big), add_vec(l.mis), add_vec(l.pieces), add_vec(l.groups), add_vec(l.groups_a)};
-    }
-};
-
-DevList resolve(const char *dbase, const SplitOffsets &o, const SplitList &l) {
-    DevList d;
-    d.tiles = reinterpret_cast<const TileDesc *>(dbase + o.tiles);
-    d.ntiles = static_cast<int64_t>(l.big.size());
-    d.mtiles = reinterpret_cast<const TileDesc *>(dbase + o.mtiles);
-    d.nmtiles = static_cast<int64_t>(l.mis.size());
-    d.pieces = reinterpret_cast<const TileDesc *>(dbase + o.pieces);
-    d.groups = reinterpret_cast<const uint32_t *>(dbase + o.groups);
-    d.ngroups = l.ngroups();
-    d.groups_a = reinterpret_cast<const uint32_t *>(dbase + o.groups_a);
-    d.ngroups_a = l.ngroups_a();
-    return d;
 }
 
 struct MessageData {
@@ -357,8 +298,10 @@ bool access_range(uint64_t p, int dev, AccessRange &r, std::string &why) {
     return true;
 }
 
-costa_status check_access(costa_layout_s *L, int dev, const char *which) {
-    if (L->checked_device == dev) return COSTA_OK;
+// With `place` set, only the blocks whose owner r has place[r] == g are
+// checked (the multi-GPU exchange), and the result is not cached.
+costa_status check_access_impl(costa_layout_s *L, int dev, const char *which, const int *place, int g) {
+    if (!place && L->checked_device == dev) return COSTA_OK;
     const int64_t es = esize_of(L->dt);
     std::vector<AccessRange> known;  // sorted by lo, disjoint
     auto covered = [&](uint64_t a, uint64_t b) {  // [a, b] inside one known range
@@ -378,9 +321,13 @@ costa_status check_access(costa_layout_s *L, int dev, const char *which) {
         for (int j = 0; j < L->nbc; ++j) {
             const int64_t cols = L->C[j + 1] - L->C[j];
             if (rows == 0 || cols == 0) continue;
+            if (place && place[L->owner[static_cast<size_t>(i) * L->nbc + j]] != g) continue;
             const DevBlock &b = L->blocks[static_cast<size_t>(i) * L->nbc + j];
             const int64_t last = b.order == COSTA_COL_MAJOR ? (rows - 1) + (cols - 1) * int64_t(b.ld)
                                                             : (rows - 1) * int64_t(b.ld) + (cols - 1);
+            if (!b.ptr)
+                return fail(COSTA_ERR_LAYOUT, "%s block (%d, %d) has no storage in this process (null pointer)",
+                            which, i, j);
             const uint64_t first = b.ptr, end = b.ptr + static_cast<uint64_t>((last + 1) * es - 1);
             if (covered(first, end)) continue;
             AccessRange r;
@@ -398,8 +345,12 @@ costa_status check_access(costa_layout_s *L, int dev, const char *which) {
             add(r);
         }
     }
-    L->checked_device = dev;
+    if (!place) L->checked_device = dev;
     return COSTA_OK;
+}
+
+costa_status check_access(costa_layout_s *L, int dev, const char *which) {
+    return check_access_impl(L, dev, which, nullptr, 0);
 }
 
 // Builds the overlay, the tile list and the device tables, and runs the
@@ -724,38 +675,6 @@ costa_status get_plan(int n, const costa_layout *A, const costa_layout *B, const
 }
 
 // Reads one scalar of element type dt at p[index].
-void read_scalar(int dt, const void *p, int index, double out[2]) {
-    switch (dt) {
-    case COSTA_F32: out[0] = static_cast<const float *>(p)[index]; out[1] = 0.0; break;
-    case COSTA_F64: out[0] = static_cast<const double *>(p)[index]; out[1] = 0.0; break;
-    case COSTA_C64:
-        out[0] = static_cast<const float *>(p)[2 * index];
-        out[1] = static_cast<const float *>(p)[2 * index + 1];
-        break;
-    default:
-        out[0] = static_cast<const double *>(p)[2 * index];
-        out[1] = static_cast<const double *>(p)[2 * index + 1];
-        break;
-    }
-}
-
-Scalars make_scalars(int dt, const void *alpha, const void *beta, int index) {
-    Scalars s{};
-    read_scalar(dt, alpha, index, s.alpha);
-    read_scalar(dt, beta, index, s.beta);
-    s.flags = 0;
-    if (s.beta[0] == 0.0 && s.beta[1] == 0.0) s.flags |= SF_BETA0;
-    if (s.alpha[0] == 1.0 && s.alpha[1] == 0.0) s.flags |= SF_ALPHA1;
-    if (s.alpha[1] != 0.0 || s.beta[1] != 0.0) s.flags |= SF_CPLX;
-    int e = 0;
-    const double fr = std::frexp(std::fabs(s.beta[0]), &e);
-    if (s.beta[1] == 0.0 && fr == 0.5 && e - 1 >= -1000 && e - 1 <= 1000) {
-        s.flags |= SF_BPOW2;  // |beta| = 2^(e-1)
-        s.beta_exp = e - 1;
-    }
-    return s;
-}
-
 bool same_scalars(const Scalars &a, const Scalars &b) { return std::memcmp(&a, &b, sizeof(Scalars)) == 0; }
 
 costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B, const costa_op *ops,
@@ -835,29 +754,7 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
     // halves: the list for the kinds that run on x-halves (null: none)
     auto launch_list = [&](const DevList &list, const DevList *halves) -> cudaError_t {
-        RemapLaunch l = L;
-        l.tiles = list.tiles;
-        l.ntiles = list.ntiles;
-        l.mtiles = list.mtiles;
-        l.nmtiles = list.nmtiles;
-        l.pieces = list.pieces;
-        l.groups = list.groups;
-        l.ngroups = list.ngroups;
-        for (int kind = 0; kind < K_NKINDS; ++kind) {
-            if (!kinds[kind]) continue;
-            RemapLaunch lk = l;
-            if (halves && (plan->esize == 4 || kind == K_AXPBY2)) {
-                lk.tiles = halves->tiles;
-                lk.ntiles = halves->ntiles;
-            }
-            if (kind_reads_a(kind)) {  // the groups of the kinds that read A
-                lk.groups = list.groups_a;
-                lk.ngroups = list.ngroups_a;
-            }
-            cudaError_t e = launch_remap(lk, kind, stream);
-            if (e != cudaSuccess) return e;
-        }
-        return cudaSuccess;
+        return launch_split(L, list, halves, plan->esize, kinds, stream);
     };
     cudaError_t ce;
     if (mode == COSTA_MODE_DIRECT) {
@@ -947,7 +844,9 @@ costa_status create_layout(costa_layout *out, int dt, int nranks, int nbr, const
                 if (blk.order != COSTA_COL_MAJOR && blk.order != COSTA_ROW_MAJOR)
                     return fail(COSTA_ERR_LAYOUT, "block (%d, %d): bad order %d", i, j, blk.order);
                 if (blk.reserved != 0) return fail(COSTA_ERR_LAYOUT, "block (%d, %d): reserved != 0", i, j);
-                if (!blk.ptr) return fail(COSTA_ERR_LAYOUT, "block (%d, %d): null pointer", i, j);
+                // a null pointer: the block's rank keeps its storage in another
+                // process (multi-GPU exchange); calls that would read or write
+                // the block reject it (check_access, check_blocks_on)
                 if (reinterpret_cast<uintptr_t>(blk.ptr) % es)
                     return fail(COSTA_ERR_LAYOUT, "block (%d, %d): pointer not aligned to %d bytes", i, j, es);
                 const int64_t need = blk.order == COSTA_COL_MAJOR ? h : w;
@@ -979,7 +878,80 @@ int64_t numroc(int64_t n, int64_t nb, int iproc, int nprocs) {
 
 }  // namespace
 
+// Every tile of a list fits the kernel's tile extent along both axes (the
+// kernel's shared-memory buffers and register passes are sized by it).
+costa_status check_extents(const std::vector<TileDesc> &list, int es, const char *what) {
+    const int ts = tile_extent(es);
+    for (const TileDesc &d : list)
+        if (d.nx < 1 || d.ny < 1 || d.nx > ts || d.ny > ts)
+            return fail(COSTA_ERR_INTERNAL, "%s tile %d x %d exceeds the tile extent %d", what, d.nx, d.ny, ts);
+    return COSTA_OK;
+}
+
+void read_scalar(int dt, const void *p, int index, double out[2]) {
+    switch (dt) {
+    case COSTA_F32: out[0] = static_cast<const float *>(p)[index]; out[1] = 0.0; break;
+    case COSTA_F64: out[0] = static_cast<const double *>(p)[index]; out[1] = 0.0; break;
+    case COSTA_C64:
+        out[0] = static_cast<const float *>(p)[2 * index];
+        out[1] = static_cast<const float *>(p)[2 * index + 1];
+        break;
+    default:
+        out[0] = static_cast<const double *>(p)[2 * index];
+        out[1] = static_cast<const double *>(p)[2 * index + 1];
+        break;
+    }
+}
+
+Scalars make_scalars(int dt, const void *alpha, const void *beta, int index) {
+    Scalars s{};
+    read_scalar(dt, alpha, index, s.alpha);
+    read_scalar(dt, beta, index, s.beta);
+    s.flags = 0;
+    if (s.beta[0] == 0.0 && s.beta[1] == 0.0) s.flags |= SF_BETA0;
+    if (s.alpha[0] == 1.0 && s.alpha[1] == 0.0) s.flags |= SF_ALPHA1;
+    if (s.alpha[1] != 0.0 || s.beta[1] != 0.0) s.flags |= SF_CPLX;
+    int e = 0;
+    const double fr = std::frexp(std::fabs(s.beta[0]), &e);
+    if (s.beta[1] == 0.0 && fr == 0.5 && e - 1 >= -1000 && e - 1 <= 1000) {
+        s.flags |= SF_BPOW2;  // |beta| = 2^(e-1)
+        s.beta_exp = e - 1;
+    }
+    return s;
+}
+
+cudaError_t launch_split(const RemapLaunch &base, const DevList &list, const DevList *halves, int esize,
+                         const bool (&kinds)[K_NKINDS], cudaStream_t stream) {
+    RemapLaunch l = base;
+    l.tiles = list.tiles;
+    l.ntiles = list.ntiles;
+    l.mtiles = list.mtiles;
+    l.nmtiles = list.nmtiles;
+    l.pieces = list.pieces;
+    l.groups = list.groups;
+    l.ngroups = list.ngroups;
+    for (int kind = 0; kind < K_NKINDS; ++kind) {
+        if (!kinds[kind]) continue;
+        RemapLaunch lk = l;
+        if (halves && (esize == 4 || kind == K_AXPBY2)) {
+            lk.tiles = halves->tiles;
+            lk.ntiles = halves->ntiles;
+        }
+        if (kind_reads_a(kind)) {  // the groups of the kinds that read A
+            lk.groups = list.groups_a;
+            lk.ngroups = list.ngroups_a;
+        }
+        cudaError_t e = launch_remap(lk, kind, stream);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
 costa_status report_error(costa_status s, const char *message) { return fail(s, "%s", message); }
+
+costa_status check_access_on(costa_layout_s *L, int dev, const char *which, const int *place, int g) {
+    return check_access_impl(L, dev, which, place, g);
+}
 
 costa_status check_pair(const costa_layout_s *A, const costa_layout_s *B, int op) {
     return validate_pair(A, B, op);
@@ -1039,7 +1011,8 @@ costa_status costa_layout_create_block_cyclic(costa_layout *out, costa_dtype dt,
             if (lld[o] < std::max<int64_t>(1, need))
                 return fail(COSTA_ERR_LAYOUT, "lld[%d] = %lld < local rows %lld", o, (long long)lld[o],
                             (long long)need);
-            blocks[b].ptr = static_cast<char *>(rank_ptrs[o]) + (lr + lc * lld[o]) * es;
+            // a null rank pointer: that rank's storage lives in another process
+            blocks[b].ptr = rank_ptrs[o] ? static_cast<char *>(rank_ptrs[o]) + (lr + lc * lld[o]) * es : nullptr;
             blocks[b].ld = lld[o];
             blocks[b].order = COSTA_COL_MAJOR;
             blocks[b].reserved = 0;
@@ -1142,6 +1115,21 @@ costa_status costa_relabel_cost(int P, const int64_t *V, const double *lat, cons
     if (cost_identity) *cost_identity = ident;
     if (cost_relabeled) *cost_relabeled = keep ? ident : best;
     return COSTA_OK;
+}
+
+costa_status costa_relabel_placement(int P, const int64_t *V, int G, const int *place, double intra, int *sigma,
+                                     double *cost_identity, double *cost_relabeled) {
+    if (P < 1) return fail(COSTA_ERR_INVALID_ARG, "P %d < 1", P);
+    if (G < 1 || !place) return fail(COSTA_ERR_INVALID_ARG, "G < 1 or null placement");
+    if (!std::isfinite(intra) || intra < 0.0) return fail(COSTA_ERR_INVALID_ARG, "intra must be finite and >= 0");
+    for (int r = 0; r < P; ++r)
+        if (place[r] < 0 || place[r] >= G) return fail(COSTA_ERR_INVALID_ARG, "place[%d] not in [0, %d)", r, G);
+    const size_t PP = static_cast<size_t>(P) * P;
+    std::vector<double> lat(PP, 0.0), bw(PP, 0.0);
+    for (int i = 0; i < P; ++i)
+        for (int k = 0; k < P; ++k)
+            if (i != k) bw[static_cast<size_t>(i) * P + k] = place[i] == place[k] ? intra : 1.0;
+    return costa_relabel_cost(P, V, lat.data(), bw.data(), sigma, cost_identity, cost_relabeled);
 }
 
 costa_status costa_relabel_greedy(int P, const int64_t *V, int *sigma, int64_t *local_volume) {

@@ -1,0 +1,86 @@
+// Device tile lists of a plan and their launch, shared by the planner of
+// the single-GPU transform (costa.cpp) and the multi-GPU exchange
+// (exchange.cpp).  Host code only.
+#pragma once
+
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
+#include "costa_internal.h"
+#include "tiles.h"
+
+namespace costa {
+
+// Device copies of a split list inside a plan's arena.
+struct DevList {
+    const TileDesc *tiles = nullptr;
+    int64_t ntiles = 0;
+    const TileDesc *mtiles = nullptr;
+    int64_t nmtiles = 0;
+    const TileDesc *pieces = nullptr;
+    const uint32_t *groups = nullptr;
+    int64_t ngroups = 0;
+    const uint32_t *groups_a = nullptr;  // the groups of the kinds that read A
+    int64_t ngroups_a = 0;
+    bool empty() const { return ntiles == 0 && nmtiles == 0 && ngroups == 0; }
+};
+
+struct SplitOffsets {
+    size_t tiles, mtiles, pieces, groups, groups_a;
+};
+
+// One device allocation holding all tables of a plan, built on the host
+// with 256-byte aligned sections and copied once.
+struct Arena {
+    std::vector<char> host;
+    size_t add(const void *p, size_t bytes) {
+        const size_t off = (host.size() + 255) & ~size_t(255);
+        host.resize(off + std::max<size_t>(bytes, 1));
+        if (bytes) std::memcpy(host.data() + off, p, bytes);
+        return off;
+    }
+    template <typename V> size_t add_vec(const std::vector<V> &v) {
+        return add(v.data(), v.size() * sizeof(V));
+    }
+    SplitOffsets add_split(const SplitList &l) {
+        return {add_vec(l.big), add_vec(l.mis), add_vec(l.pieces), add_vec(l.groups), add_vec(l.groups_a)};
+    }
+};
+
+inline DevList resolve(const char *dbase, const SplitOffsets &o, const SplitList &l) {
+    DevList d;
+    d.tiles = reinterpret_cast<const TileDesc *>(dbase + o.tiles);
+    d.ntiles = static_cast<int64_t>(l.big.size());
+    d.mtiles = reinterpret_cast<const TileDesc *>(dbase + o.mtiles);
+    d.nmtiles = static_cast<int64_t>(l.mis.size());
+    d.pieces = reinterpret_cast<const TileDesc *>(dbase + o.pieces);
+    d.groups = reinterpret_cast<const uint32_t *>(dbase + o.groups);
+    d.ngroups = l.ngroups();
+    d.groups_a = reinterpret_cast<const uint32_t *>(dbase + o.groups_a);
+    d.ngroups_a = l.ngroups_a();
+    return d;
+}
+
+
+// Every tile of a list fits the kernel's tile extent along both axes.
+costa_status check_extents(const std::vector<TileDesc> &list, int es, const char *what);
+
+// Every nonempty block of a layout whose owner r has place[r] == g lies in
+// memory the current device `dev` can address (the rule of a single-GPU
+// transform, applied to the blocks of the ranks on one GPU).
+costa_status check_access_on(costa_layout_s *L, int dev, const char *which, const int *place, int g);
+
+// One element type's scalars alpha[index], beta[index] read from host arrays
+// of that type, with the flags that choose the combine kind.
+void read_scalar(int dt, const void *p, int index, double out[2]);
+Scalars make_scalars(int dt, const void *alpha, const void *beta, int index);
+
+// Launches the remap kernel over a split tile list, once per combine kind
+// set in `kinds`: the kinds that run on x-halves take `halves` (when not
+// null) for their full-size tiles, and the kinds that read A take the
+// small pieces' groups sized for them.
+cudaError_t launch_split(const RemapLaunch &base, const DevList &list, const DevList *halves, int esize,
+                         const bool (&kinds)[K_NKINDS], cudaStream_t stream);
+
+}  // namespace costa
