@@ -185,6 +185,37 @@ costa_status costa_layout_info(costa_layout layout, int64_t *m, int64_t *n,
 costa_status costa_volume(costa_layout A, costa_layout B, costa_op op, int64_t *V,
                           void *stream);
 
+/* The volumes of costa_volume (same V, same layout of the result) computed
+ * without allocating device memory.  The paper has no counterpart: it exists
+ * for callers that cannot let a library call cudaMalloc, such as an
+ * application whose framework owns all device memory through its own pool,
+ * or code on a latency-critical path where cudaMalloc / cudaFree would
+ * synchronize the device.
+ *  - Memory: all device work happens in one fixed scratch array of 4 MiB
+ *    that is part of the library's device image; every GPU that loads the
+ *    library holds it until the process exits.  No cudaMalloc, cudaFree or
+ *    other allocating call is made, and no plan is built or cached.
+ *  - Limit: the pair needs 8 * P^2 bytes for V plus its split and owner
+ *    arrays (8 bytes per split, 4 per block of A and of B, each section
+ *    rounded up to 256 bytes); more than 4 MiB is rejected with
+ *    COSTA_ERR_INVALID_ARG and a message giving both sizes.
+ *  - Set-up: every call, with the calling device current, looks up the
+ *    array's device address (cudaGetSymbolAddress, which allocates
+ *    nothing), so the address stays valid when the device's context is
+ *    created again (after cudaDeviceReset).  The first lookup on a device
+ *    may load the library's device code: make the first call before any
+ *    stream capture.
+ *  - Sharing: every call uses the same array, which keeps the last call's
+ *    contents (V is zeroed on the stream at the start of each call).  Calls
+ *    that overlap on the GPU would race; this entry point is synchronous and
+ *    serializes its own calls (also on its error paths, which wait for the
+ *    work already queued), so they do not overlap within one process.
+ *  - Synchronization: runs on `stream` and synchronizes it before returning.
+ * V: host array of P * P int64, as in costa_volume.  Errors: INVALID_ARG,
+ * SHAPE, DTYPE, CUDA. */
+costa_status costa_volume_noalloc(costa_layout A, costa_layout B, costa_op op, int64_t *V,
+                                  void *stream);
+
 /* Communication-optimal process relabeling for the locally-free volume cost
  * (Eq. 2; Remark on the gain and Thm. 1 / Thm. 2, Sec. 4): sigma maximizes
  * sum_q V[sigma[q] * P + q], i.e. target label q is taken by process
@@ -267,6 +298,19 @@ typedef struct {
  * overlay cells, no device work.  Errors: INVALID_ARG, LAYOUT, SHAPE. */
 costa_status costa_volume_grid(const costa_grid_desc *A, const costa_grid_desc *B, costa_op op, int P,
                                int64_t *V);
+
+/* Fills the arrays of a costa_grid_desc for a block-cyclic m x n layout with
+ * mb x nb blocks on a pr x pc grid (zero source offsets; the last block of
+ * each axis may be partial): row_splits[i] = min(i * mb, m), row_procs[bi] =
+ * bi mod pr, likewise for columns, and grid[i * pc + j] = the rank of grid
+ * process (i, j): i * pc + j for grid_order 'R', i + j * pr for 'C', mapped
+ * through rank_perm when it is not NULL.  With row_splits == NULL only
+ * *nbr and *nbc are written (the array sizes: nbr + 1, nbr, nbc + 1, nbc,
+ * pr * pc).  Host only.  Errors: INVALID_ARG. */
+costa_status costa_grid_block_cyclic(int64_t m, int64_t n, int64_t mb, int64_t nb, int pr, int pc,
+                                     char grid_order, const int *rank_perm, int64_t *row_splits,
+                                     int *row_procs, int64_t *col_splits, int *col_procs, int *grid,
+                                     int *nbr, int *nbc);
 
 /* The greedy relabeling of Sec. 6 ("a simple greedy algorithm, which is a
  * 2-approximation" of the maximum-weight perfect matching): pairs (p, q) by
@@ -407,6 +451,20 @@ costa_status costa_exchange_destroy(costa_exchange x);
 costa_status costa_relabel_placement(int P, const int64_t *V, int G, const int *place, double intra, int *sigma,
                                      double *cost_identity, double *cost_relabeled);
 
+/* ---- Housekeeping ---- */
+
+/* Frees every cached plan (synchronizes the device). */
+costa_status costa_release_plans(void);
+
+/* Thread-local message of the last failed call on this thread ("" if none). */
+const char *costa_last_error(void);
+
+/* ---- Diagnostics ----
+ *
+ * Not needed to reshuffle: they expose the planner's tile lists (host only,
+ * no device work), count kernel launches, and time the phases of transform
+ * calls, for tests, tuning and profiling. */
+
 /* Diagnostics (host only, no device work): the pieces into which the plan
  * cuts one axis of A (axis 0 = rows, 1 = columns) for the pair (A, B, op).
  * Each piece is 6 int32: {A block index, op(B) block index, offset in A's
@@ -415,37 +473,6 @@ costa_status costa_relabel_placement(int P, const int64_t *V, int G, const int *
  * min(*count, cap) pieces to out (6 * cap int32) and the total to *count. */
 costa_status costa_debug_axis_pieces(costa_layout A, costa_layout B, costa_op op, int axis,
                                      int32_t *out, int64_t cap, int64_t *count);
-
-/* The volumes of costa_volume (same V, same layout of the result) computed
- * without allocating device memory.  The paper has no counterpart: it exists
- * for callers that cannot let a library call cudaMalloc, such as an
- * application whose framework owns all device memory through its own pool,
- * or code on a latency-critical path where cudaMalloc / cudaFree would
- * synchronize the device.
- *  - Memory: all device work happens in one fixed scratch array of 4 MiB
- *    that is part of the library's device image; every GPU that loads the
- *    library holds it until the process exits.  No cudaMalloc, cudaFree or
- *    other allocating call is made, and no plan is built or cached.
- *  - Limit: the pair needs 8 * P^2 bytes for V plus its split and owner
- *    arrays (8 bytes per split, 4 per block of A and of B, each section
- *    rounded up to 256 bytes); more than 4 MiB is rejected with
- *    COSTA_ERR_INVALID_ARG and a message giving both sizes.
- *  - Set-up: every call, with the calling device current, looks up the
- *    array's device address (cudaGetSymbolAddress, which allocates
- *    nothing), so the address stays valid when the device's context is
- *    created again (after cudaDeviceReset).  The first lookup on a device
- *    may load the library's device code: make the first call before any
- *    stream capture.
- *  - Sharing: every call uses the same array, which keeps the last call's
- *    contents (V is zeroed on the stream at the start of each call).  Calls
- *    that overlap on the GPU would race; this entry point is synchronous and
- *    serializes its own calls (also on its error paths, which wait for the
- *    work already queued), so they do not overlap within one process.
- *  - Synchronization: runs on `stream` and synchronizes it before returning.
- * V: host array of P * P int64, as in costa_volume.  Errors: INVALID_ARG,
- * SHAPE, DTYPE, CUDA. */
-costa_status costa_volume_noalloc(costa_layout A, costa_layout B, costa_op op, int64_t *V,
-                                  void *stream);
 
 /* Diagnostics (host only, no device work): the remap kernel's tile list for
  * (A, B, op) in direct mode, in the order the kernel's warps take the tiles.  Each tile is 32 bytes: {source address, target
@@ -503,12 +530,6 @@ costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, voi
 costa_status costa_debug_exchange(costa_layout A, costa_layout B, costa_op op, int G, const int *place, int g,
                                   uint64_t send_base, uint64_t recv_base, int which, void *out, int64_t cap,
                                   int64_t *count, int64_t *volumes);
-
-/* Frees every cached plan (synchronizes the device). */
-costa_status costa_release_plans(void);
-
-/* Thread-local message of the last failed call on this thread ("" if none). */
-const char *costa_last_error(void);
 
 /* Number of kernels this library has launched in this process. */
 int64_t costa_kernel_launch_count(void);

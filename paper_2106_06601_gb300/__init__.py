@@ -77,6 +77,7 @@ def _load():
         "costa_release_plans": [],
         "costa_debug_axis_pieces": [P, P, I, I, P, I64, P],
         "costa_volume_grid": [P, P, I, I, P],
+        "costa_grid_block_cyclic": [I64, I64, I64, I64, I, I, ctypes.c_char, P, P, P, P, P, P, P, P],
         "costa_relabel_greedy": [I, P, P, P],
         "costa_relabel_cost": [I, P, P, P, P, P, P],
         "costa_layout_create_scalapack": [P, I, P, I64, I64, I64, I64, P],
@@ -411,13 +412,18 @@ class GridLayout:
 
     @staticmethod
     def block_cyclic(m, n, mb, nb, pr, pc, grid_order="R", rank_perm=None):
-        rs = np.append(np.arange(0, m, mb, dtype=np.int64), m)
-        cs = np.append(np.arange(0, n, nb, dtype=np.int64), n)
-        ranks = np.arange(pr * pc).reshape(pr, pc) if grid_order == "R" else \
-            np.arange(pr * pc).reshape(pc, pr).T
-        if rank_perm is not None:
-            ranks = np.asarray(rank_perm)[ranks]
-        return GridLayout(rs, np.arange(len(rs) - 1) % pr, cs, np.arange(len(cs) - 1) % pc, ranks)
+        """The grid of a block-cyclic layout (costa_grid_block_cyclic)."""
+        nbr, nbc = ctypes.c_int(), ctypes.c_int()
+        perm = None if rank_perm is None else _i32(rank_perm)
+        args = (m, n, mb, nb, pr, pc, grid_order.encode(), None if perm is None else _p(perm))
+        _check(_lib.costa_grid_block_cyclic(*args, None, None, None, None, None,
+                                            ctypes.byref(nbr), ctypes.byref(nbc)))
+        rs, cs = np.zeros(nbr.value + 1, np.int64), np.zeros(nbc.value + 1, np.int64)
+        rp, cp = np.zeros(max(1, nbr.value), np.int32), np.zeros(max(1, nbc.value), np.int32)
+        grid = np.zeros((pr, pc), np.int32)
+        _check(_lib.costa_grid_block_cyclic(*args, _p(rs), _p(rp), _p(cs), _p(cp), _p(grid),
+                                            ctypes.byref(nbr), ctypes.byref(nbc)))
+        return GridLayout(rs, rp[:nbr.value], cs, cp[:nbc.value], grid)
 
 
 def costa_volume_grid(A: GridLayout, B: GridLayout, op: str, P: int) -> np.ndarray:

@@ -357,6 +357,7 @@ costa_status check_access(costa_layout_s *L, int dev, const char *which) {
 // volume kernel.
 costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, const costa_op *ops,
                         cudaStream_t stream, std::unique_ptr<Plan> &out) {
+    Trace range("costa plan");
     auto t0 = std::chrono::steady_clock::now();
     auto plan = std::make_unique<Plan>();
     cudaError_t ce = cudaGetDevice(&plan->device);
@@ -470,6 +471,7 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     plan->total_cells = cells;
 
     // volume kernel: V[p][q] over the overlay cells
+    Trace range_v("costa volume");
     auto tv = std::chrono::steady_clock::now();
     VolumeLaunch vl;
     vl.probs = reinterpret_cast<const VolumeProblemDev *>(dbase + off_vd);
@@ -501,16 +503,25 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     plan->stats.n_cells = cells;
     plan->stats.n_tiles = tiles;
     plan->stats.plan_ms = ms_since(t0);
+    log_msg(1, "plan: %d pair(s), dtype %d, P = %d, %lld cells, %lld tiles (%lld direct, %lld misaligned, "
+               "%lld small pieces), total volume %lld, local %lld; %.2f ms (volume %.2f ms)",
+            n, plan->dtype, P, (long long)cells, (long long)tiles, (long long)split.big.size(),
+            (long long)split.mis.size(), (long long)split.pieces.size(), (long long)total, (long long)trace,
+            plan->stats.plan_ms, plan->stats.volume_ms);
     out = std::move(plan);
     return COSTA_OK;
 }
 
 costa_status ensure_sigma(Plan &plan) {
     if (plan.sigma_done) return COSTA_OK;
+    Trace trace("costa relabel");
     auto t0 = std::chrono::steady_clock::now();
     int64_t best = 0;
     solve_relabel(plan.P, plan.V.data(), plan.sigma, best);
     plan.stats.relabel_ms = ms_since(t0);
+    log_msg(1, "relabel: P = %d, local volume %lld -> %lld of %lld; %.3f ms", plan.P,
+            (long long)plan.stats.local_identity, (long long)best, (long long)plan.stats.total_volume,
+            plan.stats.relabel_ms);
     plan.stats.local_relabeled = best;
     plan.sigma_done = true;
     return COSTA_OK;
@@ -526,6 +537,7 @@ costa_status ensure_sigma(Plan &plan) {
 costa_status ensure_message(Plan &plan, bool relabel) {
     MessageData &m = plan.msg[relabel ? 1 : 0];
     if (m.built) return COSTA_OK;
+    Trace trace("costa message plan");
     const int P = plan.P, es = plan.esize;
     std::vector<int> sig(P);
     if (relabel) {
@@ -644,6 +656,9 @@ costa_status ensure_message(Plan &plan, bool relabel) {
     }
     m.built = true;
     plan.stats.staging_bytes = m.staging_bytes;
+    log_msg(1, "message plan (relabel %d): staging %lld bytes, pack %lld, local %lld, unpack %lld tiles",
+            relabel ? 1 : 0, (long long)m.staging_bytes, (long long)(m.pack.ntiles + m.pack.nmtiles),
+            (long long)(m.local.ntiles + m.local.nmtiles), (long long)(m.unpack.ntiles + m.unpack.nmtiles));
     return COSTA_OK;
 }
 
@@ -709,6 +724,9 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         timer->nphases = 0;
     }
     if (plan->total_tiles == 0) return COSTA_OK;
+    Trace trace("costa transform");
+    log_msg(2, "transform: %d pair(s), %s mode, relabel %d, stream %p", n,
+            mode == COSTA_MODE_DIRECT ? "direct" : "message", relabel ? 1 : 0, static_cast<void *>(stream));
     // event k marks the end of phase k (event 0: the start)
     auto mark = [&](int k) -> cudaError_t { return timer ? cudaEventRecord(timer->ev[k], stream) : cudaSuccess; };
 
@@ -948,6 +966,24 @@ cudaError_t launch_split(const RemapLaunch &base, const DevList &list, const Dev
 }
 
 costa_status report_error(costa_status s, const char *message) { return fail(s, "%s", message); }
+
+int log_level() {
+    static const int level = [] {
+        const char *e = std::getenv("COSTA_LOG");
+        return e ? std::max(0, std::atoi(e)) : 0;
+    }();
+    return level;
+}
+
+void log_msg(int level, const char *fmt, ...) {
+    if (log_level() < level) return;
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    std::fprintf(stderr, "[costa] %s\n", buf);
+}
 
 costa_status check_access_on(costa_layout_s *L, int dev, const char *which, const int *place, int g) {
     return check_access_impl(L, dev, which, place, g);

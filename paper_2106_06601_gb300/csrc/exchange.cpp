@@ -252,6 +252,7 @@ costa_status costa_exchange_create(costa_exchange *out, costa_layout A, costa_la
                                    const int *place, int g, void *send_buf, void *recv_buf) {
     if (!out) return fail_msg(COSTA_ERR_INVALID_ARG, "out is null");
     *out = nullptr;
+    Trace trace("costa exchange plan");
     auto x = std::make_unique<costa_exchange_s>();
     cudaError_t ce = cudaGetDevice(&x->device);
     if (ce != cudaSuccess) return cuda_msg(ce, "cudaGetDevice");
@@ -327,6 +328,11 @@ costa_status costa_exchange_create(costa_exchange *out, costa_layout A, costa_la
         x->unpack_halves.tiles = reinterpret_cast<const TileDesc *>(db + o_hu);
         x->unpack_halves.ntiles = static_cast<int64_t>(h_unpack.size());
     }
+    log_msg(1, "exchange plan: GPU %d of %d, send %lld bytes, receive %lld bytes; pack %zu, local %zu, "
+               "unpack %zu tiles", g, G, (long long)(nsend * es), (long long)(nrecv * es),
+            s_pack.big.size() + s_pack.mis.size() + s_pack.pieces.size(),
+            s_local.big.size() + s_local.mis.size() + s_local.pieces.size(),
+            s_unpack.big.size() + s_unpack.mis.size() + s_unpack.pieces.size());
     *out = x.release();
     return COSTA_OK;
 }
@@ -341,16 +347,19 @@ costa_status costa_exchange_counts(costa_exchange x, int64_t *send_bytes, int64_
 }
 
 costa_status costa_exchange_pack(costa_exchange x, void *stream) {
+    Trace trace("costa exchange pack");
     if (!x) return fail_msg(COSTA_ERR_INVALID_ARG, "null exchange");
     return exchange_launch(x, x->pack, nullptr, nullptr, nullptr, stream, true);
 }
 
 costa_status costa_exchange_local(costa_exchange x, const void *alpha, const void *beta, void *stream) {
+    Trace trace("costa exchange local");
     if (!x) return fail_msg(COSTA_ERR_INVALID_ARG, "null exchange");
     return exchange_launch(x, x->local, &x->local_halves, alpha, beta, stream, false);
 }
 
 costa_status costa_exchange_unpack(costa_exchange x, const void *alpha, const void *beta, void *stream) {
+    Trace trace("costa exchange unpack");
     if (!x) return fail_msg(COSTA_ERR_INVALID_ARG, "null exchange");
     return exchange_launch(x, x->unpack, &x->unpack_halves, alpha, beta, stream, false);
 }

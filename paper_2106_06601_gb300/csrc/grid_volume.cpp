@@ -116,3 +116,42 @@ extern "C" costa_status costa_volume_grid(const costa_grid_desc *A, const costa_
         }
     return COSTA_OK;
 }
+
+extern "C" costa_status costa_grid_block_cyclic(int64_t m, int64_t n, int64_t mb, int64_t nb, int pr, int pc,
+                                                char grid_order, const int *rank_perm, int64_t *row_splits,
+                                                int *row_procs, int64_t *col_splits, int *col_procs, int *grid,
+                                                int *nbr, int *nbc) {
+    using costa::report_error;
+    if (!nbr || !nbc) return report_error(COSTA_ERR_INVALID_ARG, "costa_grid_block_cyclic: null count");
+    if (m < 0 || n < 0 || mb < 1 || nb < 1 || pr < 1 || pc < 1)
+        return report_error(COSTA_ERR_INVALID_ARG, "costa_grid_block_cyclic: bad sizes");
+    if (grid_order != 'R' && grid_order != 'C')
+        return report_error(COSTA_ERR_INVALID_ARG, "costa_grid_block_cyclic: grid_order must be 'R' or 'C'");
+    const int64_t br = (m + mb - 1) / mb, bc = (n + nb - 1) / nb;
+    if (br > (int64_t(1) << 30) || bc > (int64_t(1) << 30))
+        return report_error(COSTA_ERR_INVALID_ARG, "costa_grid_block_cyclic: too many blocks");
+    *nbr = static_cast<int>(br);
+    *nbc = static_cast<int>(bc);
+    if (!row_splits) return COSTA_OK;
+    if (!row_procs || !col_splits || !col_procs || !grid)
+        return report_error(COSTA_ERR_INVALID_ARG, "costa_grid_block_cyclic: null array");
+    const int P = pr * pc;
+    if (rank_perm) {
+        std::vector<char> seen(P, 0);
+        for (int r = 0; r < P; ++r) {
+            if (rank_perm[r] < 0 || rank_perm[r] >= P || seen[rank_perm[r]])
+                return report_error(COSTA_ERR_INVALID_ARG, "costa_grid_block_cyclic: rank_perm is not a permutation");
+            seen[rank_perm[r]] = 1;
+        }
+    }
+    for (int64_t i = 0; i <= br; ++i) row_splits[i] = std::min<int64_t>(i * mb, m);
+    for (int64_t j = 0; j <= bc; ++j) col_splits[j] = std::min<int64_t>(j * nb, n);
+    for (int64_t i = 0; i < br; ++i) row_procs[i] = static_cast<int>(i % pr);
+    for (int64_t j = 0; j < bc; ++j) col_procs[j] = static_cast<int>(j % pc);
+    for (int i = 0; i < pr; ++i)
+        for (int j = 0; j < pc; ++j) {
+            const int r = grid_order == 'R' ? i * pc + j : i + j * pr;
+            grid[i * pc + j] = rank_perm ? rank_perm[r] : r;
+        }
+    return COSTA_OK;
+}

@@ -7,6 +7,8 @@
 #include <cstring>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "costa_internal.h"
 #include "tiles.h"
 
@@ -82,5 +84,22 @@ Scalars make_scalars(int dt, const void *alpha, const void *beta, int index);
 // small pieces' groups sized for them.
 cudaError_t launch_split(const RemapLaunch &base, const DevList &list, const DevList *halves, int esize,
                          const bool (&kinds)[K_NKINDS], cudaStream_t stream);
+
+// An NVTX range over a scope (plan building, the volume kernel, relabeling,
+// message and exchange plans, the enqueue of a transform, the exchange's
+// phases), visible in Nsight tools; without a tool attached the calls do
+// nothing.
+struct Trace {
+    explicit Trace(const char *name) { nvtxRangePushA(name); }
+    ~Trace() { nvtxRangePop(); }
+    Trace(const Trace &) = delete;
+    Trace &operator=(const Trace &) = delete;
+};
+
+// Host log on stderr, lines prefixed "[costa] ": COSTA_LOG=1 logs plans
+// (sizes, tiles, times, volumes), relabelings and exchange plans; 2 also
+// every transform call.  Off (0) by default.
+int log_level();
+void log_msg(int level, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
 
 }  // namespace costa

@@ -103,3 +103,19 @@ def test_study_small_instance_against_oracle():
     assert np.array_equal(V, oracle.volume("N", _spec_of_grid(A, 4), _spec_of_grid(B, 4), 4))
     _, best = costa.costa_relabel(V)
     assert best == oracle.lap_bruteforce(V)[0]
+
+
+@pytest.mark.parametrize("order", ["R", "C"])
+def test_grid_block_cyclic_matches_layout_owners(order):
+    """costa_grid_block_cyclic's grid gives, block by block, the owners of the
+    ScaLAPACK block-cyclic layout built independently in workloads.layouts."""
+    rng = gen.IntStream(9, 77)
+    for _ in range(20):
+        m, n = rng.between(1, 300), rng.between(1, 300)
+        mb, nb = rng.between(1, 40), rng.between(1, 40)
+        pr, pc = rng.between(1, 5), rng.between(1, 5)
+        perm = rng.permutation(pr * pc)
+        g = GridLayout.block_cyclic(m, n, mb, nb, pr, pc, order, perm)
+        spec = L.block_cyclic(m, n, mb, nb, pr, pc, grid_order=order, rank_perm=perm)
+        assert np.array_equal(g.rs, spec.rsplit) and np.array_equal(g.cs, spec.csplit)
+        assert np.array_equal(g.grid[np.ix_(g.rp, g.cp)], spec.owner)
