@@ -531,6 +531,18 @@ costa_status costa_debug_exchange(costa_layout A, costa_layout B, costa_op op, i
                                   uint64_t send_base, uint64_t recv_base, int which, void *out, int64_t cap,
                                   int64_t *count, int64_t *volumes);
 
+/* Diagnostics: TMA staging of the tile kernel's source tiles.  By default
+ * (environment variable COSTA_TMA unset when a plan is built) only f64 data
+ * with a beta that is neither 0 nor +-2^k uses it (measured faster there,
+ * slower for every other kind and type); COSTA_TMA=0 turns it off and
+ * COSTA_TMA=1 on for every kind and type.  Builds the plan of (A, B, op) if needed, then writes
+ * out[0] = TMA tiles in the direct list, out[1] = in its x-halves list,
+ * out[2] = tensor maps, out[3] = TMA waits that gave up in this plan's
+ * launches (each ends its warp's work and should never happen), out[4] and
+ * out[5] = the kinds (bit per combine kind) that take the TMA tiles of the
+ * two lists.  out: host, 6 int64.  Synchronizes the device. */
+costa_status costa_debug_tma(costa_layout A, costa_layout B, costa_op op, int64_t *out);
+
 /* Number of kernels this library has launched in this process. */
 int64_t costa_kernel_launch_count(void);
 

@@ -99,6 +99,7 @@ def _load():
         "costa_exchange_destroy": [P],
         "costa_relabel_placement": [I, P, I, P, ctypes.c_double, P, P, P],
         "costa_debug_exchange": [P, P, I, I, P, I, ctypes.c_uint64, ctypes.c_uint64, I, P, I64, P, P],
+        "costa_debug_tma": [P, P, I, P],
     }
     for name, args in sigs.items():
         f = getattr(lib, name)
@@ -323,6 +324,14 @@ class Exchange:
             self.destroy()
         except Exception:
             pass
+
+
+def costa_debug_tma(A: Layout, B: Layout, op: str) -> dict:
+    """TMA staging of the plan of (A, B, op) (COSTA_TMA=1 at plan time)."""
+    out = np.zeros(6, np.int64)
+    _check(_lib.costa_debug_tma(A.handle, B.handle, OPS[op], _p(out)))
+    return {"tiles": int(out[0]), "halves_tiles": int(out[1]), "maps": int(out[2]),
+            "timeouts": int(out[3]), "kinds": int(out[4]), "halves_kinds": int(out[5])}
 
 
 def costa_debug_exchange(A: Layout, B: Layout, op: str, G: int, place, g: int, send_base: int,

@@ -73,6 +73,8 @@ struct Plan {
     DevList direct_halves;              // the same with its full aligned tiles in x-halves (4- and 8-byte types)
     Scalars *d_scalars = nullptr;
     std::vector<Scalars> cached_scalars;
+    std::vector<TmaMap> tma_maps;       // tensor maps of the TMA-staged tiles (COSTA_TMA=1)
+    unsigned int *d_err = nullptr;      // TMA waits that gave up
     int64_t total_tiles = 0, total_cells = 0;
     std::vector<int64_t> V;      // P * P, V[p * P + q]
     bool sigma_done = false;
@@ -418,14 +420,38 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
         if (st != COSTA_OK) return st;
     }
     const bool cplx = plan->dtype == COSTA_C64 || plan->dtype == COSTA_C128;
-    const SplitList split = split_small(std::move(list), es, cplx);
-    const SplitOffsets off_tiles = arena.add_split(split);
+    SplitList split = split_small(std::move(list), es, cplx);
     // The aligned tiles also as x-halves (see use_halves), for the kinds
     // that run on them (see launch_list in transform_impl).
     std::vector<char> halve(static_cast<size_t>(n), 0);
     for (int k = 0; k < n; ++k) halve[k] = use_halves(plan->probs[k], es);
-    const std::vector<TileDesc> halves = split_x_halves(split.big, ts / 2, es, halve);
+    std::vector<TileDesc> halves = split_x_halves(split.big, ts / 2, es, halve);
+    const bool had_halves = !halves.empty();
+    // TMA staging (tma.cpp): for the kinds the policy picks, the qualifying
+    // aligned tiles of a list are staged by TMA and the rest by cp.async;
+    // the other kinds keep the whole list
+    const uint32_t kinds_big = tma_policy_kinds(split.big, es, cplx, false);
+    const uint32_t kinds_halves = had_halves ? tma_policy_kinds(halves, es, cplx, true) : 0;
+    std::vector<TileDesc> rest_big, tma_big, rest_halves, tma_halves;
+    {
+        std::vector<uint64_t> keys;
+        if (kinds_big) {
+            rest_big = split.big;
+            split_tma(rest_big, tma_big, plan->tma_maps, keys, es);
+        }
+        if (kinds_halves) {
+            rest_halves = halves;
+            split_tma(rest_halves, tma_halves, plan->tma_maps, keys, es);
+        }
+    }
+    const SplitOffsets off_tiles = arena.add_split(split);
     const size_t off_halves = halves.empty() ? 0 : arena.add_vec(halves);
+    const size_t off_rest = rest_big.empty() ? 0 : arena.add_vec(rest_big);
+    const size_t off_tma = tma_big.empty() ? 0 : arena.add_vec(tma_big);
+    const size_t off_rest_h = rest_halves.empty() ? 0 : arena.add_vec(rest_halves);
+    const size_t off_tma_h = tma_halves.empty() ? 0 : arena.add_vec(tma_halves);
+    const uint32_t zero_word = 0;
+    const size_t off_err = arena.add(&zero_word, sizeof zero_word);
     std::vector<VolumeProblemDev> vd(n);
     const size_t off_vd = arena.add(vd.data(), sizeof(VolumeProblemDev) * n);
     std::vector<Scalars> sc(n);
@@ -461,11 +487,31 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     ce = cudaMemcpy(d, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(plan tables)");
     plan->direct = resolve(dbase, off_tiles, split);
+    if (!tma_big.empty()) {
+        plan->direct.rtiles = reinterpret_cast<const TileDesc *>(dbase + off_rest);
+        plan->direct.nrtiles = static_cast<int64_t>(rest_big.size());
+        plan->direct.ttiles = reinterpret_cast<const TileDesc *>(dbase + off_tma);
+        plan->direct.nttiles = static_cast<int64_t>(tma_big.size());
+        plan->direct.tma_kinds = kinds_big;
+    }
     plan->direct_halves = plan->direct;
-    if (!halves.empty()) {
+    if (had_halves) {
         plan->direct_halves.tiles = reinterpret_cast<const TileDesc *>(dbase + off_halves);
         plan->direct_halves.ntiles = static_cast<int64_t>(halves.size());
+        plan->direct_halves.rtiles = nullptr;
+        plan->direct_halves.nrtiles = 0;
+        plan->direct_halves.ttiles = nullptr;
+        plan->direct_halves.nttiles = 0;
+        plan->direct_halves.tma_kinds = 0;
+        if (!tma_halves.empty()) {
+            plan->direct_halves.rtiles = reinterpret_cast<const TileDesc *>(dbase + off_rest_h);
+            plan->direct_halves.nrtiles = static_cast<int64_t>(rest_halves.size());
+            plan->direct_halves.ttiles = reinterpret_cast<const TileDesc *>(dbase + off_tma_h);
+            plan->direct_halves.nttiles = static_cast<int64_t>(tma_halves.size());
+            plan->direct_halves.tma_kinds = kinds_halves;
+        }
     }
+    plan->d_err = reinterpret_cast<unsigned int *>(dbase + off_err);
     plan->d_scalars = reinterpret_cast<Scalars *>(dbase + off_sc);
     plan->total_tiles = tiles;
     plan->total_cells = cells;
@@ -734,6 +780,11 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     L.dtype = plan->dtype;
     L.s = make_scalars(plan->dtype, alphas, betas, 0);
     L.per_problem = nullptr;
+    TmaLists tma_base{};  // the plan's tensor maps and error word (launch_split adds the tiles)
+    tma_base.maps = plan->tma_maps.empty() ? nullptr : plan->tma_maps.data();
+    tma_base.nmaps = static_cast<int32_t>(plan->tma_maps.size());
+    tma_base.err = plan->d_err;
+    L.tma = plan->tma_maps.empty() ? nullptr : &tma_base;
     bool uniform = true;
     std::vector<Scalars> sc(n);
     for (int k = 0; k < n; ++k) {
@@ -943,6 +994,9 @@ cudaError_t launch_split(const RemapLaunch &base, const DevList &list, const Dev
     RemapLaunch l = base;
     l.tiles = list.tiles;
     l.ntiles = list.ntiles;
+    l.tma = nullptr;
+    TmaLists tl{};
+    if (base.tma) tl = *base.tma;  // the plan's maps and error word
     l.mtiles = list.mtiles;
     l.nmtiles = list.nmtiles;
     l.pieces = list.pieces;
@@ -951,9 +1005,15 @@ cudaError_t launch_split(const RemapLaunch &base, const DevList &list, const Dev
     for (int kind = 0; kind < K_NKINDS; ++kind) {
         if (!kinds[kind]) continue;
         RemapLaunch lk = l;
-        if (halves && (esize == 4 || kind == K_AXPBY2)) {
-            lk.tiles = halves->tiles;
-            lk.ntiles = halves->ntiles;
+        const DevList &full = (halves && (esize == 4 || kind == K_AXPBY2)) ? *halves : list;
+        lk.tiles = full.tiles;
+        lk.ntiles = full.ntiles;
+        if (base.tma && ((full.tma_kinds >> kind) & 1u)) {  // this kind takes the TMA split
+            lk.tiles = full.rtiles;
+            lk.ntiles = full.nrtiles;
+            tl.ttiles = full.ttiles;
+            tl.nttiles = full.nttiles;
+            lk.tma = &tl;
         }
         if (kind_reads_a(kind)) {  // the groups of the kinds that read A
             lk.groups = list.groups_a;
@@ -1335,6 +1395,26 @@ costa_status costa_debug_halves(costa_layout A, costa_layout B, costa_op op, voi
     *ntiles = static_cast<int64_t>(halves.size());
     const size_t k = static_cast<size_t>(std::min<int64_t>(cap_tiles, *ntiles));
     if (k) std::memcpy(tiles, halves.data(), k * sizeof(TileDesc));
+    return COSTA_OK;
+}
+
+costa_status costa_debug_tma(costa_layout A, costa_layout B, costa_op op, int64_t *out) {
+    if (!out) return fail(COSTA_ERR_INVALID_ARG, "out is null");
+    costa_status s = validate_pair(A, B, op);
+    if (s != COSTA_OK) return s;
+    std::lock_guard<std::mutex> lock(g_mu);
+    Plan *plan = nullptr;
+    s = get_plan(1, &A, &B, &op, nullptr, plan);
+    if (s != COSTA_OK) return s;
+    unsigned int err = 0;
+    cudaError_t ce = cudaMemcpy(&err, plan->d_err, sizeof err, cudaMemcpyDeviceToHost);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(error word)");
+    out[0] = plan->direct.nttiles;
+    out[1] = plan->direct_halves.ttiles == plan->direct.ttiles ? 0 : plan->direct_halves.nttiles;
+    out[4] = plan->direct.tma_kinds;
+    out[5] = plan->direct_halves.ttiles == plan->direct.ttiles ? 0 : plan->direct_halves.tma_kinds;
+    out[2] = static_cast<int64_t>(plan->tma_maps.size());
+    out[3] = err;
     return COSTA_OK;
 }
 

@@ -120,6 +120,24 @@ COSTA_HD inline int kind_of(int32_t flags) {
 }
 
 
+// A tensor map (CUtensorMap: 128 opaque bytes, 64-byte aligned) for the
+// TMA-staged tiles; at most kMaxTmaMaps per launch, passed by value.
+struct alignas(64) TmaMap {
+    unsigned long long opaque[16];
+};
+constexpr int kMaxTmaMaps = 4;
+
+// Aligned full-size tiles whose source is staged by TMA (the TMA instance of
+// the tile kernel): each TileDesc's src holds (y << 32) | x, the byte
+// coordinates of the source's (0, 0) in tensor map sld of `maps`.
+struct TmaLists {
+    const TileDesc *ttiles;
+    int64_t nttiles;
+    const TmaMap *maps;   // host array of nmaps maps (copied into the launch)
+    int32_t nmaps;
+    unsigned int *err;    // device word: TMA waits that gave up (0 when none)
+};
+
 struct RemapLaunch {
     const TileDesc *tiles;       // aligned full-size tiles (the tile kernel)
     int64_t ntiles;
@@ -132,6 +150,10 @@ struct RemapLaunch {
     int32_t pad;
     const Scalars *per_problem;  // device array indexed by TileDesc::prob, or nullptr: use `s`
     Scalars s;
+    // host only: the TMA-staged tiles of this launch, or null.  A pointer
+    // keeps this struct (the kernels' parameter) at 120 bytes; 40 bytes more
+    // of parameters made ptxas spill more in the tile kernel.
+    const struct TmaLists *tma;
 };
 
 struct VolumeProblemDev {

@@ -25,6 +25,13 @@ struct DevList {
     int64_t ngroups = 0;
     const uint32_t *groups_a = nullptr;  // the groups of the kinds that read A
     int64_t ngroups_a = 0;
+    // TMA staging: the kinds in tma_kinds (bit per K_*) run the aligned
+    // tiles as rtiles (cp.async) + ttiles (TMA) instead of `tiles`
+    const TileDesc *rtiles = nullptr;
+    int64_t nrtiles = 0;
+    const TileDesc *ttiles = nullptr;
+    int64_t nttiles = 0;
+    uint32_t tma_kinds = 0;
     bool empty() const { return ntiles == 0 && nmtiles == 0 && ngroups == 0; }
 };
 
@@ -72,6 +79,18 @@ costa_status check_extents(const std::vector<TileDesc> &list, int es, const char
 // memory the current device `dev` can address (the rule of a single-GPU
 // transform, applied to the blocks of the ranks on one GPU).
 costa_status check_access_on(costa_layout_s *L, int dev, const char *which, const int *place, int g);
+
+// TMA staging of source tiles (COSTA_TMA=1; see tma.cpp): moves the tiles
+// of `list` that qualify into `tma`, converted to map coordinates, adding at
+// most kMaxTmaMaps maps to `maps`.  Host code; queries the driver for
+// allocation ranges.
+// COSTA_TMA: unset = the measured policy (the f64 axpby kind with a general
+// beta; see tma.cpp), 0 = never, 1 = every kind and type (for A/B
+// measurements).
+int tma_mode();
+uint32_t tma_policy_kinds(const std::vector<TileDesc> &list, int es, bool cplx, bool halves_list);
+void split_tma(std::vector<TileDesc> &list, std::vector<TileDesc> &tma, std::vector<TmaMap> &maps,
+               std::vector<uint64_t> &keys, int es);
 
 // One element type's scalars alpha[index], beta[index] read from host arrays
 // of that type, with the flags that choose the combine kind.

@@ -453,8 +453,29 @@ __device__ __forceinline__ void load_a(const Geom<T> &g, const Sc &s, Chunk<T> (
     if (KIND == K_AXPBY2) prescale<T>(av, npass, s);
 }
 
+// ---- TMA staging layout (COSTA_TMA=1; see tma.cpp) ----
+// A TMA-staged tile is boxes of 16 runs x 128 bytes: box (br, bl) (run / 16,
+// byte along the run / 128) at (br * TBL + bl) * 2048 bytes, 1024-byte
+// aligned, each a stack of 128-byte rows whose 16-byte chunks the TMA unit
+// swizzles (128-byte mode): chunk j of row r lands at j ^ (r mod 8).
+template <typename T> struct TCfg {
+    static constexpr int TBL = Cfg<T>::TS * static_cast<int>(sizeof(T)) / 128;  // boxes along a run
+    static constexpr int BUF = 2 * TBL * 2048;                                    // up to 32 runs
+    static_assert(Cfg<T>::TS * sizeof(T) % 128 == 0, "a full run is whole boxes");
+};
+template <typename T>
+__device__ __forceinline__ unsigned char *slot_t(unsigned char *buf, int r, int c) {
+    return buf + ((r >> 4) * TCfg<T>::TBL + (c >> 3)) * 2048 + (r & 15) * 128 + (((c & 7) ^ (r & 7)) << 4);
+}
+// Chunk c of staged run r in the cp.async layout (TL = false) or the TMA one.
+template <typename T, bool TL>
+__device__ __forceinline__ unsigned char *slot_any(unsigned char *buf, int r, int c) {
+    if constexpr (TL) return slot_t<T>(buf, r, c);
+    else return slot<T>(buf, r, c);
+}
+
 // Write a staged fast tile to A, combining with A when the kind reads it.
-template <typename T, int KIND>
+template <typename T, int KIND, bool TL = false>
 __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsigned char *buf,
                                             const Chunk<T> (&av)[Cfg<T>::NPASS], int lane) {
     using C = Cfg<T>;
@@ -474,9 +495,9 @@ __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsig
                 const int cy = y / C::VEC, ey = y % C::VEC;
 #pragma unroll
                 for (int e = 0; e < C::VEC; ++e)
-                    b.e[e] = reinterpret_cast<const T *>(slot<T>(buf, x0 + e, cy))[ey];
+                    b.e[e] = reinterpret_cast<const T *>(slot_any<T, TL>(buf, x0 + e, cy))[ey];
             } else {
-                b.raw = *reinterpret_cast<const uint4 *>(slot<T>(buf, y, m.c));
+                b.raw = *reinterpret_cast<const uint4 *>(slot_any<T, TL>(buf, y, m.c));
             }
             Chunk<T> o;
 #pragma unroll
@@ -1125,6 +1146,136 @@ __global__ void __launch_bounds__(KCfg<T, KIND, MIS>::WARPS * 32, KCfg<T, KIND, 
     cp_async_wait<0>();
 }
 
+// ---- the TMA instance of the tile kernel (COSTA_TMA=1) ----
+//
+// The same pipeline as the tile kernel without look-ahead, with the source
+// staged by the TMA unit instead of per-lane cp.async copies: one lane
+// issues the tile's boxes (cp.async.bulk.tensor, tensor maps passed by
+// value in the launch) on the warp's mbarrier with the expected byte count,
+// the warp loads its A chunks meanwhile, waits on the barrier's phase and
+// drains the tile from the TMA layout.  The wait gives up after a bounded
+// number of tries: it then counts the failure in args.err, waits once more
+// for its copies, and ends the warp's work (no tile is written from a
+// partial stage).
+
+__device__ __forceinline__ unsigned smem_u32(const void *p) {
+    return static_cast<unsigned>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(unsigned bar) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() { asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory"); }
+__device__ __forceinline__ void mbar_expect_tx(unsigned bar, unsigned bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(unsigned bar, unsigned parity) {
+    unsigned ok;
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// true once the barrier's phase `parity` has completed; false after the limit
+__device__ __forceinline__ bool mbar_wait(unsigned bar, unsigned parity) {
+    for (int i = 0; i < (1 << 22); ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    return false;
+}
+__device__ __forceinline__ void tma_load_2d(unsigned dst, const TmaMap *map, int x, int y, unsigned bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// Lane 0: the tile's boxes on the warp's barrier (kept out of line, so that
+// the registers of the A chunks held across the wait are not shared with
+// this loop's).
+template <typename T>
+__device__ __noinline__ void tma_issue(const Geom<T> &g, const TmaMap *map, unsigned buf, unsigned bar) {
+    const uint64_t c = reinterpret_cast<uint64_t>(g.src);
+    const int x = static_cast<int>(c & 0xffffffffu), y = static_cast<int>(c >> 32);
+    const int runs = g.transpose ? g.nx : g.ny;
+    const int nbl = (g.transpose ? g.ny : g.nx) * static_cast<int>(sizeof(T)) / 128;
+    mbar_expect_tx(bar, static_cast<unsigned>(runs * nbl * 128));
+    for (int br = 0; br < runs / 16; ++br)
+        for (int bl = 0; bl < nbl; ++bl)
+            tma_load_2d(buf + (br * TCfg<T>::TBL + bl) * 2048, map, x + bl * 128, y + br * 16, bar);
+}
+
+struct TmaLaunch {
+    RemapLaunch a;  // a.tiles / a.ntiles: the TMA tiles
+    TmaMap maps[kMaxTmaMaps];
+    unsigned int *err;
+    int32_t nmaps;
+};
+
+#ifndef COSTA_TMA_MINB_8
+#define COSTA_TMA_MINB_8 4
+#endif
+template <typename T, int KIND> struct TmaKCfg {
+    static constexpr int MINB = sizeof(T) == 16 ? 3
+                              : (sizeof(T) == 8 && COSTA_TMA_MINB_8 > 0) ? COSTA_TMA_MINB_8 : KCfg<T, KIND>::MINB;
+};
+
+template <typename T, int KIND>
+__global__ void __launch_bounds__(Cfg<T>::WARPS * 32, TmaKCfg<T, KIND>::MINB)
+    remap_tma_kernel(const __grid_constant__ TmaLaunch p) {
+    using C = Cfg<T>;
+    const RemapLaunch &args = p.a;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char *aligned = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    unsigned char *buf = aligned + warp * TCfg<T>::BUF;
+    const unsigned bar = smem_u32(aligned + C::WARPS * TCfg<T>::BUF + warp * 8);
+    if (lane == 0) {
+        mbar_init(bar);
+        mbar_fence_init();
+    }
+    __syncwarp();
+    unsigned parity = 0;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * C::WARPS;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * C::WARPS + warp;
+    Sc s;
+    int cached = -1;
+    if (!args.per_problem) make_sc(args.s, s);
+    TileStream ts;
+    ts.j = 0;
+    ts.cur = load_batch<false>(args, first, stride, 0, lane);
+    ts.nxt = load_batch<false>(args, first, stride, 1, lane);
+    Geom<T> g;
+    while (next_tile<T, KIND, false>(args, first, stride, ts, g, lane)) {
+        // g.src = (y << 32) | x: the source's (0, 0) in bytes along the run
+        // (x) and runs (y) of tensor map g.sld
+        if (g.sld < 0 || g.sld >= p.nmaps) {  // never listed by the host
+            if (lane == 0) atomicAdd(p.err, 1u);
+            continue;
+        }
+        if (lane == 0) tma_issue<T>(g, &p.maps[g.sld], smem_u32(buf), bar);
+        if (args.per_problem && g.prob != cached) {
+            make_sc(args.per_problem[g.prob], s);
+            cached = g.prob;
+        }
+        s.conj_mask = g.conj ? 0x80000000u : 0u;
+        Chunk<T> av[C::NPASS];
+        load_a<T, KIND>(g, s, av, lane);
+        if (!mbar_wait(bar, parity)) {
+            if (lane == 0) atomicAdd(p.err, 1u);
+            mbar_wait(bar, parity);
+            return;
+        }
+        parity ^= 1u;
+        stage_drain<T, KIND, true>(g, s, buf, av, lane);
+        __syncwarp();  // the buffer is free before the next tile's boxes land in it
+    }
+}
+
 inline int sm_count() {
     static int cached = 0;
     if (!cached) {
@@ -1184,6 +1335,42 @@ cudaError_t launch_small(const RemapLaunch &a, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+template <typename T, int KIND>
+cudaError_t launch_tma(const RemapLaunch &a, cudaStream_t st) {
+    const TmaLists &t = *a.tma;
+    if (!t.maps || t.nmaps < 1 || t.nmaps > kMaxTmaMaps || !t.err) return cudaErrorInvalidValue;
+    TmaLaunch p;
+    p.a = a;
+    p.a.tiles = t.ttiles;
+    p.a.ntiles = t.nttiles;
+    p.a.mtiles = nullptr;
+    p.a.nmtiles = 0;
+    p.a.ngroups = 0;
+    p.a.tma = nullptr;
+    for (int k = 0; k < kMaxTmaMaps; ++k) p.maps[k] = t.maps[k < t.nmaps ? k : 0];
+    p.err = t.err;
+    p.nmaps = t.nmaps;
+    auto kern = remap_tma_kernel<T, KIND>;
+    constexpr int kWarps = Cfg<T>::WARPS;
+    const size_t smem = 1024 + static_cast<size_t>(kWarps) * (TCfg<T>::BUF + 8);
+    static int per_sm = 0;
+    if (per_sm == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kWarps * 32, smem);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) per_sm = 1;
+    }
+    const int64_t want = (t.nttiles + kWarps - 1) / kWarps;
+    const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;
+    const int blocks = static_cast<int>(want < cap ? want : cap);
+    if (blocks <= 0) return cudaSuccess;
+    kern<<<blocks, kWarps * 32, smem, st>>>(p);
+    count_launch();
+    return cudaGetLastError();
+}
+
 // The tile kernel over the aligned full-size tiles, then over the
 // misaligned ones, then the small-tile kernel over the groups of pieces
 // (each launched only when it has work).
@@ -1193,6 +1380,7 @@ cudaError_t launch_t(const RemapLaunch &a, cudaStream_t st) {
     // theirs is aligned and their misaligned instance is not built
     if (sizeof(T) == 16 && a.nmtiles > 0) return cudaErrorInvalidValue;
     cudaError_t e = a.ntiles > 0 ? launch_tiles<T, KIND, false>(a, st) : cudaSuccess;
+    if (e == cudaSuccess && a.tma && a.tma->nttiles > 0) e = launch_tma<T, KIND>(a, st);
     if constexpr (sizeof(T) != 16)
         if (e == cudaSuccess && a.nmtiles > 0) e = launch_tiles<T, KIND, true>(a, st);
     if (e == cudaSuccess && a.ngroups > 0) e = launch_small<T, KIND>(a, st);

@@ -63,7 +63,7 @@ void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 int64_t launches_so_far() { return g_launches.load(std::memory_order_relaxed); }
 
 cudaError_t launch_remap(const RemapLaunch &a, int kind, cudaStream_t stream) {
-    if (a.ntiles <= 0 && a.nmtiles <= 0 && a.ngroups <= 0) return cudaSuccess;
+    if (a.ntiles <= 0 && a.nmtiles <= 0 && a.ngroups <= 0 && !(a.tma && a.tma->nttiles > 0)) return cudaSuccess;
     switch (a.dtype) {
     case COSTA_F32: return launch_remap_f32(a, kind, stream);
     case COSTA_F64: return launch_remap_f64(a, kind, stream);
