@@ -142,12 +142,23 @@ def c5b(rows: int = 131072, cols: int = 4096) -> Problem:
 
 
 # Further workloads for measurement only.
-EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b}
+def c2_general_beta(n: int = 8192) -> Problem:
+    """c2's layouts and op with a general beta (alpha = -0.3, beta = 0.7):
+    the combine kind whose source tiles are staged by TMA (not one of the
+    configurations above)."""
+    p = c2(n)
+    p.name = "c2g"
+    p.alpha, p.beta = -0.3, 0.7
+    return p
+
+
+EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b, "c2g": c2_general_beta}
 
 # The same layouts and tile shapes at about 1 GB on the device, for profiler
 # captures (the workloads proper stay the ones above).
 CONFIGS_SMALL = {"c1": c1, "c2": lambda: c2(4096), "c3": lambda: c3(8192),
                  "c4": lambda: c4(16), "c5": lambda: c5(rows=16384), "bc8": lambda: small_blocks(4096),
+                 "c2g": lambda: c2_general_beta(4096),
                  "c5b": lambda: c5b(rows=16384)}
 
 WORKLOAD_TEXT = {
@@ -160,6 +171,8 @@ WORKLOAD_TEXT = {
            "(small-block case, not a configuration)",
     "c5b": "131072x4096 f64 BC32 16x16 -> 4096x131072 in 256 column panels of 512, T, alpha=1 beta=1, "
            "P=256 (the other reading of c5's target)",
+    "c2g": "8192x8192 f64 BC64 4x4 -> BC128 4x4 permuted owners, T, alpha=-0.3 beta=0.7, P=16 "
+           "(c2 with a general beta: TMA-staged source tiles; not a configuration)",
 }
 
 
