@@ -134,23 +134,43 @@ template <typename T> struct Cfg {
 //    registers of 3 blocks and use a 2-deep ring; in the misaligned-tile
 //    instance the light kinds that read A (one element per lane, a whole
 //    tile of A in registers) run 4 blocks, which their registers fit
-//    without spills.
+//    without spills, and the kinds that do not (16-byte windows) a 2-deep
+//    ring at 5 blocks.
 //  - 4-byte types: the kinds that read A run 3 blocks without look-ahead,
 //    the others 2 blocks with a 2-deep ring.
 //  - 16-byte types: the kinds that read A hold a whole 16 KB tile of A in
 //    registers and run two blocks without look-ahead.
 // Overridable at build time for tuning.
+#ifndef COSTA_MIS_MINB_4
+#define COSTA_MIS_MINB_4 COSTA_MINB_4
+#endif
+#ifndef COSTA_MIS_NBUF_4
+#define COSTA_MIS_NBUF_4 COSTA_NBUF_4
+#endif
+#ifndef COSTA_MIS_MINB_8
+#define COSTA_MIS_MINB_8 COSTA_MINB_8
+#endif
+// The window path of 8-byte types keeps one tile's copies in flight ahead
+// (measured on GB300, 8192^2 T, same box, GB/s: f64 BC50 -> BC75 copy
+// 3820 -> 4101, scale 3620 -> 4162, c64 copy 3797 -> 4093; odd leading
+// dimensions -0.4 to +1%; 3 buffers at 3 blocks helped the copy to 4300 but
+// cost the scale kind 0% and the odd-ld cases up to 1.3%, 4 buffers lost
+// 20-40%).
+#ifndef COSTA_MIS_NBUF_8
+#define COSTA_MIS_NBUF_8 2
+#endif
 template <typename T, int KIND, bool MIS = false> struct KCfg {
     static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX || KIND == K_CSCALE;
     static constexpr bool READS_A = kind_reads_a(KIND);
+    static constexpr bool WIN = MIS && !READS_A;  // the window path of the misaligned instance
     static constexpr int WARPS = Cfg<T>::WARPS;
-    static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : COSTA_MINB_4)
+    static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : WIN ? COSTA_MIS_MINB_4 : COSTA_MINB_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
                               : HEAVY ? COSTA_MINB_8H
-                              : (MIS && READS_A) ? COSTA_MIS_MINB_8A : COSTA_MINB_8;
-    static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : COSTA_NBUF_4)
+                              : (MIS && READS_A) ? COSTA_MIS_MINB_8A : WIN ? COSTA_MIS_MINB_8 : COSTA_MINB_8;
+    static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : WIN ? COSTA_MIS_NBUF_4 : COSTA_NBUF_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
-                              : HEAVY ? COSTA_NBUF_8H : COSTA_NBUF_8;
+                              : HEAVY ? COSTA_NBUF_8H : WIN ? COSTA_MIS_NBUF_8 : COSTA_NBUF_8;
 };
 
 template <typename T> struct Chunk {
