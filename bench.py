@@ -714,9 +714,25 @@ def cpu_model() -> str:
     return platform.machine()
 
 
-def run_cpu_oracle(probs, seconds_target: float, threads: int | None = None):
+CPU_SAMPLE_MAX_BYTES = 2 * 10 ** 9
+
+
+def cpu_sample(workload, probs, small):
+    """The instance the CPU legs time: the workload's first instance, or,
+    when one instance moves more than 2 GB (its host matrices alone take
+    minutes to build), the same layouts at reduced size (bench --small:
+    c3 at 8192^2, c5 with 16384 of its 131072 rows)."""
+    if small or probs[0].algorithmic_bytes() <= CPU_SAMPLE_MAX_BYTES:
+        return probs, ""
+    red = problems(workload, True)
+    p = red[0]
+    return red, f"; the same layouts at reduced size: {p.A.m}x{p.A.n}"
+
+
+def run_cpu_oracle(probs, seconds_target: float, threads: int | None = None, note: str = ""):
     """The oracle, as it stands, on a bounded row slab of the first instance
-    (the same layouts and values); returns (GB/s, threads, description)."""
+    (the same layouts and values); returns (GB/s, threads, description, rows,
+    seconds per pass, B and A host matrices)."""
     import oracle
     p = probs[0]
     threads = threads or oracle.default_threads()
@@ -743,9 +759,9 @@ def run_cpu_oracle(probs, seconds_target: float, threads: int | None = None):
     dt2 = done / reps
     gbs = rows2 * per_row_bytes / dt2 / 1e9
     desc = (f"rows 0..{rows2} of A ({rows2 * p.A.n} of {p.A.m * p.A.n} elements"
-            f"{' of instance 0 of ' + str(len(probs)) if len(probs) > 1 else ''}), "
+            f"{' of instance 0 of ' + str(len(probs)) if len(probs) > 1 else ''}{note}), "
             f"{reps} pass(es), {done:.1f} s")
-    return gbs, threads, desc, rows2, dt2
+    return gbs, threads, desc, rows2, dt2, Bh, Ah
 
 
 def workload_config(args, workload, probs, world):
@@ -786,11 +802,10 @@ def reference_arm(args, probs):
     per_step = max(0.5, min(10.0, 150.0 / (steps + warmup)))
     import oracle
     threads = oracle.default_threads()
-    gbs, threads, desc, rows, dt = run_cpu_oracle(probs, per_step)
+    probs, note = cpu_sample(args.workload, probs, args.small)
+    gbs, threads, desc, rows, dt, Bh, Ah = run_cpu_oracle(probs, per_step, note=note)
     p = probs[0]
     per_row_bytes = p.A.n * p.esize * (3 if p.beta != 0 else 2)
-    Bh = HostMatrix(p.B, p.dtype).fill(p.b_kind, p.seed, p.src_stream)
-    Ah = HostMatrix(p.A, p.dtype).fill(p.a_kind, p.seed, p.tgt_stream)
     for _ in range(warmup):
         oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, Ah.buffers(), p.B,
                          Bh.buffers(), rows=(0, rows), threads=threads)
@@ -824,11 +839,12 @@ def measure(args, workload, rank, world, local_rank):
     r = (run_exchange if use_x else run_gpu)(args, workload, rank, world, local_rank)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        gbs, threads, desc, _, _ = run_cpu_oracle(probs, args.cpu_seconds)
+        cprobs, note = cpu_sample(workload, probs, args.small)
+        gbs, threads, desc, _, _, _, _ = run_cpu_oracle(cprobs, args.cpu_seconds, note=note)
         cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
                "sample": desc, "cpu_model": cpu_model()}
         if workload in ("c1", "c2"):  # the single-threaded figure as well
-            gbs1, _, desc1, _, _ = run_cpu_oracle(probs, min(3.0, args.cpu_seconds), threads=1)
+            gbs1, _, desc1, _, _, _, _ = run_cpu_oracle(cprobs, min(3.0, args.cpu_seconds), threads=1)
             cpu["single_thread"] = {"value": round(gbs1, 4), "unit": "GB/s", "sample": desc1}
     gc.collect()
     torch.cuda.empty_cache()
