@@ -26,6 +26,9 @@
  *  - Plans: the first transform of a (layouts, op, relabel) combination
  *    builds a plan (grid overlay, volumes, relabeling, tile lists; see
  *    costa_plan_stats) and caches it.  Building a plan synchronizes `stream`.
+ *    The TMA-staged tile lists of a plan (real f64 elements, general beta)
+ *    are built by the first call of that kind, with synchronous copies; a
+ *    call made under stream capture before then uses the cp.async lists.
  *    Plans are freed when one of their layouts is destroyed or by
  *    costa_release_plans().
  *  - Concurrency: every call on one layout pair (A, B) uses the same cached

@@ -73,8 +73,13 @@ struct Plan {
     DevList direct_halves;              // the same with its full aligned tiles in x-halves (4- and 8-byte types)
     Scalars *d_scalars = nullptr;
     std::vector<Scalars> cached_scalars;
-    std::vector<TmaMap> tma_maps;       // tensor maps of the TMA-staged tiles (COSTA_TMA=1)
+    std::vector<TmaMap> tma_maps;       // tensor maps of the TMA-staged tiles
     unsigned int *d_err = nullptr;      // TMA waits that gave up
+    // TMA staging (tma.cpp): the kinds that would use it, per list; the
+    // lists are built by the first call of such a kind (ensure_tma)
+    uint32_t tma_kinds_big = 0, tma_kinds_halves = 0;
+    bool tma_built = false;
+    void *d_tma = nullptr;
     int64_t total_tiles = 0, total_cells = 0;
     std::vector<int64_t> V;      // P * P, V[p * P + q]
     bool sigma_done = false;
@@ -95,6 +100,7 @@ struct Plan {
             if (m.d_staging) cudaFree(m.d_staging);
         }
         if (d_mem) cudaFree(d_mem);
+        if (d_tma) cudaFree(d_tma);
         if (scratch_done) cudaEventDestroy(scratch_done);
     }
 };
@@ -427,29 +433,12 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     for (int k = 0; k < n; ++k) halve[k] = use_halves(plan->probs[k], es);
     std::vector<TileDesc> halves = split_x_halves(split.big, ts / 2, es, halve);
     const bool had_halves = !halves.empty();
-    // TMA staging (tma.cpp): for the kinds the policy picks, the qualifying
-    // aligned tiles of a list are staged by TMA and the rest by cp.async;
-    // the other kinds keep the whole list
-    const uint32_t kinds_big = tma_policy_kinds(split.big, es, cplx, false);
-    const uint32_t kinds_halves = had_halves ? tma_policy_kinds(halves, es, cplx, true) : 0;
-    std::vector<TileDesc> rest_big, tma_big, rest_halves, tma_halves;
-    {
-        std::vector<uint64_t> keys;
-        if (kinds_big) {
-            rest_big = split.big;
-            split_tma(rest_big, tma_big, plan->tma_maps, keys, es);
-        }
-        if (kinds_halves) {
-            rest_halves = halves;
-            split_tma(rest_halves, tma_halves, plan->tma_maps, keys, es);
-        }
-    }
+    // TMA staging (tma.cpp): the kinds the policy would give it; their lists
+    // are built by the first call of such a kind (ensure_tma)
+    plan->tma_kinds_big = tma_policy_kinds(split.big, es, cplx, false);
+    plan->tma_kinds_halves = had_halves ? tma_policy_kinds(halves, es, cplx, true) : 0;
     const SplitOffsets off_tiles = arena.add_split(split);
     const size_t off_halves = halves.empty() ? 0 : arena.add_vec(halves);
-    const size_t off_rest = rest_big.empty() ? 0 : arena.add_vec(rest_big);
-    const size_t off_tma = tma_big.empty() ? 0 : arena.add_vec(tma_big);
-    const size_t off_rest_h = rest_halves.empty() ? 0 : arena.add_vec(rest_halves);
-    const size_t off_tma_h = tma_halves.empty() ? 0 : arena.add_vec(tma_halves);
     const uint32_t zero_word = 0;
     const size_t off_err = arena.add(&zero_word, sizeof zero_word);
     std::vector<VolumeProblemDev> vd(n);
@@ -487,29 +476,10 @@ costa_status build_plan(int n, const costa_layout *As, const costa_layout *Bs, c
     ce = cudaMemcpy(d, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
     if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(plan tables)");
     plan->direct = resolve(dbase, off_tiles, split);
-    if (!tma_big.empty()) {
-        plan->direct.rtiles = reinterpret_cast<const TileDesc *>(dbase + off_rest);
-        plan->direct.nrtiles = static_cast<int64_t>(rest_big.size());
-        plan->direct.ttiles = reinterpret_cast<const TileDesc *>(dbase + off_tma);
-        plan->direct.nttiles = static_cast<int64_t>(tma_big.size());
-        plan->direct.tma_kinds = kinds_big;
-    }
     plan->direct_halves = plan->direct;
     if (had_halves) {
         plan->direct_halves.tiles = reinterpret_cast<const TileDesc *>(dbase + off_halves);
         plan->direct_halves.ntiles = static_cast<int64_t>(halves.size());
-        plan->direct_halves.rtiles = nullptr;
-        plan->direct_halves.nrtiles = 0;
-        plan->direct_halves.ttiles = nullptr;
-        plan->direct_halves.nttiles = 0;
-        plan->direct_halves.tma_kinds = 0;
-        if (!tma_halves.empty()) {
-            plan->direct_halves.rtiles = reinterpret_cast<const TileDesc *>(dbase + off_rest_h);
-            plan->direct_halves.nrtiles = static_cast<int64_t>(rest_halves.size());
-            plan->direct_halves.ttiles = reinterpret_cast<const TileDesc *>(dbase + off_tma_h);
-            plan->direct_halves.nttiles = static_cast<int64_t>(tma_halves.size());
-            plan->direct_halves.tma_kinds = kinds_halves;
-        }
     }
     plan->d_err = reinterpret_cast<unsigned int *>(dbase + off_err);
     plan->d_scalars = reinterpret_cast<Scalars *>(dbase + off_sc);
@@ -570,6 +540,66 @@ costa_status ensure_sigma(Plan &plan) {
             plan.stats.relabel_ms);
     plan.stats.local_relabeled = best;
     plan.sigma_done = true;
+    return COSTA_OK;
+}
+
+// The TMA split of the aligned lists (tma.cpp) for the kinds that use it,
+// built by the first call that needs it: the lists come back from the
+// device, are split, and go up again in an allocation of their own, with
+// synchronous copies.  Plans of other kinds never pay for it.
+costa_status ensure_tma(Plan &plan) {
+    if (plan.tma_built) return COSTA_OK;
+    plan.tma_built = true;
+    if (!plan.tma_kinds_big && !plan.tma_kinds_halves) return COSTA_OK;
+    Trace trace("costa tma lists");
+    const int es = plan.esize;
+    const bool halves = plan.direct_halves.tiles != plan.direct.tiles;
+    std::vector<TileDesc> big(static_cast<size_t>(plan.direct.ntiles));
+    std::vector<TileDesc> hv(halves && plan.tma_kinds_halves ? static_cast<size_t>(plan.direct_halves.ntiles) : 0);
+    cudaError_t ce = cudaSuccess;
+    if (plan.tma_kinds_big && !big.empty())
+        ce = cudaMemcpy(big.data(), plan.direct.tiles, sizeof(TileDesc) * big.size(), cudaMemcpyDeviceToHost);
+    if (ce == cudaSuccess && !hv.empty())
+        ce = cudaMemcpy(hv.data(), plan.direct_halves.tiles, sizeof(TileDesc) * hv.size(), cudaMemcpyDeviceToHost);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(tile lists)");
+    std::vector<TileDesc> tma_big, tma_hv;
+    std::vector<uint64_t> keys;
+    if (plan.tma_kinds_big) split_tma(big, tma_big, plan.tma_maps, keys, es);
+    if (!hv.empty()) split_tma(hv, tma_hv, plan.tma_maps, keys, es);
+    if (tma_big.empty() && tma_hv.empty()) return COSTA_OK;
+    Arena arena;
+    const size_t o_rb = arena.add_vec(big), o_tb = arena.add_vec(tma_big);
+    const size_t o_rh = arena.add_vec(hv), o_th = arena.add_vec(tma_hv);
+    ce = cudaMalloc(&plan.d_tma, arena.host.size());
+    if (ce != cudaSuccess) {
+        plan.d_tma = nullptr;
+        return fail(COSTA_ERR_ALLOC, "cudaMalloc(TMA tile lists): %s", cudaGetErrorString(ce));
+    }
+    ce = cudaMemcpy(plan.d_tma, arena.host.data(), arena.host.size(), cudaMemcpyHostToDevice);
+    if (ce != cudaSuccess) return cuda_fail(ce, "cudaMemcpy(TMA tile lists)");
+    const char *db = static_cast<const char *>(plan.d_tma);
+    if (!tma_big.empty()) {
+        DevList &d = plan.direct;
+        d.rtiles = reinterpret_cast<const TileDesc *>(db + o_rb);
+        d.nrtiles = static_cast<int64_t>(big.size());
+        d.ttiles = reinterpret_cast<const TileDesc *>(db + o_tb);
+        d.nttiles = static_cast<int64_t>(tma_big.size());
+        d.tma_kinds = plan.tma_kinds_big;
+    }
+    DevList &h = plan.direct_halves;
+    if (!halves) {  // the halves list is the direct list
+        const DevList tiles_only = h;
+        h = plan.direct;
+        h.tiles = tiles_only.tiles;
+        h.ntiles = tiles_only.ntiles;
+    } else if (!tma_hv.empty()) {
+        h.rtiles = reinterpret_cast<const TileDesc *>(db + o_rh);
+        h.nrtiles = static_cast<int64_t>(hv.size());
+        h.ttiles = reinterpret_cast<const TileDesc *>(db + o_th);
+        h.nttiles = static_cast<int64_t>(tma_hv.size());
+        h.tma_kinds = plan.tma_kinds_halves;
+    }
+    log_msg(1, "TMA lists: %zu + %zu tiles, %zu map(s)", tma_big.size(), tma_hv.size(), plan.tma_maps.size());
     return COSTA_OK;
 }
 
@@ -780,16 +810,24 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
     L.dtype = plan->dtype;
     L.s = make_scalars(plan->dtype, alphas, betas, 0);
     L.per_problem = nullptr;
-    TmaLists tma_base{};  // the plan's tensor maps and error word (launch_split adds the tiles)
-    tma_base.maps = plan->tma_maps.empty() ? nullptr : plan->tma_maps.data();
-    tma_base.nmaps = static_cast<int32_t>(plan->tma_maps.size());
-    tma_base.err = plan->d_err;
-    L.tma = plan->tma_maps.empty() ? nullptr : &tma_base;
     bool uniform = true;
     std::vector<Scalars> sc(n);
     for (int k = 0; k < n; ++k) {
         sc[k] = make_scalars(plan->dtype, alphas, betas, k);
         if (!same_scalars(sc[k], sc[0])) uniform = false;
+    }
+    // one launch per combine kind present in the batch
+    bool kinds[K_NKINDS] = {};
+    for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
+    if (!plan->tma_built && mode == COSTA_MODE_DIRECT) {
+        bool want = false;
+        for (int kind = 0; kind < K_NKINDS; ++kind)
+            want |= kinds[kind] && (((plan->tma_kinds_big | plan->tma_kinds_halves) >> kind) & 1u);
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (want && cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone) {
+            s = ensure_tma(*plan);  // under capture the cp.async lists serve
+            if (s != COSTA_OK) return s;
+        }
     }
     // the calls that use the plan's scratch are ordered (Plan::scratch_done)
     const bool uses_scratch = !uniform || mode == COSTA_MODE_MESSAGE;
@@ -818,9 +856,11 @@ costa_status transform_impl(int n, const costa_layout *A, const costa_layout *B,
         }
         L.per_problem = plan->d_scalars;
     }
-    // one launch per combine kind present in the batch
-    bool kinds[K_NKINDS] = {};
-    for (int k = 0; k < n; ++k) kinds[kind_of(sc[k].flags)] = true;
+    TmaLists tma_base{};  // the plan's tensor maps and error word (launch_split adds the tiles)
+    tma_base.maps = plan->tma_maps.empty() ? nullptr : plan->tma_maps.data();
+    tma_base.nmaps = static_cast<int32_t>(plan->tma_maps.size());
+    tma_base.err = plan->d_err;
+    L.tma = plan->tma_maps.empty() ? nullptr : &tma_base;
     // halves: the list for the kinds that run on x-halves (null: none)
     auto launch_list = [&](const DevList &list, const DevList *halves) -> cudaError_t {
         return launch_split(L, list, halves, plan->esize, kinds, stream);
@@ -1405,6 +1445,7 @@ costa_status costa_debug_tma(costa_layout A, costa_layout B, costa_op op, int64_
     std::lock_guard<std::mutex> lock(g_mu);
     Plan *plan = nullptr;
     s = get_plan(1, &A, &B, &op, nullptr, plan);
+    if (s == COSTA_OK) s = ensure_tma(*plan);
     if (s != COSTA_OK) return s;
     unsigned int err = 0;
     cudaError_t ce = cudaMemcpy(&err, plan->d_err, sizeof err, cudaMemcpyDeviceToHost);
