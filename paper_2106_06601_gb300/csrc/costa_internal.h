@@ -83,7 +83,7 @@ struct TileDesc {
     uint16_t flags;  // TF_*
 };
 static_assert(sizeof(TileDesc) == 32, "TileDesc layout");
-enum : uint16_t { TF_TRANSPOSE = 1, TF_FAST = 2, TF_CONJ = 4 };
+enum : uint16_t { TF_TRANSPOSE = 1, TF_FAST = 2, TF_CONJ = 4, TF_ELEM = 8 };
 
 // Scalars of one problem, as doubles ({re, im}); float data carries values
 // that are exactly representable in float.

@@ -328,7 +328,7 @@ template <typename T> struct Geom {
     int64_t dld, sld;
     int nx, ny;
     int prob;
-    bool transpose, fast, conj;
+    bool transpose, fast, conj, elem;
 };
 
 // Chunk c of staged row r lives in slot c ^ swz(r): across the VEC rows that
@@ -680,21 +680,74 @@ __device__ __forceinline__ Chunk<T> staged_window(const Geom<T> &g, unsigned cha
 }
 
 // Writes the tile columns of x0 .. x0 + VEC - 1 (a window chunk of tile row
-// y) that lie in [0, nx): with one 16-byte store when all do (FULL).
-template <typename T, int KIND, bool FULL>
-__device__ __forceinline__ void drain_window(const Geom<T> &g, const Sc &s, unsigned char *buf, int x0, int y) {
+// y) that lie in [0, nx), element by element.
+template <typename T, int KIND>
+__device__ __forceinline__ void drain_partial_w(const Geom<T> &g, const Sc &s, unsigned char *buf, int x0, int y) {
     using C = Cfg<T>;
     const Chunk<T> b = staged_window<T>(g, buf, x0, y);
-    Chunk<T> o;
-#pragma unroll
-    for (int i = 0; i < C::VEC; ++i) o.e[i] = combine<KIND>(b.e[i], T(), s);
     T *row = g.dst + static_cast<int64_t>(y) * g.dld;
-    if constexpr (FULL) {
-        store(row + x0, o);
-    } else {
 #pragma unroll
-        for (int i = 0; i < C::VEC; ++i)
-            if (x0 + i >= 0 && x0 + i < g.nx) row[x0 + i] = o.e[i];
+    for (int i = 0; i < C::VEC; ++i)
+        if (x0 + i >= 0 && x0 + i < g.nx) row[x0 + i] = combine<KIND>(b.e[i], T(), s);
+}
+
+// The full window chunks of one lane: tile columns x0 .. x0 + VEC - 1 (all
+// inside the tile) of rows r0, r0 + rpp, ...  rpp is a multiple of VEC, so
+// every staged run the lane reads keeps its phase and its offset within a
+// chunk from pass to pass: they are computed once, and a pass advances the
+// staged chunk index only.
+template <typename T, int KIND>
+__device__ __forceinline__ void drain_full_w(const Geom<T> &g, const Sc &s, unsigned char *buf, int x0, int r0,
+                                             int rpp) {
+    using C = Cfg<T>;
+    constexpr int V = C::VEC, ES = static_cast<int>(sizeof(T)), ROW = C::CPR * 16;
+    T *d = g.dst + static_cast<int64_t>(r0) * g.dld + x0;
+    const int64_t dstep = static_cast<int64_t>(rpp) * g.dld;
+    if (g.transpose) {
+        // element (x0 + e, y): staged run x0 + e, window position ph + y
+        const int dj = rpp / V;
+        int j0[V], sw[V], off[V], xo[V];
+#pragma unroll
+        for (int e = 0; e < V; ++e) {
+            const int x = x0 + e, q = phase<T>(g.src, g.sld, x) + r0;
+            j0[e] = q / V;
+            sw[e] = swz<T>(x);
+            off[e] = x * ROW + (q % V) * ES;
+            xo[e] = WCfg<T>::XCOL + x * 16 + (q % V) * ES;
+        }
+#pragma unroll 4
+        for (int p = 0, y = r0; y < g.ny; ++p, y += rpp) {
+            Chunk<T> b, o;
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+                const int j = j0[e] + p * dj;
+                b.e[e] = *reinterpret_cast<const T *>(buf + (j < C::CPR ? off[e] + ((j ^ sw[e]) << 4) : xo[e]));
+            }
+#pragma unroll
+            for (int e = 0; e < V; ++e) o.e[e] = combine<KIND>(b.e[e], T(), s);
+            store(d, o);
+            d += dstep;
+        }
+    } else {
+        // row y: staged run y, window positions q .. q + VEC - 1 (chunk j
+        // from element w, then chunk j + 1)
+        const int q = phase<T>(g.src, g.sld, r0) + x0, j = q / V, w = q % V;
+#pragma unroll 4
+        for (int y = r0; y < g.ny; y += rpp) {
+            const int sw = swz<T>(y);
+            const int o0 = j < C::CPR ? y * ROW + ((j ^ sw) << 4) : WCfg<T>::XCOL + y * 16;
+            const int o1 = j + 1 < C::CPR ? y * ROW + (((j + 1) ^ sw) << 4) : WCfg<T>::XCOL + y * 16;
+            Chunk<T> b, o;
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+                const int k = w + e;
+                b.e[e] = *reinterpret_cast<const T *>(buf + (k < V ? o0 + k * ES : o1 + (k - V) * ES));
+            }
+#pragma unroll
+            for (int e = 0; e < V; ++e) o.e[e] = combine<KIND>(b.e[e], T(), s);
+            store(d, o);
+            d += dstep;
+        }
     }
 }
 
@@ -709,15 +762,14 @@ __device__ __forceinline__ void stage_drain_w(const Geom<T> &g, const Sc &s, uns
     const LaneMap m = lane_map(cm, lane);
     const int x0 = m.c * C::VEC - phase<T>(g.dst, g.dld, m.r0);  // first tile column of the lane's chunk
     if (m.c < cm && x0 >= 0 && x0 + C::VEC <= g.nx) {
-#pragma unroll 4
-        for (int y = m.r0; y < g.ny; y += m.rpp) drain_window<T, KIND, true>(g, s, buf, x0, y);
+        drain_full_w<T, KIND>(g, s, buf, x0, m.r0, m.rpp);
     }
     if (lane < g.ny) {
         const int ph = phase<T>(g.dst, g.dld, lane);
         const int last = (ph + g.nx - 1) / C::VEC;  // last window chunk of the row
         const int xl = last * C::VEC - ph;
-        if (ph > 0) drain_window<T, KIND, false>(g, s, buf, -ph, lane);
-        if (xl + C::VEC > g.nx && (last > 0 || ph == 0)) drain_window<T, KIND, false>(g, s, buf, xl, lane);
+        if (ph > 0) drain_partial_w<T, KIND>(g, s, buf, -ph, lane);
+        if (xl + C::VEC > g.nx && (last > 0 || ph == 0)) drain_partial_w<T, KIND>(g, s, buf, xl, lane);
     }
 }
 
@@ -788,6 +840,19 @@ __device__ __forceinline__ void stage_drain_e(const Geom<T> &g, const Sc &s, uns
             const T b = g.transpose ? *slot_e<T>(buf, m.c, y) : *slot_e<T>(buf, y, m.c);
             g.dst[static_cast<int64_t>(y) * g.dld + m.c] = combine<KIND>(b, elem<T>(av, p), s);
         }
+    }
+}
+
+// stage_drain_e for the kinds that do not read A.
+template <typename T, int KIND>
+__device__ __forceinline__ void stage_drain_e1(const Geom<T> &g, const Sc &s, unsigned char *buf, int lane) {
+    static_assert(!kind_reads_a(KIND), "kinds that read A hold A in registers");
+    const LaneMap m = lane_map(g.nx, lane);
+    if (m.c >= g.nx) return;
+#pragma unroll 4
+    for (int y = m.r0; y < g.ny; y += m.rpp) {
+        const T b = g.transpose ? *slot_e<T>(buf, m.c, y) : *slot_e<T>(buf, y, m.c);
+        g.dst[static_cast<int64_t>(y) * g.dld + m.c] = combine<KIND>(b, T(), s);
     }
 }
 
@@ -865,6 +930,7 @@ template <typename T> __device__ __forceinline__ Geom<T> geom_of(const TileDesc 
     g.transpose = (d.flags & TF_TRANSPOSE) != 0;
     g.fast = (d.flags & TF_FAST) != 0;
     g.conj = ET<T>::CPLX && (d.flags & TF_CONJ) != 0;
+    g.elem = (d.flags & TF_ELEM) != 0;
     return g;
 }
 
@@ -1066,7 +1132,10 @@ __global__ void __launch_bounds__(SCfg<T, KIND>::WARPS * 32, SCfg<T, KIND>::MINB
 template <typename T, int KIND, bool MIS>
 __device__ __forceinline__ void stage_any(const Geom<T> &g, unsigned char *buf, int lane) {
     if constexpr (MIS && KCfg<T, KIND>::READS_A) stage_issue_e<T>(g, buf, lane);
-    else if constexpr (MIS) stage_issue_w<T>(g, buf, lane);
+    else if constexpr (MIS) {
+        if (sizeof(T) == 4 && g.elem) stage_issue_e<T>(g, buf, lane);  // the host flags 4-byte tiles only
+        else stage_issue_w<T>(g, buf, lane);
+    }
     else if (g.fast) stage_issue<T>(g, buf, lane);  // the element-wise fallback stages nothing
 }
 
@@ -1090,7 +1159,8 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
     } else if constexpr (MIS) {
         cp_async_wait<NB - 1>();
         __syncwarp();
-        stage_drain_w<T, KIND>(g, s, buf, lane);
+        if (sizeof(T) == 4 && g.elem) stage_drain_e1<T, KIND>(g, s, buf, lane);
+        else stage_drain_w<T, KIND>(g, s, buf, lane);
     } else if (g.fast) {
         Chunk<T> av[C::NPASS];
         load_a<T, KIND>(g, s, av, lane);

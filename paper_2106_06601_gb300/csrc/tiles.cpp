@@ -193,6 +193,20 @@ SplitList split_small(std::vector<TileDesc> &&all, int es, bool cplx) {
             list.reserve(all.size() - nmis);
             out.mis.reserve(nmis);
             for (const TileDesc &d : all) ((d.flags & TF_FAST) ? list : out.mis).push_back(d);
+            // 4-byte tiles whose target runs are misaligned take the
+            // one-element-per-lane path in every kind (TF_ELEM): one warp
+            // store then writes a whole target run, the partial 32-byte
+            // sectors at its ends included, where the window path writes
+            // the partial chunks in a second pass.  Measured on GB300,
+            // 8192^2 T copy, BC64 -> BC128, GB/s window -> element: A's ld
+            // = 1 mod 4 3586 -> 4320 (N: 3695 -> 4378), both lds odd 3675 ->
+            // 4380, BC50 -> BC75 2235 -> 2455; B's ld odd alone 5300 ->
+            // 4760 (so the window path keeps it); 8-byte types lose 5-15%.
+            if (es == 4) {
+                for (TileDesc &d : out.mis)
+                    if (!aligned16(d.dst, static_cast<int64_t>(d.dld) * es) || d.nx % 4 != 0)
+                        d.flags = static_cast<uint16_t>(d.flags | TF_ELEM);
+            }
         }
     }
     const int64_t n = static_cast<int64_t>(list.size());

@@ -238,6 +238,13 @@ def check_split(p, exact=False):
         LB.destroy()
     area = lambda t: int((t["nx"].astype(np.int64) * t["ny"].astype(np.int64)).sum())
     assert area(big) + area(pieces) == p.A.m * p.A.n == area(whole)
+    # the one-element-per-lane flag: only on misaligned 4-byte tiles whose
+    # target runs are off 16-byte boundaries, and on all of those
+    assert not np.any(whole["flags"] & 8) and not np.any(pieces["flags"] & 8)
+    fast = (big["flags"] & 2) != 0
+    elem = (big["flags"] & 8) != 0
+    a_mis = ((big["dst"] % 16) != 0) | ((big["dld"].astype(np.int64) * es) % 16 != 0) | (big["nx"] % 4 != 0)
+    assert np.array_equal(elem, ~fast & a_mis if es == 4 else np.zeros_like(fast))
     if len(pieces):
         nx, ny = pieces["nx"].astype(np.int64), pieces["ny"].astype(np.int64)
         tr = (pieces["flags"] & 1) != 0

@@ -1,8 +1,8 @@
 """CPU check of the index arithmetic of the misaligned-tile paths: the
-16-byte window path (`stage_issue_w`, `stage_drain_w` in the remap kernel
-source) and the one-element-per-lane path of the kinds that read A
-(`stage_issue_e`, `load_a_e`, `stage_drain_e`), replayed per lane for random
-tiles before any kernel runs them.
+16-byte window path (`stage_issue_w`, `stage_drain_w`, `drain_full_w` in the
+remap kernel source) and the one-element-per-lane path (`stage_issue_e`,
+`load_a_e`, `stage_drain_e`, and `stage_drain_e1` for the kinds that do not
+read A), replayed per lane for random tiles before any kernel runs them.
 
 For a tile of nx x ny elements (nx, ny <= 32), transposed or not, with any
 element-aligned start addresses and leading dimensions of source and target,
@@ -99,15 +99,39 @@ def replay(es, rnd):
                 assert (y, x0 + i) not in written
                 written.add((y, x0 + i))
 
-    # stage_drain_w
+    def hoisted(x0, r0, rpp, p, y):
+        """drain_full_w's staged offsets for pass p (row y), per element."""
+        row = cpr * 16
+        if tr:
+            out = []
+            for e in range(vec):
+                x = x0 + e
+                q = phase(src, sld, x) + r0
+                j = q // vec + p * (rpp // vec)
+                off = x * row + (q % vec) * es
+                out.append(off + ((j ^ ((x // vec) & 7)) << 4) if j < cpr else xcol + x * 16 + (q % vec) * es)
+            return out
+        q = phase(src, sld, r0) + x0
+        j, w = q // vec, q % vec
+        sw = (y // vec) & 7
+        o0 = y * row + ((j ^ sw) << 4) if j < cpr else xcol + y * 16
+        o1 = y * row + (((j + 1) ^ sw) << 4) if j + 1 < cpr else xcol + y * 16
+        return [o0 + (w + e) * es if w + e < vec else o1 + (w + e - vec) * es for e in range(vec)]
+
+    # stage_drain_w: full chunks (drain_full_w)
     cmd = wmain(nx)
     for lane in range(32):
         c, r0, rpp = lane_map(cmd, lane)
         x0 = c * vec - phase(dst, dld, r0)
         if c < cmd and x0 >= 0 and x0 + vec <= nx:
-            for y in range(r0, ny, rpp):
+            for p, y in enumerate(range(r0, ny, rpp)):
                 assert c * vec - phase(dst, dld, y) == x0
+                want = [welem(x0 + e, phase(src, sld, x0 + e) + y) if tr else welem(y, phase(src, sld, y) + x0 + e)
+                        for e in range(vec)]
+                assert hoisted(x0, r0, rpp, p, y) == want
                 drain(x0, y, True)
+    # partial chunks (drain_partial_w): lane = tile row
+    for lane in range(32):
         if lane < ny:
             ph = phase(dst, dld, lane)
             last = (ph + nx - 1) // vec
@@ -200,6 +224,17 @@ def replay_elements(es, rnd):
             stored.append(a)
     assert len(stored) == len(set(stored)) and set(stored) == every
     assert len(loaded) == len(set(loaded)) and set(loaded) == every
+    # stage_drain_e1 (kinds that do not read A): rows r0, r0 + rpp, ...
+    stored1 = []
+    for lane in range(32):
+        c, r0, rpp = lane_map(nx, lane)
+        if c >= nx:
+            continue
+        for y in range(r0, ny, rpp):
+            want = src + ((c * sld + y) if tr else (y * sld + c)) * es
+            assert smem.get(slot_e(c, y) if tr else slot_e(y, c)) == want
+            stored1.append(target(y, c))
+    assert len(stored1) == len(set(stored1)) and set(stored1) == every
 
 
 @pytest.mark.parametrize("es", [4, 8])
