@@ -1174,8 +1174,9 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
 }
 
 // The tile kernel.  MIS = false moves the aligned ("fast") tiles of
-// args.tiles with 16-byte chunks; MIS = true moves the misaligned tiles of
-// args.mtiles (see "misaligned tiles" above).  The host puts every tile in
+// args.tiles with 16-byte chunks; MIS = true moves the tiles of args.mtiles
+// (see "misaligned tiles" above): the misaligned ones and, in a list that
+// is mostly misaligned, the aligned ones too, which its paths also move.  The host puts every tile in
 // the right list, so no 16-byte access is ever made at a misaligned
 // address.
 template <typename T, int KIND, bool MIS>
