@@ -135,7 +135,7 @@ template <typename T> struct Cfg {
 //    instance the light kinds that read A (one element per lane, a whole
 //    tile of A in registers) run 4 blocks, which their registers fit
 //    without spills, and the kinds that do not (16-byte windows) a 2-deep
-//    ring at 5 blocks.
+//    ring (shared memory then holds 3 blocks of 4 warps).
 //  - 4-byte types: the kinds that read A run 3 blocks without look-ahead,
 //    the others 2 blocks with a 2-deep ring.
 //  - 16-byte types: the kinds that read A hold a whole 16 KB tile of A in
@@ -153,9 +153,11 @@ template <typename T> struct Cfg {
 // The window path of 8-byte types keeps one tile's copies in flight ahead
 // (measured on GB300, 8192^2 T, same box, GB/s: f64 BC50 -> BC75 copy
 // 3820 -> 4101, scale 3620 -> 4162, c64 copy 3797 -> 4093; odd leading
-// dimensions -0.4 to +1%; 3 buffers at 3 blocks helped the copy to 4300 but
-// cost the scale kind 0% and the odd-ld cases up to 1.3%, 4 buffers lost
-// 20-40%).
+// dimensions -0.4 to +1%; 3 buffers (2 blocks fit) helped the copy to 4300
+// but cost the scale kind 0% and the odd-ld cases up to 1.3%, 4 buffers
+// lost 20-40%).  An 8-byte window buffer is 8.5 KB, so shared memory, not
+// the register bound, sets the blocks per SM: 6 blocks with 1 buffer, 3
+// with 2, 2 with 3.
 #ifndef COSTA_MIS_NBUF_8
 #define COSTA_MIS_NBUF_8 2
 #endif
