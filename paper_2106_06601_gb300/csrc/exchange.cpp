@@ -180,7 +180,7 @@ costa_status plan_exchange(const costa_layout_s *A, const costa_layout_s *B, int
     // The lists that write A take the direct path's order in the target's
     // own storage where that one does (the offsets above are fixed already,
     // so this changes only which tiles are in flight together).
-    if (use_local_order(ph))
+    if (use_local_order(ph, out.local.data(), out.local.size()))
         for (std::vector<TileDesc> *l : {&out.local, &out.unpack}) {
             bool contiguous = true;
             for (size_t i = 0; i < l->size() && contiguous; ++i) contiguous = (*l)[i].nx == (*l)[i].dld;

@@ -180,6 +180,19 @@ std::vector<TileDesc> split_x_halves(const std::vector<TileDesc> &list, int hx, 
     return out;
 }
 
+bool mostly_misaligned(const TileDesc *tiles, size_t n, int es, bool target_only) {
+    int64_t mis = 0, all = 0;
+    for (size_t i = 0; i < n; ++i) {
+        const TileDesc &d = tiles[i];
+        const int64_t e = static_cast<int64_t>(d.nx) * d.ny;
+        all += e;
+        const bool m = target_only ? !aligned16(d.dst, static_cast<int64_t>(d.dld) * es) || d.nx % (16 / es) != 0
+                                   : !(d.flags & TF_FAST);
+        if (m) mis += e;
+    }
+    return n > 0 && 2 * mis >= all;
+}
+
 SplitList split_small(std::vector<TileDesc> &&all, int es, bool cplx) {
     SplitList out;
     // misaligned tiles go to their own instance of the tile kernel
@@ -199,13 +212,7 @@ SplitList split_small(std::vector<TileDesc> &&all, int es, bool cplx) {
             // GB300, 8192^2 T, BC50 -> BC75 (88% of the elements
             // misaligned), GB/s two launches -> one: f64 copy 4255 -> 4606,
             // scale 4249 -> 4689, c64 copy 4251 -> 4596.
-            int64_t mis_elems = 0, all_elems = 0;
-            for (const TileDesc &d : all) {
-                const int64_t e = static_cast<int64_t>(d.nx) * d.ny;
-                all_elems += e;
-                if (!(d.flags & TF_FAST)) mis_elems += e;
-            }
-            const bool one_list = 2 * mis_elems >= all_elems;
+            const bool one_list = mostly_misaligned(all.data(), all.size(), es, false);
             if (one_list) {
                 out.mis = std::move(all);
             } else {
@@ -350,13 +357,17 @@ int super_tile(int esize) {
 // kLocalStrip tiles across its non-contiguous axis, each strip down the
 // buffer's contiguous axis, so that concurrent tiles form long contiguous
 // runs of target memory.  Measured on GB300: +6.6% on 16384^2 c128 (C) and
-// +2% on 8192^2 f64 (T); no gain for 4-byte elements (32 x 32 f32 tiles) and
-// a loss for op = N, whose source runs the global order keeps.  The
-// environment variable COSTA_TILE_ORDER (global | local) overrides the rule,
-// for tuning.
+// +2% on 8192^2 f64 (T); for 4-byte elements no gain on aligned layouts
+// (32 x 32 f32 tiles) and a loss when only the source is misaligned (B's
+// ld odd: 5350 -> 4786 GB/s), but +7 to +9% when most of the target runs
+// are misaligned (8192^2 f32 T copy, A's ld = 1 mod 4: 4305 -> 4696; both
+// lds odd 4371 -> 4678; BC50 -> BC75 +2%), where neighbouring tiles share
+// the partial sectors at their ends; a loss for op = N, whose source runs
+// the global order keeps.  The environment variable COSTA_TILE_ORDER (global |
+// local) overrides the rule, for tuning.
 constexpr int kLocalStrip = 2;
 
-bool use_local_order(const ProblemHost &ph) {
+bool use_local_order(const ProblemHost &ph, const TileDesc *tiles, size_t n) {
     static const int env = [] {
         const char *e = std::getenv("COSTA_TILE_ORDER");
         if (!e) return -1;
@@ -365,7 +376,9 @@ bool use_local_order(const ProblemHost &ph) {
         return -1;
     }();
     if (env >= 0) return env == 1;
-    return ph.op != COSTA_OP_N && esize_of(ph.A->dt) >= 8;
+    if (ph.op == COSTA_OP_N) return false;
+    const int es = esize_of(ph.A->dt);
+    return es >= 8 || mostly_misaligned(tiles, n, es, true);
 }
 
 // Stable LSD radix sort of (key, index) pairs by key, 11 bits per pass (the
@@ -476,7 +489,7 @@ void append_direct_tiles(const ProblemHost &ph, int prob, int es, int ts, std::v
                     }
         }
     });
-    if (!use_local_order(ph)) return;
+    if (!use_local_order(ph, list.data() + first, list.size() - first)) return;
     // a target whose tiles are each one contiguous run gains nothing
     bool contiguous = true;
     for (size_t i = first; i < list.size() && contiguous; ++i) contiguous = list[i].nx == list[i].dld;

@@ -106,7 +106,12 @@ bool aligned16(uint64_t addr, int64_t ld_bytes);
 TileDesc direct_tile(const ProblemHost &ph, const AxisTile &rt, const AxisTile &ct, int es, int prob);
 void set_fast(TileDesc &d, int es);
 
-bool use_local_order(const ProblemHost &ph);
+// True when misaligned tiles (with target_only, tiles whose target runs are
+// misaligned) hold at least half of the elements.
+bool mostly_misaligned(const TileDesc *tiles, size_t n, int es, bool target_only);
+// Whether a problem's tiles take the target-local order; `tiles` are the
+// problem's tiles (their alignment flags set).
+bool use_local_order(const ProblemHost &ph, const TileDesc *tiles, size_t n);
 void radix_sort_pairs(std::vector<std::pair<uint64_t, uint32_t>> &v);
 void order_tiles_local(std::vector<TileDesc> &list, size_t first, size_t last, int es, int ts);
 void append_direct_tiles(const ProblemHost &ph, int prob, int es, int ts, std::vector<TileDesc> &list);
