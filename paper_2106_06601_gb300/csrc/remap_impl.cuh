@@ -158,6 +158,15 @@ template <typename T> struct Cfg {
 // lost 20-40%).  An 8-byte window buffer is 8.5 KB, so shared memory, not
 // the register bound, sets the blocks per SM: 6 blocks with 1 buffer, 3
 // with 2, 2 with 3.
+// The copy kind keeps two tiles ahead (3 buffers, 2 blocks of 4 warps):
+// same box, 8192^2 T copy, GB/s against 2 buffers: BC50 -> BC75 4518 ->
+// 4677, BC75 -> BC75 4468 -> 5237, BC64 -> BC75 5050 -> 5380, c64 BC50 ->
+// BC75 4534 -> 4755, A's ld odd +0.4%, B's ld odd -0.4%, both -1.5%; the
+// scale kind lost 17% with it (8 warps per SM leave its FP64 multiplies
+// exposed) and keeps 2.
+#ifndef COSTA_MIS_NBUF_8C
+#define COSTA_MIS_NBUF_8C 3
+#endif
 #ifndef COSTA_MIS_NBUF_8
 #define COSTA_MIS_NBUF_8 2
 #endif
@@ -172,7 +181,8 @@ template <typename T, int KIND, bool MIS = false> struct KCfg {
                               : (MIS && READS_A) ? COSTA_MIS_MINB_8A : WIN ? COSTA_MIS_MINB_8 : COSTA_MINB_8;
     static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : WIN ? COSTA_MIS_NBUF_4 : COSTA_NBUF_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
-                              : HEAVY ? COSTA_NBUF_8H : WIN ? COSTA_MIS_NBUF_8 : COSTA_NBUF_8;
+                              : HEAVY ? COSTA_NBUF_8H
+                              : WIN ? (KIND == K_COPY ? COSTA_MIS_NBUF_8C : COSTA_MIS_NBUF_8) : COSTA_NBUF_8;
 };
 
 template <typename T> struct Chunk {
