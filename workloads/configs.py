@@ -152,13 +152,34 @@ def c2_general_beta(n: int = 8192) -> Problem:
     return p
 
 
-EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b, "c2g": c2_general_beta}
+def f32_lld(n: int = 8192, pad: int = 1) -> Problem:
+    """A ScaLAPACK-style target with an odd local leading dimension: f32,
+    T copy, B BC64 4x4 -> A BC128 4x4 with A's ld = local rows + pad (pad =
+    1: ld = 1 mod 4, every target run off 16-byte boundaries; pad = 0: the
+    same layouts aligned).  Not a configuration."""
+    B = L.block_cyclic(n, n, 64, 64, 4, 4, name="B")
+    A = L.block_cyclic(n, n, 128, 128, 4, 4, ld_pad=pad, name="A")
+    return Problem("ld1" if pad else "ld0", "f32", "T", 1.0, 0.0, A, B, "uniform", "uniform", _seed(7))
+
+
+def odd_blocks(n: int = 8192, dtype: str = "f64") -> Problem:
+    """Odd block sizes on both sides: T copy, B BC50 4x4 -> A BC75 4x4 (cells
+    of 25 x 25 and 25 x 50 elements, runs at odd 8-byte phases).  Not a
+    configuration."""
+    B = L.block_cyclic(n, n, 50, 50, 4, 4, name="B")
+    A = L.block_cyclic(n, n, 75, 75, 4, 4, name="A")
+    return Problem("odd", dtype, "T", 1.0, 0.0, A, B, "uniform", "uniform", _seed(7))
+
+
+EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b, "c2g": c2_general_beta,
+                   "ld1": f32_lld, "ld0": lambda: f32_lld(pad=0), "odd": odd_blocks}
 
 # The same layouts and tile shapes at about 1 GB on the device, for profiler
 # captures (the workloads proper stay the ones above).
 CONFIGS_SMALL = {"c1": c1, "c2": lambda: c2(4096), "c3": lambda: c3(8192),
                  "c4": lambda: c4(16), "c5": lambda: c5(rows=16384), "bc8": lambda: small_blocks(4096),
                  "c2g": lambda: c2_general_beta(4096),
+                 "ld1": lambda: f32_lld(8192), "ld0": lambda: f32_lld(8192, 0), "odd": lambda: odd_blocks(4096),
                  "c5b": lambda: c5b(rows=16384)}
 
 WORKLOAD_TEXT = {
@@ -173,6 +194,12 @@ WORKLOAD_TEXT = {
            "P=256 (the other reading of c5's target)",
     "c2g": "8192x8192 f64 BC64 4x4 -> BC128 4x4 permuted owners, T, alpha=-0.3 beta=0.7, P=16 "
            "(c2 with a general beta: TMA-staged source tiles; not a configuration)",
+    "ld1": "8192x8192 f32 BC64 4x4 -> BC128 4x4 with A's ld = 1 mod 4, T, alpha=1 beta=0, P=16 "
+           "(misaligned target runs; not a configuration)",
+    "ld0": "8192x8192 f32 BC64 4x4 -> BC128 4x4, T, alpha=1 beta=0, P=16 (ld1's layouts aligned; "
+           "not a configuration)",
+    "odd": "8192x8192 f64 BC50 4x4 -> BC75 4x4, T, alpha=1 beta=0, P=16 (odd block sizes; "
+           "not a configuration)",
 }
 
 
