@@ -159,7 +159,7 @@ def f32_lld(n: int = 8192, pad: int = 1) -> Problem:
     same layouts aligned).  Not a configuration."""
     B = L.block_cyclic(n, n, 64, 64, 4, 4, name="B")
     A = L.block_cyclic(n, n, 128, 128, 4, 4, ld_pad=pad, name="A")
-    return Problem("ld1" if pad else "ld0", "f32", "T", 1.0, 0.0, A, B, "uniform", "uniform", _seed(7))
+    return Problem("ld1" if pad else "ld0", "f32", "T", 1.0, 0.0, A, B, "uniform", "nan", _seed(7))
 
 
 def odd_blocks(n: int = 8192, dtype: str = "f64") -> Problem:
@@ -168,7 +168,7 @@ def odd_blocks(n: int = 8192, dtype: str = "f64") -> Problem:
     configuration."""
     B = L.block_cyclic(n, n, 50, 50, 4, 4, name="B")
     A = L.block_cyclic(n, n, 75, 75, 4, 4, name="A")
-    return Problem("odd", dtype, "T", 1.0, 0.0, A, B, "uniform", "uniform", _seed(7))
+    return Problem("odd", dtype, "T", 1.0, 0.0, A, B, "uniform", "nan", _seed(7))
 
 
 EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b, "c2g": c2_general_beta,
