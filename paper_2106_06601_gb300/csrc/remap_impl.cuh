@@ -230,6 +230,7 @@ __device__ __forceinline__ double fmar(double a, double b, double c) { return __
 
 struct Sc {
     double ar, ai, br, bi;
+    bool alpha_mid;      // both components of alpha zero or of magnitude in [2^-480, 2^480)
     uint32_t conj_mask;  // 0x80000000 flips the sign of b's imaginary part (op = C)
     int32_t bexp;        // |beta| = 2^bexp (K_AXPBY2)
     uint32_t bsign_hi;   // sign bit of beta in a high word (K_AXPBY2)
@@ -294,6 +295,29 @@ template <typename R> struct Dot2 {
     __device__ __forceinline__ R result() const { return isfinite(p) ? addr(p, s) : p; }
 };
 
+// A double that is zero or of magnitude in [2^-480, 2^480): products of two
+// such values neither overflow nor lose their rounding error to underflow.
+__device__ __forceinline__ bool mid_range(double v) {
+    const unsigned hi = static_cast<unsigned>(__double2hiint(v));
+    const unsigned lo = static_cast<unsigned>(__double2loint(v));
+    const unsigned e = (hi >> 20) & 0x7FFu;
+    return (((hi & 0x7FFFFFFFu) | lo) == 0u) || (e - (1023u - 480u)) < 960u;
+}
+
+// x * y + sgn * (z * t) with Kahan's algorithm for 2 x 2 determinants: w =
+// z * t rounded, its error e exactly by one fma, then (x * y + sgn * w)
+// rounded by a second fma and sgn * e added.  Jeannerod, Louvet and Muller
+// ("Further analysis of Kahan's algorithm for the accurate computation of
+// 2 x 2 determinants", Math. Comp. 82, 2013) bound its error by 2u|exact|
+// when nothing overflows or underflows: within 2 ulps of the exact value,
+// and so of the oracle's compensated result.  4 FP64 operations instead of
+// Dot2's 13.
+__device__ __forceinline__ double kahan2(double x, double y, double z, double t, bool minus) {
+    const double w = __dmul_rn(z, t);
+    const double e = __fma_rn(z, t, -w);  // z * t = w + e exactly
+    return minus ? __dsub_rn(__fma_rn(x, y, -w), e) : __dadd_rn(__fma_rn(x, y, w), e);
+}
+
 template <int KIND, typename C, typename R>
 __device__ __forceinline__ C combine_c(C b, C a, const Sc &s) {
     b.y = flip_sign(b.y, s.conj_mask);
@@ -302,6 +326,16 @@ __device__ __forceinline__ C combine_c(C b, C a, const Sc &s) {
         o.x = comb_real<KIND, R>(b.x, a.x, s);
         o.y = comb_real<KIND, R>(b.y, a.y, s);
         return o;
+    }
+    if constexpr (KIND == K_CSCALE && sizeof(R) == 8) {
+        // the FP64 pipe is this kind's limit: two-term components take
+        // Kahan's algorithm when every operand is in the middle range (the
+        // others, and all non-finite values, take Dot2 below)
+        if (s.alpha_mid && mid_range(b.x) && mid_range(b.y)) {
+            o.x = kahan2(s.ar, b.x, s.ai, b.y, true);   // ar bx - ai by
+            o.y = kahan2(s.ar, b.y, s.ai, b.x, false);  // ar by + ai bx
+            return o;
+        }
     }
     const R ar = R(s.ar), ai = R(s.ai);
     Dot2<R> re(ar, b.x), im(ar, b.y);
@@ -871,6 +905,7 @@ __device__ __forceinline__ void stage_drain_e1(const Geom<T> &g, const Sc &s, un
 // Scalars of a problem in the kernel's form.
 __device__ __forceinline__ void make_sc(const Scalars &S, Sc &s) {
     s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
+    s.alpha_mid = mid_range(S.alpha[0]) && mid_range(S.alpha[1]);
     s.conj_mask = 0u;
     s.bexp = S.beta_exp;
     s.bsign_hi = static_cast<unsigned>(__double2hiint(S.beta[0])) & 0x80000000u;

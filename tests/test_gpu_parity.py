@@ -235,6 +235,39 @@ def test_special_values_power_of_two_beta(dtype, beta, dev):
         g.close()
 
 
+@pytest.mark.parametrize("dtype", ["f64", "c128", "f32"])
+@pytest.mark.parametrize("alpha", [2.0, -1.0, 0.25, -(2.0 ** -1000), 2.0 ** 1000])
+def test_special_values_power_of_two_alpha(dtype, alpha, dev):
+    """alpha * b with beta = 0 and alpha = +-2^k is exact wherever it stays
+    in range: the scale kind must equal the oracle bit for bit, with zeros,
+    subnormals, infinities and NaNs among the inputs and products that
+    underflow below the normal range or overflow."""
+    if dtype == "f32" and abs(alpha) in (2.0 ** -1000, 2.0 ** 1000):
+        pytest.skip("alpha is not representable in float")
+    rng = np.random.default_rng(6)
+    B = L.block_cyclic(64, 48, 16, 16, 2, 2)
+    A = L.block_cyclic(48, 64, 8, 32, 2, 2, storage="C")
+    p = C.Problem("special-a", dtype, "T", alpha, 0.0, A, B, "uniform", "nan", C.SEED0)
+    g = OnDevice(p, dev)
+    try:
+        real = np.float64 if dtype in ("f64", "c128") else np.float32
+        fi = np.finfo(real)
+        specials = np.array([0.0, -0.0, fi.tiny, -fi.tiny, fi.tiny / 4, -fi.smallest_subnormal,
+                             fi.max / 4, -fi.max, np.inf, -np.inf, np.nan, 1.5, -3.0,
+                             fi.tiny * 2, fi.max / 8, 1e-300 if real is np.float64 else 1e-30],
+                            dtype=real)
+        v = g.Bh.arena.view(real)
+        idx = rng.integers(0, v.size, v.size // 3)
+        v[idx] = specials[rng.integers(0, specials.size, idx.size)]
+        g.Bd.upload(g.Bh)
+        g.run(relabel=False)
+        got, want = g.Ad.download(), g.oracle_result()
+        ok = (got.arena == want.arena) | (np.isnan(got.arena) & np.isnan(want.arena))
+        assert np.all(ok), (np.flatnonzero(~ok)[:5], got.arena[~ok][:5], want.arena[~ok][:5])
+    finally:
+        g.close()
+
+
 def test_phase_timing(dev):
     """Phase events: one phase in direct mode, pack/local/unpack in message
     mode; results are unchanged by the timing; a call with no tiles leaves
