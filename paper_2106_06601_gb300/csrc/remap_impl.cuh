@@ -86,6 +86,23 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_NBUF_8H
 #define COSTA_NBUF_8H 2
 #endif
+// c64 with complex scalars (same box, 8192^2, BC64 -> BC128, GB/s against
+// 3 blocks with 2 buffers): complex beta runs 4 blocks without look-ahead
+// (T 4484 -> 5482, N 4495 -> 5495), complex alpha with beta = 0 keeps two
+// tiles ahead (3 buffers, so 2 blocks fit: 5551 -> 5955); the real general
+// kind loses with either (6492 -> 6400 and 6082).
+#ifndef COSTA_MINB_8C
+#define COSTA_MINB_8C 4
+#endif
+#ifndef COSTA_NBUF_8C
+#define COSTA_NBUF_8C 1
+#endif
+#ifndef COSTA_MINB_8CS
+#define COSTA_MINB_8CS 2
+#endif
+#ifndef COSTA_NBUF_8CS
+#define COSTA_NBUF_8CS 3
+#endif
 #ifndef COSTA_WARPS_16
 #define COSTA_WARPS_16 4
 #endif
@@ -130,8 +147,9 @@ template <typename T> struct Cfg {
 // shared-memory buffers per warp (the warp keeps NBUF - 1 tiles' copies in
 // flight ahead of the tile it writes).
 //  - 8-byte types: the light kinds run more warps without look-ahead; the
-//    general kinds (non-power-of-two beta, complex scalars) need the
-//    registers of 3 blocks and use a 2-deep ring; in the misaligned-tile
+//    real general kind (non-power-of-two beta) needs the registers of 3
+//    blocks and uses a 2-deep ring, the complex kinds have shapes of their
+//    own (below); in the misaligned-tile
 //    instance the light kinds that read A (one element per lane, a whole
 //    tile of A in registers) run 4 blocks, which their registers fit
 //    without spills, and the kinds that do not (16-byte windows) a 2-deep
@@ -177,10 +195,12 @@ template <typename T, int KIND, bool MIS = false> struct KCfg {
     static constexpr int WARPS = Cfg<T>::WARPS;
     static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : WIN ? COSTA_MIS_MINB_4 : COSTA_MINB_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
+                              : KIND == K_CPLX ? COSTA_MINB_8C : KIND == K_CSCALE ? COSTA_MINB_8CS
                               : HEAVY ? COSTA_MINB_8H
                               : (MIS && READS_A) ? COSTA_MIS_MINB_8A : WIN ? COSTA_MIS_MINB_8 : COSTA_MINB_8;
     static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : WIN ? COSTA_MIS_NBUF_4 : COSTA_NBUF_4)
                               : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
+                              : KIND == K_CPLX ? COSTA_NBUF_8C : KIND == K_CSCALE ? COSTA_NBUF_8CS
                               : HEAVY ? COSTA_NBUF_8H
                               : WIN ? (KIND == K_COPY ? COSTA_MIS_NBUF_8C : COSTA_MIS_NBUF_8) : COSTA_NBUF_8;
 };
