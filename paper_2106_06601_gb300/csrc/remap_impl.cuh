@@ -91,6 +91,25 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 // (T 4484 -> 5482, N 4495 -> 5495), complex alpha with beta = 0 keeps two
 // tiles ahead (3 buffers, so 2 blocks fit: 5551 -> 5955); the real general
 // kind loses with either (6492 -> 6400 and 6082).
+// The scale kind (real alpha, beta = 0) of f64 and c128 has multiplies on
+// the narrow FP64 pipe, and hides their latency with more tiles in flight
+// than the copy: f64 keeps two tiles ahead (3 buffers, 2 blocks), c128 runs
+// 3 blocks without look-ahead.  Same box, 8192^2, BC64 -> BC128, GB/s: f64 T
+// alpha=2 5400 -> 6204, N alpha=-0.7 5361 -> 6147 (the copy's rate); c128 T
+// 4410 -> 5853, N 4343 -> 5746.  c64 (float multiplies) lost 11% with the
+// f64 shape and keeps the light kinds'.
+#ifndef COSTA_MINB_8S
+#define COSTA_MINB_8S 2
+#endif
+#ifndef COSTA_NBUF_8S
+#define COSTA_NBUF_8S 3
+#endif
+#ifndef COSTA_MINB_16S
+#define COSTA_MINB_16S 3
+#endif
+#ifndef COSTA_NBUF_16S
+#define COSTA_NBUF_16S 1
+#endif
 #ifndef COSTA_MINB_8C
 #define COSTA_MINB_8C 4
 #endif
@@ -194,13 +213,15 @@ template <typename T, int KIND, bool MIS = false> struct KCfg {
     static constexpr bool WIN = MIS && !READS_A;  // the window path of the misaligned instance
     static constexpr int WARPS = Cfg<T>::WARPS;
     static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : WIN ? COSTA_MIS_MINB_4 : COSTA_MINB_4)
-                              : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : COSTA_MINB_16)
+                              : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : KIND == K_SCALE ? COSTA_MINB_16S : COSTA_MINB_16)
                               : KIND == K_CPLX ? COSTA_MINB_8C : KIND == K_CSCALE ? COSTA_MINB_8CS
+                              : (KIND == K_SCALE && !MIS && !ET<T>::CPLX) ? COSTA_MINB_8S
                               : HEAVY ? COSTA_MINB_8H
                               : (MIS && READS_A) ? COSTA_MIS_MINB_8A : WIN ? COSTA_MIS_MINB_8 : COSTA_MINB_8;
     static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : WIN ? COSTA_MIS_NBUF_4 : COSTA_NBUF_4)
-                              : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : COSTA_NBUF_16)
+                              : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : KIND == K_SCALE ? COSTA_NBUF_16S : COSTA_NBUF_16)
                               : KIND == K_CPLX ? COSTA_NBUF_8C : KIND == K_CSCALE ? COSTA_NBUF_8CS
+                              : (KIND == K_SCALE && !MIS && !ET<T>::CPLX) ? COSTA_NBUF_8S
                               : HEAVY ? COSTA_NBUF_8H
                               : WIN ? (KIND == K_COPY ? COSTA_MIS_NBUF_8C : COSTA_MIS_NBUF_8) : COSTA_NBUF_8;
 };
