@@ -538,8 +538,10 @@ costa_status costa_debug_exchange(costa_layout A, costa_layout B, costa_op op, i
  * (environment variable COSTA_TMA unset when a plan is built) only f64 data
  * with a beta that is neither 0 nor +-2^k uses it (measured faster there,
  * slower for every other kind and type); COSTA_TMA=0 turns it off and
- * COSTA_TMA=1 on for every kind and type.  Builds the plan of (A, B, op) if needed, then writes
- * out[0] = TMA tiles in the direct list, out[1] = in its x-halves list,
+ * COSTA_TMA=1 on for every kind and type.  Builds the plan of (A, B, op)
+ * and its TMA-staged lists if needed (a transform builds them on the first
+ * call of a kind that uses them), then writes out[0] = TMA tiles in the
+ * direct list, out[1] = in its x-halves list,
  * out[2] = tensor maps, out[3] = TMA waits that gave up in this plan's
  * launches (each ends its warp's work and should never happen), out[4] and
  * out[5] = the kinds (bit per combine kind) that take the TMA tiles of the

@@ -124,3 +124,63 @@ def test_default_policy_general_beta_matches_oracle():
                        capture_output=True, text=True, timeout=900)
     assert r.returncode == 0, (r.stdout[-3000:], r.stderr[-3000:])
     assert "c2beta" in r.stdout
+
+
+def test_lists_built_after_capture_keep_the_graph_valid():
+    """The TMA-staged lists are built by the first eager call of a kind that
+    uses them, never inside a stream capture.  A general-beta f64 transform
+    captured in a CUDA graph before that call replays on the cp.async lists;
+    the eager call then builds the TMA lists (and takes them), and the graph
+    still replays correctly afterwards.  Every step is compared with the
+    oracle applied to the A it started from, within the tolerance."""
+    script = r"""
+import numpy as np
+import torch
+import oracle
+import paper_2106_06601_gb300 as costa
+from tests._util import assert_close, global_matrix, op_apply
+from workloads import configs as C
+from workloads.materialize import DeviceMatrix
+dev = torch.device("cuda:0")
+torch.cuda.set_device(dev)
+p = C.c2(2048)
+p.alpha, p.beta = -0.3, 0.7
+Bd = DeviceMatrix(p.B, p.dtype, dev).fill(p.b_kind, p.seed, p.src_stream)
+Ad = DeviceMatrix(p.A, p.dtype, dev).fill(p.a_kind, p.seed, p.tgt_stream)
+Bh = Bd.download()
+LA = costa.costa_layout_from_spec(p.A, p.dtype, Ad.block_ptrs())
+LB = costa.costa_layout_from_spec(p.B, p.dtype, Bd.block_ptrs())
+al, be = oracle.scalar(p.dtype, p.alpha), oracle.scalar(p.dtype, p.beta)
+X = op_apply(p.op, global_matrix(p.B, Bh.buffers()))
+s = torch.cuda.Stream(dev)
+costa.costa_plan_stats_get(LA, LB, p.op, relabel=True)  # the plan, without a transform
+graph = torch.cuda.CUDAGraph()
+with torch.cuda.graph(graph, stream=s):
+    costa.costa_transform(LA, LB, p.op, p.alpha, p.beta, relabel=True,
+                          stream=torch.cuda.current_stream().cuda_stream)
+
+def step(run):
+    before = Ad.download()
+    run()
+    torch.cuda.synchronize(dev)
+    want = before.copy()
+    oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, want.buffers(), p.B, Bh.buffers())
+    got = Ad.download()
+    assert_close(p.dtype, global_matrix(p.A, got.buffers()), global_matrix(p.A, want.buffers()),
+                 al, be, X, global_matrix(p.A, before.buffers()), exact=False)
+
+step(graph.replay)
+step(graph.replay)
+step(lambda: costa.costa_transform(LA, LB, p.op, p.alpha, p.beta, relabel=True, stream=s.cuda_stream))
+st = costa.costa_debug_tma(LA, LB, p.op)
+assert st["tiles"] > 0 and st["timeouts"] == 0, st
+step(graph.replay)
+step(lambda: costa.costa_transform(LA, LB, p.op, p.alpha, p.beta, relabel=True, stream=s.cuda_stream))
+print("ok", st)
+"""
+    env = dict(os.environ)
+    env.pop("COSTA_TMA", None)
+    r = subprocess.run([sys.executable, "-c", script], cwd=ROOT, env=env, capture_output=True,
+                       text=True, timeout=600)
+    assert r.returncode == 0, (r.stdout[-3000:], r.stderr[-3000:])
+    assert "ok" in r.stdout
