@@ -105,8 +105,9 @@ enum : int32_t { SF_BETA0 = 1, SF_ALPHA1 = 2, SF_CPLX = 4, SF_BPOW2 = 8 };
 //   K_AXPBY2 as K_AXPBY with beta = +-2^k: beta * a is formed exactly on the
 //            integer pipes (exponent add), saving one multiply on the scarce
 //            FP64 pipe; same bits as K_AXPBY
-//   K_CSCALE complex alpha, beta = 0   out = alpha * op(b) by Dot2; A is not
-//            read (BLAS convention), so NaN in A does not propagate
+//   K_CSCALE complex alpha, beta = 0   out = alpha * op(b) by Dot2 (double
+//            data in the middle range: Kahan's 2 x 2 determinant algorithm);
+//            A is not read (BLAS convention), so NaN in A does not propagate
 enum : int { K_COPY = 0, K_SCALE = 1, K_AXPBY = 2, K_CPLX = 3, K_AXPBY2 = 4, K_CSCALE = 5, K_NKINDS = 6 };
 
 // The kinds whose output depends on A's old value (beta != 0).

@@ -53,9 +53,64 @@ template <> struct ET<double>  { enum { VEC = 2, CPLX = 0 }; typedef double R; }
 template <> struct ET<float2>  { enum { VEC = 2, CPLX = 1 }; typedef float R; };
 template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; };
 
+// Launch shape of the tile kernel per element size, combine kind and
+// instance, all measured on GB300 (same box, 8192^2, GB/s): warps per
+// block, the resident blocks per SM that the registers must allow (MINB),
+// and shared-memory buffers per warp (NBUF: a warp keeps NBUF - 1 tiles'
+// copies in flight ahead of the tile it writes).
+//
+//   element  instance     kinds                         warps  MINB  NBUF
+//   4-byte   both         copy, scale                     8      2     2
+//            both         kinds that read A               8      3     1
+//   8-byte   aligned      copy, axpby2 (beta = +-2^k)     4      5     1
+//            aligned      f64 scale                       4      2     3
+//            aligned      c64 scale                       4      5     1
+//            both         real general beta               4      3     2
+//            both         complex beta                    4      4     1
+//            both         complex alpha, beta = 0         4      2     3
+//            misaligned   copy (16-byte windows)          4      5     3
+//            misaligned   scale (16-byte windows)         4      5     2
+//            misaligned   axpby2 (one element per lane)   4      4     1
+//   16-byte  both         copy                            4      1     2
+//            both         scale                           4      3     1
+//            both         complex alpha, beta = 0         4      2     1
+//            both         kinds that read A               4      2     1
+//
+// Why, where a row departs from its neighbours:
+//  - 8-byte light kinds (copy, axpby2) run more warps without look-ahead;
+//    the real general kind needs the registers of 3 blocks.
+//  - f64 and c128 scale: one multiply per element on the narrow FP64 pipe,
+//    hidden by more tiles in flight than the copy has: f64 T alpha=2 5400
+//    -> 6204, N alpha=-0.7 5361 -> 6147 (the copy's rate) with two tiles
+//    ahead; c128 T 4410 -> 5853, N 4343 -> 5746 with 3 blocks.  c64
+//    (float multiplies) lost 11% with f64's shape and keeps the light one.
+//    c128 with a complex alpha (FP64-bound at 8 operations per element):
+//    T and N 1458 -> 2133 with 2 to 4 blocks.
+//  - c64 complex scalars, against 3 blocks with 2 buffers: complex beta
+//    T 4484 -> 5482, N 4495 -> 5495 with 4 blocks and no look-ahead;
+//    complex alpha T 5551 -> 5955 with two tiles ahead; the real general
+//    kind loses with either (6492 -> 6400 and 6082).
+//  - 8-byte window path (misaligned instance, kinds that do not read A):
+//    an 8.5 KB buffer per tile, so shared memory, not MINB, sets the blocks
+//    per SM (6 with 1 buffer, 3 with 2, 2 with 3).  One tile ahead took f64
+//    BC50 -> BC75 copy 3820 -> 4101, scale 3620 -> 4162, c64 copy 3797 ->
+//    4093 (odd leading dimensions -0.4 to +1%); two tiles ahead took the
+//    copy further (BC50 -> BC75 4518 -> 4677, BC75 -> BC75 4468 -> 5237,
+//    BC64 -> BC75 5050 -> 5380, c64 BC50 -> BC75 4534 -> 4755; odd lds
+//    -1.5 to +0.4%) but cost the scale kind 17%, whose FP64 multiplies 8
+//    warps per SM leave exposed; 4 buffers lost 20-40%.
+//  - 8-byte element path (misaligned, kinds that read A): a whole tile of A
+//    in registers, which 4 blocks fit without spills.
+//  - 16-byte kinds that read A hold a whole 16 KB tile of A in registers.
+// Each entry is overridable at build time for tuning (COSTA_WARPS_4/8,
+// COSTA_MINB_* and COSTA_NBUF_*).
 #ifndef COSTA_WARPS_4
 #define COSTA_WARPS_4 8
 #endif
+#ifndef COSTA_WARPS_8
+#define COSTA_WARPS_8 4
+#endif
+// 4-byte: light kinds, kinds that read A
 #ifndef COSTA_MINB_4
 #define COSTA_MINB_4 2
 #endif
@@ -68,47 +123,25 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_NBUF_4A
 #define COSTA_NBUF_4A 1
 #endif
-#ifndef COSTA_WARPS_8
-#define COSTA_WARPS_8 4
-#endif
+// 8-byte: light kinds (L), f64 scale (S), real general (H), complex beta
+// (C), complex alpha (CS), window path (W: copy WC), element path (A)
 #ifndef COSTA_MINB_8
 #define COSTA_MINB_8 5
 #endif
 #ifndef COSTA_NBUF_8
 #define COSTA_NBUF_8 1
 #endif
-#ifndef COSTA_MINB_8H
-#define COSTA_MINB_8H 3
-#endif
-#ifndef COSTA_MIS_MINB_8A
-#define COSTA_MIS_MINB_8A 4
-#endif
-#ifndef COSTA_NBUF_8H
-#define COSTA_NBUF_8H 2
-#endif
-// c64 with complex scalars (same box, 8192^2, BC64 -> BC128, GB/s against
-// 3 blocks with 2 buffers): complex beta runs 4 blocks without look-ahead
-// (T 4484 -> 5482, N 4495 -> 5495), complex alpha with beta = 0 keeps two
-// tiles ahead (3 buffers, so 2 blocks fit: 5551 -> 5955); the real general
-// kind loses with either (6492 -> 6400 and 6082).
-// The scale kind (real alpha, beta = 0) of f64 and c128 has multiplies on
-// the narrow FP64 pipe, and hides their latency with more tiles in flight
-// than the copy: f64 keeps two tiles ahead (3 buffers, 2 blocks), c128 runs
-// 3 blocks without look-ahead.  Same box, 8192^2, BC64 -> BC128, GB/s: f64 T
-// alpha=2 5400 -> 6204, N alpha=-0.7 5361 -> 6147 (the copy's rate); c128 T
-// 4410 -> 5853, N 4343 -> 5746.  c64 (float multiplies) lost 11% with the
-// f64 shape and keeps the light kinds'.
 #ifndef COSTA_MINB_8S
 #define COSTA_MINB_8S 2
 #endif
 #ifndef COSTA_NBUF_8S
 #define COSTA_NBUF_8S 3
 #endif
-#ifndef COSTA_MINB_16S
-#define COSTA_MINB_16S 3
+#ifndef COSTA_MINB_8H
+#define COSTA_MINB_8H 3
 #endif
-#ifndef COSTA_NBUF_16S
-#define COSTA_NBUF_16S 1
+#ifndef COSTA_NBUF_8H
+#define COSTA_NBUF_8H 2
 #endif
 #ifndef COSTA_MINB_8C
 #define COSTA_MINB_8C 4
@@ -122,14 +155,36 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_NBUF_8CS
 #define COSTA_NBUF_8CS 3
 #endif
-#ifndef COSTA_WARPS_16
-#define COSTA_WARPS_16 4
+#ifndef COSTA_MINB_8W
+#define COSTA_MINB_8W COSTA_MINB_8
 #endif
+#ifndef COSTA_NBUF_8W
+#define COSTA_NBUF_8W 2
+#endif
+#ifndef COSTA_NBUF_8WC
+#define COSTA_NBUF_8WC 3
+#endif
+#ifndef COSTA_MINB_8A
+#define COSTA_MINB_8A 4
+#endif
+// 16-byte: light kinds, scale, kinds that read A
 #ifndef COSTA_MINB_16
 #define COSTA_MINB_16 1
 #endif
 #ifndef COSTA_NBUF_16
 #define COSTA_NBUF_16 2
+#endif
+#ifndef COSTA_MINB_16S
+#define COSTA_MINB_16S 3
+#endif
+#ifndef COSTA_NBUF_16S
+#define COSTA_NBUF_16S 1
+#endif
+#ifndef COSTA_MINB_16CS
+#define COSTA_MINB_16CS 2
+#endif
+#ifndef COSTA_NBUF_16CS
+#define COSTA_NBUF_16CS 1
 #endif
 #ifndef COSTA_MINB_16A
 #define COSTA_MINB_16A 2
@@ -137,6 +192,31 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #ifndef COSTA_NBUF_16A
 #define COSTA_NBUF_16A 1
 #endif
+
+struct Shape {
+    int minb, nbuf;
+};
+
+// The table above.  es: element size; cplx: complex elements; mis: the
+// misaligned-tile instance.
+constexpr Shape launch_shape(int es, bool cplx, int kind, bool mis) {
+    const bool reads_a = kind_reads_a(kind);
+    if (es == 4) return reads_a ? Shape{COSTA_MINB_4A, COSTA_NBUF_4A} : Shape{COSTA_MINB_4, COSTA_NBUF_4};
+    if (es == 16) {
+        if (reads_a) return {COSTA_MINB_16A, COSTA_NBUF_16A};
+        if (kind == K_CSCALE) return {COSTA_MINB_16CS, COSTA_NBUF_16CS};
+        return kind == K_SCALE ? Shape{COSTA_MINB_16S, COSTA_NBUF_16S} : Shape{COSTA_MINB_16, COSTA_NBUF_16};
+    }
+    if (kind == K_CPLX) return {COSTA_MINB_8C, COSTA_NBUF_8C};
+    if (kind == K_CSCALE) return {COSTA_MINB_8CS, COSTA_NBUF_8CS};
+    if (kind == K_AXPBY) return {COSTA_MINB_8H, COSTA_NBUF_8H};
+    if (mis) {
+        if (reads_a) return {COSTA_MINB_8A, COSTA_NBUF_8};
+        return {COSTA_MINB_8W, kind == K_COPY ? COSTA_NBUF_8WC : COSTA_NBUF_8W};
+    }
+    if (kind == K_SCALE && !cplx) return {COSTA_MINB_8S, COSTA_NBUF_8S};
+    return {COSTA_MINB_8, COSTA_NBUF_8};
+}
 
 // Per element type: tile extent TS, 16-byte chunk width VEC (elements), and
 // the lane mapping: CPR chunks cover one run of TS elements, a warp pass
@@ -152,7 +232,7 @@ template <typename T> struct Cfg {
     static constexpr int PITCH = TS + 1;
     static constexpr int BUF_BYTES_RAW = TS * PITCH * static_cast<int>(sizeof(T));
     static constexpr int BUF_BYTES = (BUF_BYTES_RAW + 127) / 128 * 128;
-    static constexpr int WARPS = sizeof(T) == 4 ? COSTA_WARPS_4 : sizeof(T) == 16 ? COSTA_WARPS_16 : COSTA_WARPS_8;
+    static constexpr int WARPS = sizeof(T) == 4 ? COSTA_WARPS_4 : COSTA_WARPS_8;
     // Lane maps give a run at most 32 lanes: a run's chunks (aligned path),
     // its elements (misaligned path of the kinds that read A) and one lane
     // per run or row (the window path's last pass) must each fit in a warp.
@@ -161,69 +241,13 @@ template <typename T> struct Cfg {
     static_assert(TS >= 1 && TS <= 32 && TS % VEC == 0, "tile extent must be a multiple of VEC in [VEC, 32]");
 };
 
-// Launch shape per element type and combine kind (measured on GB300): warps
-// per block, resident blocks per SM the registers must allow, and
-// shared-memory buffers per warp (the warp keeps NBUF - 1 tiles' copies in
-// flight ahead of the tile it writes).
-//  - 8-byte types: the light kinds run more warps without look-ahead; the
-//    real general kind (non-power-of-two beta) needs the registers of 3
-//    blocks and uses a 2-deep ring, the complex kinds have shapes of their
-//    own (below); in the misaligned-tile
-//    instance the light kinds that read A (one element per lane, a whole
-//    tile of A in registers) run 4 blocks, which their registers fit
-//    without spills, and the kinds that do not (16-byte windows) a 2-deep
-//    ring (shared memory then holds 3 blocks of 4 warps).
-//  - 4-byte types: the kinds that read A run 3 blocks without look-ahead,
-//    the others 2 blocks with a 2-deep ring.
-//  - 16-byte types: the kinds that read A hold a whole 16 KB tile of A in
-//    registers and run two blocks without look-ahead.
-// Overridable at build time for tuning.
-#ifndef COSTA_MIS_MINB_4
-#define COSTA_MIS_MINB_4 COSTA_MINB_4
-#endif
-#ifndef COSTA_MIS_NBUF_4
-#define COSTA_MIS_NBUF_4 COSTA_NBUF_4
-#endif
-#ifndef COSTA_MIS_MINB_8
-#define COSTA_MIS_MINB_8 COSTA_MINB_8
-#endif
-// The window path of 8-byte types keeps one tile's copies in flight ahead
-// (measured on GB300, 8192^2 T, same box, GB/s: f64 BC50 -> BC75 copy
-// 3820 -> 4101, scale 3620 -> 4162, c64 copy 3797 -> 4093; odd leading
-// dimensions -0.4 to +1%; 3 buffers (2 blocks fit) helped the copy to 4300
-// but cost the scale kind 0% and the odd-ld cases up to 1.3%, 4 buffers
-// lost 20-40%).  An 8-byte window buffer is 8.5 KB, so shared memory, not
-// the register bound, sets the blocks per SM: 6 blocks with 1 buffer, 3
-// with 2, 2 with 3.
-// The copy kind keeps two tiles ahead (3 buffers, 2 blocks of 4 warps):
-// same box, 8192^2 T copy, GB/s against 2 buffers: BC50 -> BC75 4518 ->
-// 4677, BC75 -> BC75 4468 -> 5237, BC64 -> BC75 5050 -> 5380, c64 BC50 ->
-// BC75 4534 -> 4755, A's ld odd +0.4%, B's ld odd -0.4%, both -1.5%; the
-// scale kind lost 17% with it (8 warps per SM leave its FP64 multiplies
-// exposed) and keeps 2.
-#ifndef COSTA_MIS_NBUF_8C
-#define COSTA_MIS_NBUF_8C 3
-#endif
-#ifndef COSTA_MIS_NBUF_8
-#define COSTA_MIS_NBUF_8 2
-#endif
 template <typename T, int KIND, bool MIS = false> struct KCfg {
     static constexpr bool HEAVY = KIND == K_AXPBY || KIND == K_CPLX || KIND == K_CSCALE;
     static constexpr bool READS_A = kind_reads_a(KIND);
-    static constexpr bool WIN = MIS && !READS_A;  // the window path of the misaligned instance
     static constexpr int WARPS = Cfg<T>::WARPS;
-    static constexpr int MINB = sizeof(T) == 4 ? (READS_A ? COSTA_MINB_4A : WIN ? COSTA_MIS_MINB_4 : COSTA_MINB_4)
-                              : sizeof(T) == 16 ? (READS_A ? COSTA_MINB_16A : KIND == K_SCALE ? COSTA_MINB_16S : COSTA_MINB_16)
-                              : KIND == K_CPLX ? COSTA_MINB_8C : KIND == K_CSCALE ? COSTA_MINB_8CS
-                              : (KIND == K_SCALE && !MIS && !ET<T>::CPLX) ? COSTA_MINB_8S
-                              : HEAVY ? COSTA_MINB_8H
-                              : (MIS && READS_A) ? COSTA_MIS_MINB_8A : WIN ? COSTA_MIS_MINB_8 : COSTA_MINB_8;
-    static constexpr int NBUF = sizeof(T) == 4 ? (READS_A ? COSTA_NBUF_4A : WIN ? COSTA_MIS_NBUF_4 : COSTA_NBUF_4)
-                              : sizeof(T) == 16 ? (READS_A ? COSTA_NBUF_16A : KIND == K_SCALE ? COSTA_NBUF_16S : COSTA_NBUF_16)
-                              : KIND == K_CPLX ? COSTA_NBUF_8C : KIND == K_CSCALE ? COSTA_NBUF_8CS
-                              : (KIND == K_SCALE && !MIS && !ET<T>::CPLX) ? COSTA_NBUF_8S
-                              : HEAVY ? COSTA_NBUF_8H
-                              : WIN ? (KIND == K_COPY ? COSTA_MIS_NBUF_8C : COSTA_MIS_NBUF_8) : COSTA_NBUF_8;
+    static constexpr Shape SHAPE = launch_shape(static_cast<int>(sizeof(T)), ET<T>::CPLX != 0, KIND, MIS);
+    static constexpr int MINB = SHAPE.minb;
+    static constexpr int NBUF = SHAPE.nbuf;
 };
 
 template <typename T> struct Chunk {
