@@ -331,7 +331,7 @@ __device__ __forceinline__ double flip_sign(double v, uint32_t m) {
 // compensated dot product Dot2 of Ogita, Rump and Oishi ("Accurate sum and
 // dot product", SIAM J. Sci. Comput. 26(6), 2005) over its 2 or 4 products,
 // built on TwoProduct (one fma gives a product's rounding error exactly) and
-// Knuth's TwoSum.  The result lies within u|x| + gamma_n^2 * sum|terms| of
+// an error-free sum (two_sum below).  The result lies within u|x| + gamma_n^2 * sum|terms| of
 // the exact component x (u the unit roundoff, n the number of terms): as if
 // computed in twice the working precision and rounded once.  The running sum
 // p is the plain sum of the rounded products; when it is not finite (an
@@ -342,6 +342,25 @@ __device__ __forceinline__ double addr(double a, double b) { return __dadd_rn(a,
 __device__ __forceinline__ float subr(float a, float b) { return __fsub_rn(a, b); }
 __device__ __forceinline__ double subr(double a, double b) { return __dsub_rn(a, b); }
 
+// p + h = t + q exactly.  Float: Knuth's TwoSum (6 operations).  Double:
+// the two operands ordered by exponent on the integer pipes (their high
+// words without the sign), then Dekker's Fast2Sum (3 operations), which is
+// exact when the first operand's exponent is not below the second's: the
+// same t and q, with half the FP64 operations, the pipe that bounds the
+// complex kinds of c128 on GB300.
+__device__ __forceinline__ void two_sum(float p, float h, float &t, float &q) {
+    t = addr(p, h);
+    const float z = subr(t, p);
+    q = addr(subr(p, subr(t, z)), subr(h, z));
+}
+__device__ __forceinline__ void two_sum(double p, double h, double &t, double &q) {
+    const unsigned ep = static_cast<unsigned>(__double2hiint(p)) & 0x7FFFFFFFu;
+    const unsigned eh = static_cast<unsigned>(__double2hiint(h)) & 0x7FFFFFFFu;
+    const double a = eh > ep ? h : p, b = eh > ep ? p : h;  // exponent of a >= exponent of b
+    t = addr(a, b);
+    q = subr(b, subr(t, a));
+}
+
 template <typename R> struct Dot2 {
     R p, s;  // running sum of the rounded products; sum of the error terms
     __device__ __forceinline__ Dot2(R x, R y) {
@@ -351,9 +370,8 @@ template <typename R> struct Dot2 {
     __device__ __forceinline__ void add(R x, R y) {
         const R h = mulr(x, y);
         const R r = fmar(x, y, -h);  // x * y = h + r exactly
-        const R t = addr(p, h);
-        const R z = subr(t, p);
-        const R q = addr(subr(p, subr(t, z)), subr(h, z));  // p + h = t + q exactly
+        R t, q;
+        two_sum(p, h, t, q);
         p = t;
         s = addr(s, addr(q, r));
     }
