@@ -350,21 +350,24 @@ int super_tile(int esize) {
 }
 
 
-// Tile order in the target's own storage.  For a transposed problem (op = T
-// or C) the source tiles that warps read at the same time are scattered
-// across the source whatever the order, so the order serves the target,
-// which is read and written: each target buffer is walked in strips of
-// kLocalStrip tiles across its non-contiguous axis, each strip down the
-// buffer's contiguous axis, so that concurrent tiles form long contiguous
-// runs of target memory.  Measured on GB300: +6.6% on 16384^2 c128 (C) and
-// +2% on 8192^2 f64 (T); for 4-byte elements no gain on aligned layouts
-// (32 x 32 f32 tiles) and a loss when only the source is misaligned (B's
-// ld odd: 5350 -> 4786 GB/s), but +7 to +9% when most of the target runs
-// are misaligned (8192^2 f32 T copy, A's ld = 1 mod 4: 4305 -> 4696; both
-// lds odd 4371 -> 4678; BC50 -> BC75 +2%), where neighbouring tiles share
-// the partial sectors at their ends; a loss for op = N, whose source runs
-// the global order keeps.  The environment variable COSTA_TILE_ORDER (global |
-// local) overrides the rule, for tuning.
+// Tile order in the target's own storage: each target buffer is walked in
+// strips of kLocalStrip tiles across its non-contiguous axis, each strip
+// down the buffer's contiguous axis, so that concurrent tiles form long
+// contiguous runs of target memory (which is read and written; for a
+// transposed problem the source tiles read at the same time are scattered
+// whatever the order).  Measured on GB300, 8192^2 unless noted, GB/s:
+//  - 8- and 16-byte elements, every op: +6.6% on 16384^2 c128 (C), +2% on
+//    f64 (T); op = N: c128 copy BC64 -> BC128 5960 -> 6704, BC128 -> BC32
+//    6069 -> 6693, BC32 -> BC256 5962 -> 6350, f64 +1 to +4%, c64 0 to
+//    +1.5%;
+//  - 4-byte elements: no gain on aligned layouts (32 x 32 f32 tiles; c4
+//    -0.3%, f32 N BC16 -> BC64 -20%) and a loss when only the source is
+//    misaligned (B's ld odd: 5350 -> 4786), but +7 to +9% when most of the
+//    target runs are misaligned and op != N (f32 T copy, A's ld = 1 mod 4:
+//    4305 -> 4696; both lds odd 4371 -> 4678; BC50 -> BC75 +2%), where
+//    neighbouring tiles share the partial sectors at their ends.
+// The environment variable COSTA_TILE_ORDER (global | local) overrides the
+// rule, for tuning.
 constexpr int kLocalStrip = 2;
 
 bool use_local_order(const ProblemHost &ph, const TileDesc *tiles, size_t n) {
@@ -376,9 +379,9 @@ bool use_local_order(const ProblemHost &ph, const TileDesc *tiles, size_t n) {
         return -1;
     }();
     if (env >= 0) return env == 1;
-    if (ph.op == COSTA_OP_N) return false;
     const int es = esize_of(ph.A->dt);
-    return es >= 8 || mostly_misaligned(tiles, n, es, true);
+    if (es >= 8) return true;
+    return ph.op != COSTA_OP_N && mostly_misaligned(tiles, n, es, true);
 }
 
 // Stable LSD radix sort of (key, index) pairs by key, 11 bits per pass (the

@@ -126,10 +126,10 @@ def _tile_dst(p, rows, cols, u, v):
 
 
 def check_order(p):
-    """The kernel's tile order.  Transposed problems whose target tiles are
-    not each one contiguous run, of 8- and 16-byte elements or with tiles
-    whose target runs are misaligned holding at least half of the elements,
-    walk each target
+    """The kernel's tile order.  Problems whose target tiles are not each
+    one contiguous run, of 8- and 16-byte elements (every op) or transposed
+    with tiles whose target runs are misaligned holding at least half of the
+    elements, walk each target
     buffer in strips of 2 tiles (64 elements for 8-byte and 4-byte
     elements) across its non-contiguous axis, by address inside a strip, one
     target stride group after another; the others follow the global
@@ -161,7 +161,7 @@ def check_order(p):
     area = t["nx"].astype(np.int64) * t["ny"].astype(np.int64)
     a_mis = ((t["dst"] % 16) != 0) | ((t["dld"].astype(np.int64) * es) % 16 != 0) | (t["nx"] % (16 // es) != 0)
     mostly_mis = 2 * area[a_mis].sum() >= area.sum()
-    if p.op == "N" or (es < 8 and not mostly_mis) or contiguous:
+    if (es < 8 and (p.op == "N" or not mostly_mis)) or contiguous:
         assert np.array_equal(dst, want)
         return
     ld = t["dld"].astype(np.int64)
