@@ -21,10 +21,16 @@
 //      transform after receive).
 // If A and the source share their contiguous axis the staged rows are read
 // straight; otherwise they are read across rows (the transposing kernel of
-// Sec. 6).  Tiles whose runs
-// are not 16-byte aligned take the same pipeline in a second instance of the
-// kernel: over aligned 16-byte windows of their runs, or one element per
-// lane for the kinds that read A.
+// Sec. 6).  Tiles whose runs are not 16-byte aligned take the same pipeline
+// in a second instance of the kernel: over aligned 16-byte windows of their
+// runs, or one element per lane (the kinds that read A, and 4-byte tiles
+// whose target runs are misaligned).  A third instance stages the aligned
+// source tiles of one kind (f64, general beta) by TMA, and a separate
+// kernel moves lists of small tiles as grouped one-pass pieces.
+//
+// "alpha and beta as one fma" holds for real scalars; complex scalars take
+// a compensated evaluation per component (Dot2, or Kahan's algorithm for
+// the two-term components of double data), see combine_c.
 //
 // The kernel walks a list of tile descriptors (TileDesc) resolved on the host:
 // the direct list (every tile: B -> A), or the message path of Alg. 3 /
@@ -602,7 +608,7 @@ __device__ __forceinline__ void load_a(const Geom<T> &g, const Sc &s, Chunk<T> (
     if (KIND == K_AXPBY2) prescale<T>(av, npass, s);
 }
 
-// ---- TMA staging layout (COSTA_TMA=1; see tma.cpp) ----
+// ---- TMA staging layout (the f64 general-beta kind; every kind with COSTA_TMA=1; see tma.cpp) ----
 // A TMA-staged tile is boxes of 16 runs x 128 bytes: box (br, bl) (run / 16,
 // byte along the run / 128) at (br * TBL + bl) * 2048 bytes, 1024-byte
 // aligned, each a stack of 128-byte rows whose 16-byte chunks the TMA unit
@@ -707,13 +713,16 @@ __device__ __forceinline__ void tile_general(const Geom<T> &g, const Sc &s, unsi
 //
 // A tile whose runs do not start on 16-byte boundaries (an odd leading
 // dimension, a block at an odd offset) or whose extents are not whole chunks
-// takes one of two paths, by combine kind (measured on GB300: each is the
-// faster one for its kinds).
+// takes one of two paths (measured on GB300: each is the faster one where
+// it is used).
 //  - Kinds that do not read A move 16-byte chunks over each run's window
-//    (the aligned chunks that cover the run), like an aligned tile.
+//    (the aligned chunks that cover the run), like an aligned tile; 4-byte
+//    tiles whose target runs are misaligned (flag TF_ELEM, set by the host)
+//    take the element path instead.
 //  - Kinds that read A move one element per lane.
-// Both stage into the TS x CPR swizzled slots of an aligned tile's buffer
-// plus one extra column of TS chunks.
+// The window path stages into the TS x CPR swizzled slots of an aligned
+// tile's buffer plus one extra column of TS chunks, the element path into
+// TS x TS elements of the same buffer.
 
 // ---- 16-byte windows (kinds that do not read A) ----
 //
@@ -1367,7 +1376,7 @@ __global__ void __launch_bounds__(KCfg<T, KIND, MIS>::WARPS * 32, KCfg<T, KIND, 
     cp_async_wait<0>();
 }
 
-// ---- the TMA instance of the tile kernel (COSTA_TMA=1) ----
+// ---- the TMA instance of the tile kernel (tma.cpp decides which tiles it takes) ----
 //
 // The same pipeline as the tile kernel without look-ahead, with the source
 // staged by the TMA unit instead of per-lane cp.async copies: one lane

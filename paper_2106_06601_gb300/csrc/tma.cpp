@@ -1,5 +1,8 @@
 // TMA staging of the tile kernel's source tiles (cp.async.bulk.tensor), an
-// alternative to per-lane 16-byte cp.async copies, enabled with COSTA_TMA=1.
+// alternative to per-lane 16-byte cp.async copies: by default for the f64
+// general-beta kind (tma_policy_kinds), for every kind with COSTA_TMA=1,
+// for none with COSTA_TMA=0.  A plan's TMA lists are built by the first
+// call of a kind that uses them (costa.cpp, ensure_tma).
 //
 // A tensor map describes one 2-D surface of bytes: an allocation of device
 // memory viewed as columns of ld_bytes (a block's leading dimension times
