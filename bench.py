@@ -49,6 +49,7 @@ from workloads.materialize import DeviceMatrix, HostMatrix  # noqa: E402
 
 L2_BYTES = 129 * 1024 * 1024
 KERNEL_SOURCES = ["paper_2106_06601_gb300/csrc/remap_impl.cuh",
+                  "paper_2106_06601_gb300/csrc/fxdot.h",  # fixed-point sums of the complex kinds
                   "paper_2106_06601_gb300/csrc/remap_f64.cu",
                   "paper_2106_06601_gb300/csrc/remap_f32.cu",
                   "paper_2106_06601_gb300/csrc/remap_c64.cu",

@@ -548,6 +548,19 @@ costa_status costa_debug_exchange(costa_layout A, costa_layout B, costa_op op, i
  * two lists.  out: host, 6 int64.  Synchronizes the device. */
 costa_status costa_debug_tma(costa_layout A, costa_layout B, costa_op op, int64_t *out);
 
+/* Diagnostics (host only, no device work): the fixed-point sum of products
+ * that the remap kernels use for each component of alpha * op(B) + beta * A
+ * with complex scalars on double complex data (Eq. 1), evaluated on the host
+ * by the same code.  For each of `count` sets, out[k] = the sum over
+ * i < n of (-1)^neg[k n + i] x[k n + i] * y[k n + i], rounded once to
+ * double (within 0.5 ulp of the result plus n * 2^-7 ulp of the largest
+ * product of the exact sum); n is 2 or 4.  x, y, neg, out: host arrays.
+ * Every factor must be zero or of magnitude in [2^-480, 2^480), the range
+ * in which the kernels take this evaluation; COSTA_ERR_INVALID_ARG
+ * otherwise, with nothing written. */
+costa_status costa_debug_fxdot(int n, int64_t count, const double *x, const double *y, const int32_t *neg,
+                               double *out);
+
 /* Number of kernels this library has launched in this process. */
 int64_t costa_kernel_launch_count(void);
 

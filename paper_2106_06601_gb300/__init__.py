@@ -100,6 +100,7 @@ def _load():
         "costa_relabel_placement": [I, P, I, P, ctypes.c_double, P, P, P],
         "costa_debug_exchange": [P, P, I, I, P, I, ctypes.c_uint64, ctypes.c_uint64, I, P, I64, P, P],
         "costa_debug_tma": [P, P, I, P],
+        "costa_debug_fxdot": [I, I64, P, P, P, P],
     }
     for name, args in sigs.items():
         f = getattr(lib, name)
@@ -332,6 +333,20 @@ def costa_debug_tma(A: Layout, B: Layout, op: str) -> dict:
     _check(_lib.costa_debug_tma(A.handle, B.handle, OPS[op], _p(out)))
     return {"tiles": int(out[0]), "halves_tiles": int(out[1]), "maps": int(out[2]),
             "timeouts": int(out[3]), "kinds": int(out[4]), "halves_kinds": int(out[5])}
+
+
+def costa_debug_fxdot(x, y, neg) -> np.ndarray:
+    """out[k] = sum_i (-1)^neg[k, i] x[k, i] y[k, i] by the kernels' fixed-point
+    evaluation of complex-scalar components (host build); x, y, neg: [count, n]
+    with n = 2 or 4."""
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.ascontiguousarray(y, dtype=np.float64)
+    ng = np.ascontiguousarray(neg, dtype=np.int32)
+    if x.ndim != 2 or x.shape != y.shape or x.shape != ng.shape:
+        raise ValueError("x, y and neg must be [count, n] arrays of one shape")
+    out = np.empty(x.shape[0], np.float64)
+    _check(_lib.costa_debug_fxdot(x.shape[1], x.shape[0], _p(x), _p(y), _p(ng), _p(out)))
+    return out
 
 
 def costa_debug_exchange(A: Layout, B: Layout, op: str, G: int, place, g: int, send_base: int,

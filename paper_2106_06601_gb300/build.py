@@ -34,7 +34,7 @@ def _cuda_home() -> str:
 def sources():
     cu = sorted(f for f in os.listdir(CSRC) if f.endswith(".cu"))
     cpp = sorted(f for f in os.listdir(CSRC) if f.endswith(".cpp"))
-    hdr = sorted(f for f in os.listdir(CSRC) if f.endswith(".h"))
+    hdr = sorted(f for f in os.listdir(CSRC) if f.endswith((".h", ".cuh")))
     return cu, cpp, hdr
 
 

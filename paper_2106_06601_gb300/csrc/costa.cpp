@@ -21,6 +21,7 @@
 #include <cuda_runtime_api.h>
 
 #include "costa_internal.h"
+#include "fxdot.h"
 #include "plan_lists.h"
 #include "tiles.h"
 
@@ -1456,6 +1457,30 @@ costa_status costa_debug_tma(costa_layout A, costa_layout B, costa_op op, int64_
     out[5] = plan->direct_halves.ttiles == plan->direct.ttiles ? 0 : plan->direct_halves.tma_kinds;
     out[2] = static_cast<int64_t>(plan->tma_maps.size());
     out[3] = err;
+    return COSTA_OK;
+}
+
+costa_status costa_debug_fxdot(int n, int64_t count, const double *x, const double *y, const int32_t *neg,
+                               double *out) {
+    if ((n != 2 && n != 4) || count < 0 || (count > 0 && (!x || !y || !neg || !out)))
+        return fail(COSTA_ERR_INVALID_ARG, "costa_debug_fxdot: n must be 2 or 4 and the arrays non-null");
+    for (int64_t k = 0; k < count * n; ++k)
+        if (!fx::in_range(x[k]) || !fx::in_range(y[k]))
+            return fail(COSTA_ERR_INVALID_ARG, "costa_debug_fxdot: factor %lld is outside [2^-480, 2^480)",
+                        (long long)k);
+    for (int64_t k = 0; k < count; ++k) {
+        const double *xk = x + k * n, *yk = y + k * n;
+        const int32_t *nk = neg + k * n;
+        if (n == 2) {
+            const fx::Term t[2] = {fx::mul(fx::unpack(xk[0]), fx::unpack(yk[0]), nk[0] ? 1u : 0u),
+                                   fx::mul(fx::unpack(xk[1]), fx::unpack(yk[1]), nk[1] ? 1u : 0u)};
+            out[k] = fx::sum(t);
+        } else {
+            fx::Term t[4];
+            for (int i = 0; i < 4; ++i) t[i] = fx::mul(fx::unpack(xk[i]), fx::unpack(yk[i]), nk[i] ? 1u : 0u);
+            out[k] = fx::sum(t);
+        }
+    }
     return COSTA_OK;
 }
 

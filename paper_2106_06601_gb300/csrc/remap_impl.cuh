@@ -29,8 +29,9 @@
 // kernel moves lists of small tiles as grouped one-pass pieces.
 //
 // "alpha and beta as one fma" holds for real scalars; complex scalars take
-// a compensated evaluation per component (Dot2, or Kahan's algorithm for
-// the two-term components of double data), see combine_c.
+// a compensated evaluation per component (Dot2; for double data Kahan's
+// algorithm when a component has two terms, and a fixed-point sum on the
+// integer pipes when it has four), see combine_c.
 //
 // The kernel walks a list of tile descriptors (TileDesc) resolved on the host:
 // the direct list (every tile: B -> A), or the message path of Alg. 3 /
@@ -49,6 +50,7 @@
 #include <cstdint>
 
 #include "costa_internal.h"
+#include "fxdot.h"
 
 namespace costa {
 namespace remap {
@@ -79,7 +81,7 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 //            misaligned   axpby2 (one element per lane)   4      4     1
 //   16-byte  both         copy                            4      1     2
 //            both         scale                           4      3     1
-//            both         complex alpha, beta = 0         4      2     1
+//            both         complex alpha, beta = 0         4      3     1
 //            both         kinds that read A               4      2     1
 //
 // Why, where a row departs from its neighbours:
@@ -90,8 +92,11 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 //    -> 6204, N alpha=-0.7 5361 -> 6147 (the copy's rate) with two tiles
 //    ahead; c128 T 4410 -> 5853, N 4343 -> 5746 with 3 blocks.  c64
 //    (float multiplies) lost 11% with f64's shape and keeps the light one.
-//    c128 with a complex alpha (FP64-bound at 8 operations per element):
-//    T and N 1458 -> 2133 with 2 to 4 blocks.
+//    c128 with a complex alpha (FP64-bound at 8 operations per element
+//    with Kahan's algorithm alone): T and N 1458 -> 2133 with 2 to 4
+//    blocks; with every other element summed in fixed point on the integer
+//    pipes (COSTA_FX_CS_PERIOD) 2557 at 2 blocks, 2660 at 3 (one pass in 3 or 4
+//    in fixed point: 2553, 2569).
 //  - c64 complex scalars, against 3 blocks with 2 buffers: complex beta
 //    T 4484 -> 5482, N 4495 -> 5495 with 4 blocks and no look-ahead;
 //    complex alpha T 5551 -> 5955 with two tiles ahead; the real general
@@ -108,6 +113,10 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 //  - 8-byte element path (misaligned, kinds that read A): a whole tile of A
 //    in registers, which 4 blocks fit without spills.
 //  - 16-byte kinds that read A hold a whole 16 KB tile of A in registers.
+//    With a complex beta each component is a fixed-point sum on the integer
+//    pipes (498 GB/s with Dot2 on the FP64 pipe), evaluated COSTA_FX_GROUP
+//    passes at a time: 1105 -> 1186 GB/s with 2 (1194 with 4, 12 more
+//    registers).
 // Each entry is overridable at build time for tuning (COSTA_WARPS_4/8,
 // COSTA_MINB_* and COSTA_NBUF_*).
 #ifndef COSTA_WARPS_4
@@ -187,7 +196,7 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 #define COSTA_NBUF_16S 1
 #endif
 #ifndef COSTA_MINB_16CS
-#define COSTA_MINB_16CS 2
+#define COSTA_MINB_16CS 3
 #endif
 #ifndef COSTA_NBUF_16CS
 #define COSTA_NBUF_16CS 1
@@ -302,6 +311,7 @@ __device__ __forceinline__ double fmar(double a, double b, double c) { return __
 struct Sc {
     double ar, ai, br, bi;
     bool alpha_mid;      // both components of alpha zero or of magnitude in [2^-480, 2^480)
+    bool scal_mid;       // the same for alpha and beta
     uint32_t conj_mask;  // 0x80000000 flips the sign of b's imaginary part (op = C)
     int32_t bexp;        // |beta| = 2^bexp (K_AXPBY2)
     uint32_t bsign_hi;   // sign bit of beta in a high word (K_AXPBY2)
@@ -407,6 +417,61 @@ __device__ __forceinline__ double kahan2(double x, double y, double z, double t,
     return minus ? __dsub_rn(__fma_rn(x, y, -w), e) : __dadd_rn(__fma_rn(x, y, w), e);
 }
 
+// Passes of a tile that the drain of double complex data with complex
+// scalars evaluates together (stage_drain).
+#ifndef COSTA_FX_GROUP
+#define COSTA_FX_GROUP 2
+#endif
+// Passes that the drain of double complex data with a complex alpha and
+// beta = 0 evaluates together: the last in fixed point, the others by
+// Kahan's algorithm (0: every pass by Kahan's algorithm, one at a time).
+#ifndef COSTA_FX_CS_PERIOD
+#define COSTA_FX_CS_PERIOD 2
+#endif
+
+// Every operand of a double complex alpha * b + beta * a in the middle range
+// (b as it enters the combine, after any conjugation).
+__device__ __forceinline__ bool cplx_mid(const double2 &b, const double2 &a, const Sc &s) {
+    return s.scal_mid && mid_range(b.x) && mid_range(b.y) && mid_range(a.x) && mid_range(a.y);
+}
+template <typename C> __device__ __forceinline__ bool cplx_mid(const C &, const C &, const Sc &) {
+    return false;
+}
+
+// alpha * b + beta * a for double complex data and complex scalars, each
+// component the sum of its four products in fixed point on the integer pipes
+// (fxdot.h): within 0.5 ulp of the component plus 2^-5 ulp of its largest
+// product, with no FP64 operation.  Dot2 takes 24 FP64 operations per
+// component, and the FP64 pipe is narrow on GB300.  Every operand must be in
+// the middle range (cplx_mid).
+__device__ __forceinline__ double2 fx_cplx(const double2 &b, const double2 &a, const Sc &s) {
+    const fx::Op fbx = fx::unpack(b.x), fby = fx::unpack(b.y), fax = fx::unpack(a.x), fay = fx::unpack(a.y);
+    const fx::Op far = fx::unpack(s.ar), fai = fx::unpack(s.ai), fbr = fx::unpack(s.br), fbi = fx::unpack(s.bi);
+    // ar bx - ai by + br ax - bi ay;  ar by + ai bx + br ay + bi ax
+    const fx::Term re[4] = {fx::mul(far, fbx, 0u), fx::mul(fai, fby, 1u), fx::mul(fbr, fax, 0u),
+                            fx::mul(fbi, fay, 1u)};
+    const fx::Term im[4] = {fx::mul(far, fby, 0u), fx::mul(fai, fbx, 0u), fx::mul(fbr, fay, 0u),
+                            fx::mul(fbi, fax, 0u)};
+    double2 o;
+    o.x = fx::sum(re);
+    o.y = fx::sum(im);
+    return o;
+}
+
+// alpha * b for double complex data and a complex alpha, each component the
+// sum of its two products in fixed point on the integer pipes (fxdot.h).
+// Every operand must be in the middle range.
+__device__ __forceinline__ double2 fx_cscale(const double2 &b, const Sc &s) {
+    const fx::Op fbx = fx::unpack(b.x), fby = fx::unpack(b.y);
+    const fx::Op far = fx::unpack(s.ar), fai = fx::unpack(s.ai);
+    const fx::Term re[2] = {fx::mul(far, fbx, 0u), fx::mul(fai, fby, 1u)};  // ar bx - ai by
+    const fx::Term im[2] = {fx::mul(far, fby, 0u), fx::mul(fai, fbx, 0u)};  // ar by + ai bx
+    double2 o;
+    o.x = fx::sum(re);
+    o.y = fx::sum(im);
+    return o;
+}
+
 template <int KIND, typename C, typename R>
 __device__ __forceinline__ C combine_c(C b, C a, const Sc &s) {
     b.y = flip_sign(b.y, s.conj_mask);
@@ -425,6 +490,11 @@ __device__ __forceinline__ C combine_c(C b, C a, const Sc &s) {
             o.y = kahan2(s.ar, b.y, s.ai, b.x, false);  // ar by + ai bx
             return o;
         }
+    }
+    if constexpr (KIND == K_CPLX && sizeof(R) == 8) {
+        // four-term components: in fixed point on the integer pipes when
+        // every operand is in the middle range (fx_cplx)
+        if (cplx_mid(b, a, s)) return fx_cplx(b, a, s);
     }
     const R ar = R(s.ar), ai = R(s.ai);
     Dot2<R> re(ar, b.x), im(ar, b.y);
@@ -639,6 +709,60 @@ __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsig
     if (m.c >= chunks) return;
     const int x0 = m.c * C::VEC;
     const int npass = (g.ny + m.rpp - 1) / m.rpp;
+    if constexpr ((KIND == K_CPLX || (KIND == K_CSCALE && COSTA_FX_CS_PERIOD > 0)) && sizeof(T) == 16) {
+        // double complex with complex scalars: G passes at a time in
+        // straight-line code, so that their evaluations overlap.  Four-term
+        // components (complex beta) are all summed in fixed point on the
+        // integer pipes (about 150 instructions each, in long dependent
+        // chains); two-term ones (complex alpha, beta = 0) split the passes
+        // between Kahan's algorithm on the FP64 pipe and the fixed-point sum,
+        // so that both pipes work
+        constexpr int G = KIND == K_CPLX ? COSTA_FX_GROUP : COSTA_FX_CS_PERIOD;
+#pragma unroll
+        for (int p0 = 0; p0 < C::NPASS; p0 += G) {
+            if (p0 >= npass) break;  // uniform across the warp
+            T bb[G], aa[G];
+            bool ok[G];
+#pragma unroll
+            for (int j = 0; j < G; ++j) {
+                const int y = (p0 + j) * m.rpp + m.r0;
+                ok[j] = p0 + j < npass && y < g.ny;
+                bb[j] = ok[j] ? *reinterpret_cast<const T *>(slot_any<T, TL>(buf, g.transpose ? x0 : y,
+                                                                            g.transpose ? y : m.c))
+                              : T{0.0, 0.0};
+                bb[j].y = flip_sign(bb[j].y, s.conj_mask);
+                aa[j] = KIND == K_CPLX && ok[j] ? av[p0 + j].e[0] : T{0.0, 0.0};  // beta = 0: A unread
+            }
+            bool mid = KIND == K_CPLX || s.alpha_mid;
+#pragma unroll
+            for (int j = 0; j < G; ++j)
+                mid = mid && (KIND == K_CPLX ? cplx_mid(bb[j], aa[j], s) : mid_range(bb[j].x) && mid_range(bb[j].y));
+            T o[G];
+            if (mid) {
+#pragma unroll
+                for (int j = 0; j < G; ++j) {
+                    if (KIND == K_CPLX) {
+                        o[j] = fx_cplx(bb[j], aa[j], s);
+                    } else if (j == G - 1) {
+                        o[j] = fx_cscale(bb[j], s);
+                    } else {
+                        o[j].x = kahan2(s.ar, bb[j].x, s.ai, bb[j].y, true);   // ar bx - ai by
+                        o[j].y = kahan2(s.ar, bb[j].y, s.ai, bb[j].x, false);  // ar by + ai bx
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < G; ++j) {
+                    bb[j].y = flip_sign(bb[j].y, s.conj_mask);  // combine conjugates again
+                    o[j] = combine<KIND>(bb[j], aa[j], s);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < G; ++j)
+                if (ok[j]) *(g.dst + static_cast<int64_t>((p0 + j) * m.rpp + m.r0) * g.dld + x0) = o[j];
+        }
+        return;
+    }
 #pragma unroll
     for (int p = 0; p < C::NPASS; ++p) {
         if (p >= npass) break;  // uniform across the warp
@@ -998,6 +1122,7 @@ __device__ __forceinline__ void stage_drain_e1(const Geom<T> &g, const Sc &s, un
 __device__ __forceinline__ void make_sc(const Scalars &S, Sc &s) {
     s.ar = S.alpha[0]; s.ai = S.alpha[1]; s.br = S.beta[0]; s.bi = S.beta[1];
     s.alpha_mid = mid_range(S.alpha[0]) && mid_range(S.alpha[1]);
+    s.scal_mid = s.alpha_mid && mid_range(S.beta[0]) && mid_range(S.beta[1]);
     s.conj_mask = 0u;
     s.bexp = S.beta_exp;
     s.bsign_hi = static_cast<unsigned>(__double2hiint(S.beta[0])) & 0x80000000u;

@@ -92,13 +92,16 @@ def tolerance(dtype: str, alpha, beta, bvals, avals, want=None) -> np.ndarray:
 
     Complex scalars: M = the largest of the component's product terms
     (2 with beta = 0, 4 otherwise) and of the oracle's value `want`.  The
-    kernel evaluates each component with Dot2 (Ogita, Rump & Oishi 2005) in
-    the data's precision, within u|x| + gamma_4^2 * sum|terms| of the exact
-    value x; the oracle uses Dot2 for double data and, for float data, a
-    double sum of the exact products rounded once to float, within the same
-    bound.  The two differ by less than 2u|x| + 2 gamma_4^2 * 4M.  With
-    |x| <= M the first term is below 2 ulp(M) and the second below
-    2^-45 ulp(M) in double (2^-16 in float), so the test asserts 2 ulp(M).
+    oracle uses Dot2 (Ogita, Rump & Oishi 2005) for double data and, for
+    float data, a double sum of the exact products rounded once to float:
+    within u|x| + gamma_4^2 * sum|terms| of the exact value x.  The kernel
+    uses Dot2 in the data's precision (the same bound; the two differ by
+    less than 2u|x| + 2 gamma_4^2 * 4M, below 2 ulp(M) plus 2^-45 ulp(M) in
+    double and 2^-16 in float); for double data in the middle range
+    Kahan's algorithm for two terms (within 2u|x|, Jeannerod, Louvet &
+    Muller 2013) or a fixed-point sum on the integer pipes (within 0.5
+    ulp(x) + 2^-5 ulp(M), fxdot.h), both under 2 ulp(M) from the oracle.
+    The test asserts 2 ulp(M).
     Returned as (re_tol, im_tol) arrays (im_tol zero for real types).
     """
     alpha, beta = complex(alpha), complex(beta)

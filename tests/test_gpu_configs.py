@@ -167,6 +167,53 @@ def test_config_full_size(name, dev):
         mat.close()
 
 
+@pytest.mark.parametrize("name", ["zb", "za"])
+def test_complex_scalars_full_size(name, dev):
+    """c2's layouts with double complex data and complex scalars (zb: beta =
+    0.5 + 0.25i, four products per component; za: alpha = 0.3 - 0.4i, beta =
+    0, two), the kinds summed in fixed point on the integer pipes.  Every
+    element of A is compared with the oracle, row slab by row slab, within
+    2 ulp of the component's largest term; B must be bitwise unchanged."""
+    import paper_2106_06601_gb300 as costa
+    p = C.EXTRA_WORKLOADS[name]()
+    mat = Mat(p, dev)
+    try:
+        a_host, b_host = mat.Ad.download(), mat.Bd.download()
+        a_pre = a_host.arena.copy()
+        b_bits = bits(mat.Bd.arena).clone()
+        stream = torch.cuda.current_stream().cuda_stream
+        costa.costa_transform(mat.LA, mat.LB, p.op, p.alpha, p.beta, relabel=True, stream=stream)
+        torch.cuda.synchronize()
+        assert torch.equal(bits(mat.Bd.arena), b_bits), "B was modified"
+        del b_bits
+        got = mat.Ad.download().arena
+        oracle.transform(p.dtype, p.op, p.alpha, p.beta, p.A, a_host.buffers(), p.B, b_host.buffers())
+        want = a_host.arena
+        al, be = oracle.scalar(p.dtype, p.alpha), oracle.scalar(p.dtype, p.beta)
+        assert not exact_case(p.dtype, al, be)
+        rows = 256
+        for i0 in range(0, p.A.m, rows):
+            i1 = min(p.A.m, i0 + rows)
+            ii, jj = np.meshgrid(np.arange(i0, i1), np.arange(p.A.n), indexing="ij")
+            ij = np.stack([ii.ravel(), jj.ravel()], 1)
+            _, abuf, aoff = oracle.locate(p.A, ij)
+            _, bbuf, boff = oracle.locate(p.B, ij[:, ::-1].copy())
+            ia, ib = a_host.starts[abuf] + aoff, b_host.starts[bbuf] + boff
+            bvals = b_host.arena[ib].astype(np.complex128)
+            if p.op == "C":
+                bvals = np.conj(bvals)
+            assert_close(p.dtype, got[ia], want[ia], al, be, bvals, a_pre[ia], exact=False)
+        # padding and alignment gaps of A keep their values
+        covered = np.zeros(got.size, bool)
+        for i0 in range(0, p.A.m, 2048):
+            ii, jj = np.meshgrid(np.arange(i0, min(p.A.m, i0 + 2048)), np.arange(p.A.n), indexing="ij")
+            _, abuf, aoff = oracle.locate(p.A, np.stack([ii.ravel(), jj.ravel()], 1))
+            covered[a_host.starts[abuf] + aoff] = True
+        assert count_mismatches(got[~covered], a_pre[~covered]) == 0
+    finally:
+        mat.close()
+
+
 def test_config_c3_volume_matches_oracle_count(dev):
     """c3's irregular target grid has no closed form: compare V with the
     oracle's element-by-element count."""

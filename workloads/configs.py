@@ -171,8 +171,23 @@ def odd_blocks(n: int = 8192, dtype: str = "f64") -> Problem:
     return Problem("odd", dtype, "T", 1.0, 0.0, A, B, "uniform", "nan", _seed(7))
 
 
+def c2_complex_scalars(n: int = 8192, complex_beta: bool = True) -> Problem:
+    """c2's layouts and op with double complex data and complex scalars:
+    alpha = 1, beta = 0.5 + 0.25i (every component a sum of four products)
+    or alpha = 0.3 - 0.4i, beta = 0 (two products; A is not read).  The
+    kinds whose arithmetic, not memory, sets the rate.  Not configurations."""
+    p = c2(n)
+    p.dtype = "c128"
+    if complex_beta:
+        p.name, p.alpha, p.beta = "zb", 1.0, complex(0.5, 0.25)
+    else:
+        p.name, p.alpha, p.beta, p.a_kind = "za", complex(0.3, -0.4), 0.0, "nan"
+    return p
+
+
 EXTRA_WORKLOADS = {"bc8": small_blocks, "c5b": c5b, "c2g": c2_general_beta,
-                   "ld1": f32_lld, "ld0": lambda: f32_lld(pad=0), "odd": odd_blocks}
+                   "ld1": f32_lld, "ld0": lambda: f32_lld(pad=0), "odd": odd_blocks,
+                   "zb": c2_complex_scalars, "za": lambda: c2_complex_scalars(complex_beta=False)}
 
 # The same layouts and tile shapes at about 1 GB on the device, for profiler
 # captures (the workloads proper stay the ones above).
@@ -180,7 +195,8 @@ CONFIGS_SMALL = {"c1": c1, "c2": lambda: c2(4096), "c3": lambda: c3(8192),
                  "c4": lambda: c4(16), "c5": lambda: c5(rows=16384), "bc8": lambda: small_blocks(4096),
                  "c2g": lambda: c2_general_beta(4096),
                  "ld1": lambda: f32_lld(8192), "ld0": lambda: f32_lld(8192, 0), "odd": lambda: odd_blocks(4096),
-                 "c5b": lambda: c5b(rows=16384)}
+                 "c5b": lambda: c5b(rows=16384), "zb": lambda: c2_complex_scalars(4096),
+                 "za": lambda: c2_complex_scalars(4096, complex_beta=False)}
 
 WORKLOAD_TEXT = {
     "c1": "256x256 f64 BC16 2x2R -> BC32 2x2C, N, alpha=1 beta=0, P=4",
@@ -200,6 +216,10 @@ WORKLOAD_TEXT = {
            "not a configuration)",
     "odd": "8192x8192 f64 BC50 4x4 -> BC75 4x4, T, alpha=1 beta=0, P=16 (odd block sizes; "
            "not a configuration)",
+    "zb": "8192x8192 c128 BC64 4x4 -> BC128 4x4 permuted owners, T, alpha=1 beta=0.5+0.25i, P=16 "
+          "(complex beta: four products per component; not a configuration)",
+    "za": "8192x8192 c128 BC64 4x4 -> BC128 4x4 permuted owners, T, alpha=0.3-0.4i beta=0, P=16 "
+          "(complex alpha: two products per component; not a configuration)",
 }
 
 
