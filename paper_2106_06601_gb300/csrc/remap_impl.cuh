@@ -95,8 +95,9 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 //    c128 with a complex alpha (FP64-bound at 8 operations per element
 //    with Kahan's algorithm alone): T and N 1458 -> 2133 with 2 to 4
 //    blocks; with every other element summed in fixed point on the integer
-//    pipes (COSTA_FX_CS_PERIOD) 2557 at 2 blocks, 2660 at 3 (one pass in 3 or 4
-//    in fixed point: 2553, 2569).
+//    pipes (COSTA_FX_CS_PERIOD), unrolled, 2557 at 2 blocks, 2660 at 3 (one
+//    pass in 3 or 4 in fixed point: 2553, 2569); in the rolled loop, 3 blocks,
+//    3259.
 //  - c64 complex scalars, against 3 blocks with 2 buffers: complex beta
 //    T 4484 -> 5482, N 4495 -> 5495 with 4 blocks and no look-ahead;
 //    complex alpha T 5551 -> 5955 with two tiles ahead; the real general
@@ -112,11 +113,14 @@ template <> struct ET<double2> { enum { VEC = 1, CPLX = 1 }; typedef double R; }
 //    warps per SM leave exposed; 4 buffers lost 20-40%.
 //  - 8-byte element path (misaligned, kinds that read A): a whole tile of A
 //    in registers, which 4 blocks fit without spills.
-//  - 16-byte kinds that read A hold a whole 16 KB tile of A in registers.
-//    With a complex beta each component is a fixed-point sum on the integer
-//    pipes (498 GB/s with Dot2 on the FP64 pipe), evaluated COSTA_FX_GROUP
-//    passes at a time: 1105 -> 1186 GB/s with 2 (1194 with 4, 12 more
-//    registers).
+//  - 16-byte kinds that read A hold a whole 16 KB tile of A in registers,
+//    except with a complex beta: there each component is a fixed-point sum
+//    on the integer pipes (498 GB/s with Dot2 on the FP64 pipe), and the
+//    drain is a rolled loop over COSTA_FX_GROUP passes at a time that loads
+//    A two groups ahead (unrolled with A's tile in registers: 1105 one pass
+//    at a time, 1186 with 2, 1194 with 4, instruction fetch the limit;
+//    rolled: 2286 with 1, 2340 with 2 at 136 registers and 3 blocks, 2115
+//    with 4).
 // Each entry is overridable at build time for tuning (COSTA_WARPS_4/8,
 // COSTA_MINB_* and COSTA_NBUF_*).
 #ifndef COSTA_WARPS_4
@@ -699,6 +703,13 @@ __device__ __forceinline__ unsigned char *slot_any(unsigned char *buf, int r, in
     else return slot<T>(buf, r, c);
 }
 
+// The drain of double complex data with a complex beta loads A itself, a
+// few passes ahead (stage_drain); for the other kinds that read A the
+// caller loads the tile's A chunks into registers first (load_a).
+template <typename T, int KIND> __host__ __device__ constexpr bool drain_loads_a() {
+    return KIND == K_CPLX && sizeof(T) == 16;
+}
+
 // Write a staged fast tile to A, combining with A when the kind reads it.
 template <typename T, int KIND, bool TL = false>
 __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsigned char *buf,
@@ -716,12 +727,34 @@ __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsig
         // integer pipes (about 150 instructions each, in long dependent
         // chains); two-term ones (complex alpha, beta = 0) split the passes
         // between Kahan's algorithm on the FP64 pipe and the fixed-point sum,
-        // so that both pipes work
+        // so that both pipes work.  The loop stays rolled: unrolled over the
+        // tile's passes, the fixed-point sums made a body of about 14,000
+        // instructions, and instruction fetch stalled the warps.  So A is
+        // not held as a whole tile in registers (av is unused here; the
+        // callers do not load it for this kind): each iteration loads the A
+        // chunks of the group two ahead of the one it combines.
         constexpr int G = KIND == K_CPLX ? COSTA_FX_GROUP : COSTA_FX_CS_PERIOD;
+        T a_next[2][G];
+        auto load_group = [&](int q0, T (&dst)[G]) {
 #pragma unroll
-        for (int p0 = 0; p0 < C::NPASS; p0 += G) {
-            if (p0 >= npass) break;  // uniform across the warp
+            for (int j = 0; j < G; ++j) {
+                const int y = (q0 + j) * m.rpp + m.r0;
+                dst[j] = T{0.0, 0.0};
+                if (KIND == K_CPLX && q0 + j < npass && y < g.ny)
+                    dst[j] = load_rw(g.dst + static_cast<int64_t>(y) * g.dld + x0).e[0];
+            }
+        };
+        load_group(0, a_next[0]);
+        load_group(G, a_next[1]);
+#pragma unroll 1
+        for (int p0 = 0; p0 < npass; p0 += G) {
             T bb[G], aa[G];
+#pragma unroll
+            for (int j = 0; j < G; ++j) {
+                aa[j] = a_next[0][j];
+                a_next[0][j] = a_next[1][j];
+            }
+            load_group(p0 + 2 * G, a_next[1]);
             bool ok[G];
 #pragma unroll
             for (int j = 0; j < G; ++j) {
@@ -731,7 +764,6 @@ __device__ __forceinline__ void stage_drain(const Geom<T> &g, const Sc &s, unsig
                                                                             g.transpose ? y : m.c))
                               : T{0.0, 0.0};
                 bb[j].y = flip_sign(bb[j].y, s.conj_mask);
-                aa[j] = KIND == K_CPLX && ok[j] ? av[p0 + j].e[0] : T{0.0, 0.0};  // beta = 0: A unread
             }
             bool mid = KIND == K_CPLX || s.alpha_mid;
 #pragma unroll
@@ -1427,7 +1459,7 @@ __device__ __forceinline__ void write_tile(const RemapLaunch &a, const Geom<T> &
         else stage_drain_w<T, KIND>(g, s, buf, lane);
     } else if (g.fast) {
         Chunk<T> av[C::NPASS];
-        load_a<T, KIND>(g, s, av, lane);
+        if constexpr (!drain_loads_a<T, KIND>()) load_a<T, KIND>(g, s, av, lane);
         cp_async_wait<NB - 1>();
         __syncwarp();
         stage_drain<T, KIND>(g, s, buf, av, lane);
@@ -1619,7 +1651,7 @@ __global__ void __launch_bounds__(Cfg<T>::WARPS * 32, TmaKCfg<T, KIND>::MINB)
         }
         s.conj_mask = g.conj ? 0x80000000u : 0u;
         Chunk<T> av[C::NPASS];
-        load_a<T, KIND>(g, s, av, lane);
+        if constexpr (!drain_loads_a<T, KIND>()) load_a<T, KIND>(g, s, av, lane);
         if (!mbar_wait(bar, parity)) {
             if (lane == 0) atomicAdd(p.err, 1u);
             mbar_wait(bar, parity);
