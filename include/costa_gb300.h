@@ -47,11 +47,18 @@
  *  - Arithmetic (Eq. 1): with real alpha and beta each element, or each
  *    component of a complex element, is fma(alpha, b, beta * a) in the
  *    element type's precision (alpha * b when beta == 0, b when also
- *    alpha == 1).  With a complex alpha or beta each component is the
- *    compensated dot product Dot2 (Ogita, Rump & Oishi 2005) of its 2
- *    (beta == 0) or 4 products: as if evaluated in twice the precision and
- *    rounded once.  When beta == 0, A is never read, so NaN or garbage in A
- *    does not propagate.
+ *    alpha == 1).  With a complex alpha or beta each component, the sum of
+ *    its 2 (beta == 0) or 4 products, is evaluated so that it lies within
+ *    2 ulp of the largest product (or of the result, if larger) of the
+ *    exactly rounded value: by the compensated dot product Dot2 (Ogita,
+ *    Rump & Oishi 2005) for single-precision data; for double-precision
+ *    data whose operands are all zero or of magnitude in [2^-480, 2^480),
+ *    by an exact fixed-point sum on the integer pipes rounded once (every
+ *    four-product component, every other element of two-product ones)
+ *    and by Kahan's algorithm for 2 x 2 determinants (the other
+ *    two-product ones); Dot2 otherwise.  Repeated calls on one pair give
+ *    the same bits.  When beta == 0, A is never read, so NaN or garbage in
+ *    A does not propagate.
  */
 #ifndef COSTA_GB300_H
 #define COSTA_GB300_H
