@@ -116,3 +116,37 @@ def test_fxdot_agrees_with_the_oracle_combine(alpha, beta):
     got = (costa.costa_debug_fxdot(re_x, re_y, re_n) + 1j * costa.costa_debug_fxdot(im_x, im_y, im_n))
     from tests._util import assert_close
     assert_close("c128", got, want, al, be, b, a, exact=False)
+
+
+def test_fxdot_property_against_exact_rationals():
+    """Random factors anywhere in the admitted range, drawn by hypothesis
+    (where installed): the bound of the exact-sum test holds."""
+    hyp = pytest.importorskip("hypothesis")
+    st = hyp.strategies
+
+    def in_range(v):
+        return v == 0 or 2.0 ** -480 <= abs(v) < 2.0 ** 480
+
+    factor = st.floats(min_value=-(2.0 ** 479), max_value=2.0 ** 479, allow_nan=False,
+                       allow_infinity=False).filter(in_range)
+
+    @hyp.settings(max_examples=3000, deadline=None, derandomize=True)
+    @hyp.given(st.sampled_from([2, 4]).flatmap(
+        lambda n: st.tuples(st.lists(factor, min_size=n, max_size=n), st.lists(factor, min_size=n, max_size=n),
+                            st.lists(st.integers(0, 1), min_size=n, max_size=n))))
+    def check(case):
+        xs, ys, ns = case
+        got = costa.costa_debug_fxdot(np.array([xs]), np.array([ys]), np.array([ns], np.int32))[0]
+        prods = [Fraction(x) * Fraction(y) * (-1 if k else 1) for x, y, k in zip(xs, ys, ns)]
+        exact = sum(prods)
+        M = max(abs(p) for p in prods)
+        if M == 0:
+            assert got == 0.0
+            return
+        n = len(xs)
+        ulp_m = Fraction(math.ulp(float(M)))
+        rounded = float(exact)
+        bound = n * ulp_m / 128 + (Fraction(math.ulp(rounded)) / 2 if rounded else 0)
+        assert abs(Fraction(float(got)) - exact) <= bound
+
+    check()
